@@ -1,0 +1,308 @@
+/*
+ * nmv_oracle.c -- plain, slow, single-threaded CPU oracle for numerical
+ * validation with failure forensics.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the
+ * benchmark's CPU-baseline leg may load this library.  The product path
+ * (the CUDA library and its Python binding) never calls it, includes it or
+ * shares a line of code, a header or a table with it.
+ *
+ * What it computes comes from the paper's problem statement (Section 3.2,
+ * Eq. 1 and the constraint Validate(K_fixed, R, T_ext, tau) = true): a
+ * candidate output is checked against a reference output within a numerical
+ * tolerance tau, and the diagnostic evidence D given to the repair agent
+ * includes "numerical-deviation metrics" (Section 3.2).  The paper gives no
+ * formula for the check, so every definition below is a written-out reading:
+ *
+ *   P1 pass predicate (allclose form, equal_nan = false), per element i,
+ *      after widening both stored values to fp64 exactly:
+ *         pass(i) = (c == r)  OR  (c, r finite AND
+ *                   fl(|fl(c - r)|) <= fl(atol + fl(rtol * |r|)))
+ *      NaN never passes; an infinity passes only against the same infinity.
+ *   P2 counts: mismatch = #!pass; NaN/+Inf/-Inf counts of c and of r;
+ *      n_finite_pairs = #{both finite}.  The match rate of Table S4 /
+ *      Section 4.3 ("per-case pass/fail, numerical match rates") is
+ *      (numel - mismatch) / numel.
+ *   P3 error statistics over the both-finite set: d = fl(c - r), a = |d|,
+ *      max a with the lowest index attaining it; rel = fl(a / |r|) for r != 0,
+ *      max rel with the lowest index; sse = sum of fl(d * d) accumulated with
+ *      Neumaier's compensated summation (Neumaier 1974).  No eligible
+ *      element: max = 0.0, argmax = -1.
+ *   P4 localisation (the "localize" step of the forensics, Section 4.2 and
+ *      S2.2): 2-D view [M = prod(shape[:-1]), N = shape[-1]], row = i / N,
+ *      col = i % N; for every mismatch tile_hist[(row/th)*GC + col/tw] += 1,
+ *      row_prof[row % th] += 1, col_prof[col % tw] += 1.
+ *   P5 first-K: the K lowest mismatching linear indices in ascending order,
+ *      each with c and r widened to fp64.
+ *   P6 degenerate-output flags (the "repair by degeneration" and bypass
+ *      hazards, Sections 1, 2.2 and 4.3): see oracle_validate below.
+ *
+ * Build: gcc -std=c11 -O2 -ffp-contract=off -fPIC -shared (no FMA
+ * contraction: every rounding above happens exactly where it is written).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+enum { OR_F32 = 0, OR_F16 = 1, OR_BF16 = 2, OR_I32 = 3 };
+
+/* Flag bits of the degenerate-output mask (interface format). */
+#define OR_FLAG_CAND_EQ_INPUT 1u
+#define OR_FLAG_CAND_ALL_ZERO 2u
+#define OR_FLAG_CAND_CONSTANT 4u
+#define OR_FLAG_REF_ALL_ZERO 8u
+#define OR_FLAG_REF_CONSTANT 16u
+
+/* ---- decoders: stored bit pattern -> exact fp64 value ------------------ */
+
+/* IEEE 754 binary16: 1 sign bit, 5 exponent bits (bias 15), 10 fraction. */
+double oracle_decode_f16(uint32_t bits)
+{
+    uint32_t sign = (bits >> 15) & 1u;
+    uint32_t expo = (bits >> 10) & 31u;
+    uint32_t frac = bits & 1023u;
+    double v;
+    if (expo == 0) {
+        v = ldexp((double)frac, -24); /* subnormal: frac * 2^(1-15-10) */
+    } else if (expo == 31) {
+        v = (frac == 0) ? INFINITY : NAN;
+    } else {
+        v = ldexp((double)(1024u + frac), (int)expo - 25);
+    }
+    return sign ? -v : v;
+}
+
+/* bfloat16: 1 sign bit, 8 exponent bits (bias 127), 7 fraction bits. */
+double oracle_decode_bf16(uint32_t bits)
+{
+    uint32_t sign = (bits >> 15) & 1u;
+    uint32_t expo = (bits >> 7) & 255u;
+    uint32_t frac = bits & 127u;
+    double v;
+    if (expo == 0) {
+        v = ldexp((double)frac, -133); /* subnormal: frac * 2^(1-127-7) */
+    } else if (expo == 255) {
+        v = (frac == 0) ? INFINITY : NAN;
+    } else {
+        v = ldexp((double)(128u + frac), (int)expo - 134);
+    }
+    return sign ? -v : v;
+}
+
+/* IEEE 754 binary32: 1 sign bit, 8 exponent bits (bias 127), 23 fraction. */
+double oracle_decode_f32(uint32_t bits)
+{
+    uint32_t sign = bits >> 31;
+    uint32_t expo = (bits >> 23) & 255u;
+    uint32_t frac = bits & 0x7fffffu;
+    double v;
+    if (expo == 0) {
+        v = ldexp((double)frac, -149);
+    } else if (expo == 255) {
+        v = (frac == 0) ? INFINITY : NAN;
+    } else {
+        v = ldexp((double)(0x800000u + frac), (int)expo - 150);
+    }
+    return sign ? -v : v;
+}
+
+static int elem_size(int dtype)
+{
+    return (dtype == OR_F16 || dtype == OR_BF16) ? 2 : 4;
+}
+
+/* Raw stored bit pattern of element i (zero-extended to 32 bits). */
+static uint32_t load_bits(const void *p, int dtype, int64_t i)
+{
+    if (elem_size(dtype) == 2) {
+        uint16_t h;
+        memcpy(&h, (const char *)p + 2 * i, 2);
+        return h;
+    }
+    uint32_t w;
+    memcpy(&w, (const char *)p + 4 * i, 4);
+    return w;
+}
+
+static double decode(uint32_t bits, int dtype)
+{
+    switch (dtype) {
+    case OR_F32: return oracle_decode_f32(bits);
+    case OR_F16: return oracle_decode_f16(bits);
+    case OR_BF16: return oracle_decode_bf16(bits);
+    default: return (double)(int32_t)bits;
+    }
+}
+
+/* P1: the pass predicate, exactly as written (no contraction). */
+int oracle_pass(double c, double r, double rtol, double atol)
+{
+    if (c == r) return 1;
+    if (!isfinite(c) || !isfinite(r)) return 0;
+    double diff = c - r;
+    double err = fabs(diff);
+    double scaled = rtol * fabs(r);
+    double allowed = atol + scaled;
+    return err <= allowed;
+}
+
+/*
+ * Validate one candidate/reference pair.
+ *
+ *   cand, ref      host buffers of numel elements of `dtype`, row-major.
+ *   ncols          N = the last dimension (the 2-D view is [numel/N, N]);
+ *                  for numel == 0 any value >= 1 is accepted.
+ *   inputs[j]      optional operator inputs with input_dtype[j] and
+ *                  input_numel[j]; only those with the candidate's dtype and
+ *                  numel take part in the pass-through check.
+ *
+ * Outputs (all caller-allocated):
+ *   counts[9]   mismatch, cand_nan, cand_posinf, cand_neginf, ref_nan,
+ *               ref_posinf, ref_neginf, n_finite_pairs, k_out
+ *   fstats[3]   max_abs, max_rel, sse
+ *   argmax[2]   argmax_abs, argmax_rel
+ *   tile_hist[GR*GC], row_prof[th], col_prof[tw]   (zeroed here)
+ *   fk_index[K], fk_cand[K], fk_ref[K]
+ *   input_eq[n_inputs]   pass-through count, or -1 when not eligible
+ *   flags[1], passthrough[1]
+ *
+ * P6, the degenerate-output flags (our reading; the paper implements its
+ * anti-cheat check on source code and gives no numeric rule):
+ *   input_eq[j] = #{i : bits(c_i) == bits(x_ij) and bits(r_i) != bits(x_ij)}
+ *   CAND_EQ_INPUT  some eligible j has input_eq[j] >= max(1, ceil(numel/100))
+ *   CAND_ALL_ZERO  numel >= 1 and every c_i == 0 by value (+0 and -0)
+ *   CAND_CONSTANT  numel >= 2 and every bits(c_i) == bits(c_0)
+ *   REF_ALL_ZERO, REF_CONSTANT  the same two rules applied to r
+ *   passthrough = the lowest flagged j, else -1.
+ */
+int oracle_validate(const void *cand, const void *ref, int dtype, int64_t numel,
+                    int64_t ncols, int n_inputs, const void *const *inputs,
+                    const int *input_dtype, const int64_t *input_numel,
+                    double rtol, double atol, int64_t tile_rows,
+                    int64_t tile_cols, int64_t first_k, int64_t *counts,
+                    double *fstats, int64_t *argmax, int64_t *tile_hist,
+                    int64_t *row_prof, int64_t *col_prof, int64_t *fk_index,
+                    double *fk_cand, double *fk_ref, int64_t *input_eq,
+                    uint32_t *flags, int32_t *passthrough)
+{
+    if (ncols < 1 || tile_rows < 1 || tile_cols < 1 || first_k < 0) return -1;
+    if (n_inputs < 0 || n_inputs > 64) return -1;
+    int64_t nrows = numel / ncols;
+    int64_t grid_rows = (nrows + tile_rows - 1) / tile_rows;
+    int64_t grid_cols = (ncols + tile_cols - 1) / tile_cols;
+    if (numel == 0) grid_rows = grid_cols = 0;
+
+    for (int64_t t = 0; t < grid_rows * grid_cols; ++t) tile_hist[t] = 0;
+    for (int64_t t = 0; t < tile_rows; ++t) row_prof[t] = 0;
+    for (int64_t t = 0; t < tile_cols; ++t) col_prof[t] = 0;
+
+    int64_t mismatch = 0, cand_nan = 0, cand_posinf = 0, cand_neginf = 0;
+    int64_t ref_nan = 0, ref_posinf = 0, ref_neginf = 0, n_finite = 0;
+    int64_t k_out = 0;
+    double max_abs = 0.0, max_rel = 0.0;
+    int64_t arg_abs = -1, arg_rel = -1;
+    double sse_sum = 0.0, sse_comp = 0.0; /* Neumaier: running sum + correction */
+
+    int eligible[64];
+    for (int j = 0; j < n_inputs; ++j) {
+        eligible[j] = (input_dtype[j] == dtype && input_numel[j] == numel);
+        input_eq[j] = eligible[j] ? 0 : -1;
+    }
+
+    int cand_all_zero = 1, cand_constant = 1, ref_all_zero = 1, ref_constant = 1;
+    uint32_t c0 = 0, r0 = 0;
+    if (numel > 0) {
+        c0 = load_bits(cand, dtype, 0);
+        r0 = load_bits(ref, dtype, 0);
+    }
+
+    for (int64_t i = 0; i < numel; ++i) {
+        uint32_t cb = load_bits(cand, dtype, i);
+        uint32_t rb = load_bits(ref, dtype, i);
+        double c = decode(cb, dtype);
+        double r = decode(rb, dtype);
+
+        /* P2: classes of each side. */
+        if (isnan(c)) cand_nan++;
+        else if (isinf(c)) { if (c > 0) cand_posinf++; else cand_neginf++; }
+        if (isnan(r)) ref_nan++;
+        else if (isinf(r)) { if (r > 0) ref_posinf++; else ref_neginf++; }
+
+        /* P1 + P4 + P5 */
+        if (!oracle_pass(c, r, rtol, atol)) {
+            mismatch++;
+            int64_t row = i / ncols;
+            int64_t col = i % ncols;
+            tile_hist[(row / tile_rows) * grid_cols + col / tile_cols] += 1;
+            row_prof[row % tile_rows] += 1;
+            col_prof[col % tile_cols] += 1;
+            if (k_out < first_k) {
+                fk_index[k_out] = i;
+                fk_cand[k_out] = c;
+                fk_ref[k_out] = r;
+                k_out++;
+            }
+        }
+
+        /* P3 over the both-finite set, in ascending index order. */
+        if (isfinite(c) && isfinite(r)) {
+            n_finite++;
+            double d = c - r;
+            double a = fabs(d);
+            if (arg_abs < 0 || a > max_abs) { max_abs = a; arg_abs = i; }
+            if (r != 0.0) {
+                double rel = a / fabs(r);
+                if (arg_rel < 0 || rel > max_rel) { max_rel = rel; arg_rel = i; }
+            }
+            double term = d * d;
+            double t = sse_sum + term;
+            if (fabs(sse_sum) >= fabs(term)) sse_comp += (sse_sum - t) + term;
+            else sse_comp += (term - t) + sse_sum;
+            sse_sum = t;
+        }
+
+        /* P6 */
+        if (!(c == 0.0)) cand_all_zero = 0;
+        if (!(r == 0.0)) ref_all_zero = 0;
+        if (cb != c0) cand_constant = 0;
+        if (rb != r0) ref_constant = 0;
+        for (int j = 0; j < n_inputs; ++j) {
+            if (!eligible[j]) continue;
+            uint32_t xb = load_bits(inputs[j], dtype, i);
+            if (cb == xb && rb != xb) input_eq[j] += 1;
+        }
+    }
+
+    uint32_t f = 0;
+    int32_t pt = -1;
+    int64_t threshold = (numel + 99) / 100; /* ceil(numel / 100) */
+    if (threshold < 1) threshold = 1;
+    for (int j = 0; j < n_inputs; ++j) {
+        if (eligible[j] && input_eq[j] >= threshold) {
+            f |= OR_FLAG_CAND_EQ_INPUT;
+            if (pt < 0) pt = j;
+        }
+    }
+    if (numel >= 1 && cand_all_zero) f |= OR_FLAG_CAND_ALL_ZERO;
+    if (numel >= 2 && cand_constant) f |= OR_FLAG_CAND_CONSTANT;
+    if (numel >= 1 && ref_all_zero) f |= OR_FLAG_REF_ALL_ZERO;
+    if (numel >= 2 && ref_constant) f |= OR_FLAG_REF_CONSTANT;
+
+    counts[0] = mismatch;
+    counts[1] = cand_nan;
+    counts[2] = cand_posinf;
+    counts[3] = cand_neginf;
+    counts[4] = ref_nan;
+    counts[5] = ref_posinf;
+    counts[6] = ref_neginf;
+    counts[7] = n_finite;
+    counts[8] = k_out;
+    fstats[0] = max_abs;
+    fstats[1] = max_rel;
+    fstats[2] = sse_sum + sse_comp;
+    argmax[0] = arg_abs;
+    argmax[1] = arg_rel;
+    flags[0] = f;
+    passthrough[0] = pt;
+    return 0;
+}
