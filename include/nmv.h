@@ -1,0 +1,174 @@
+/*
+ * nmv.h -- numerical validation with failure forensics on one NVIDIA GB300
+ * (sm_103a).  C ABI of libnmv.so.
+ *
+ * The operation is the engine's validation step of the paper (Section 3.2,
+ * Eq. 1: a repaired operator must satisfy Validate(K_fixed, R, T_ext, tau) =
+ * true, i.e. its outputs must match the reference outputs within the
+ * numerical tolerance tau over the extended test suite), together with the
+ * numerical-deviation evidence the engine hands to the repair agent (Section
+ * 3.2, "numerical-deviation metrics"; Section 4.2, localisation of diffuse
+ * deviation; S2.2, NaN/Inf forensics), the per-case pass/fail and match-rate
+ * evidence of full-coverage evaluation (Section 4.3, Table S4 "x% matched
+ * cases"), and value-level flags for the degeneration / bypass hazards the
+ * integrity layer guards against (Sections 1, 2.2, 4.3).
+ *
+ * The paper gives no formula for the check.  This library implements the
+ * following reading (the same one the CPU oracle of the test suite writes
+ * out), element by element after widening both stored values to fp64
+ * exactly:
+ *
+ *   pass(i) = (c == r) OR (c, r finite AND
+ *             fl(|fl(c - r)|) <= fl(atol + fl(rtol * |r|)))
+ *
+ * so NaN never passes and an infinity passes only against the same infinity.
+ * Results are bit-identical to that fp64 arithmetic (the sum of squared
+ * errors to a relative 1e-9), and bit-identical from run to run.
+ *
+ * Threading: every entry point may be called from any host thread; calls
+ * are serialised on an internal lock (the device workspace is shared).
+ */
+#ifndef NMV_H
+#define NMV_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- limits ------------------------------------------------------------ */
+#define NMV_MAX_RANK 8
+#define NMV_MAX_INPUTS 8
+#define NMV_MAX_TILE (1LL << 24)      /* tile_rows, tile_cols <= this        */
+#define NMV_MAX_HIST_BINS (1LL << 26) /* grid_rows * grid_cols <= this       */
+#define NMV_MAX_FIRST_K (1LL << 24)   /* first_k <= this                     */
+#define NMV_MAX_CASES (1LL << 20)     /* cases per nmv_validate_batch call   */
+
+/* ---- status codes (return values and nmv_result.status) --------------- */
+#define NMV_OK 0
+#define NMV_EINVAL (-1)       /* an argument breaks a rule stated here      */
+#define NMV_ENOMEM (-2)       /* host or device allocation failed           */
+#define NMV_ECUDA (-3)        /* a CUDA call failed (no device, bad stream,
+                                 a kernel error); see nmv_last_error()      */
+#define NMV_EUNSUPPORTED (-4) /* the device is not sm_103                   */
+
+/* ---- element types ----------------------------------------------------- */
+typedef enum nmv_dtype {
+    NMV_F32 = 0,  /* IEEE binary32                                        */
+    NMV_F16 = 1,  /* IEEE binary16                                        */
+    NMV_BF16 = 2, /* bfloat16                                             */
+    NMV_I32 = 3   /* two's-complement int32 (never NaN or infinite)       */
+} nmv_dtype;
+
+/* ---- degenerate-output flags (nmv_result.flags) ------------------------ */
+/* Value-level stand-ins for the integrity hazards of Sections 1 and 4.3
+ * (host-fallback bypass, "repair by degeneration").  The paper checks
+ * integrity on source code; these numeric rules are this library's. */
+#define NMV_FLAG_CAND_EQ_INPUT 1u  /* some input j with the candidate's dtype
+                                      and numel has input_eq[j] >=
+                                      max(1, ceil(numel / 100)), where
+                                      input_eq[j] = #{i : bits(c_i) ==
+                                      bits(x_j,i) and bits(r_i) != bits(x_j,i)} */
+#define NMV_FLAG_CAND_ALL_ZERO 2u  /* numel >= 1, every c_i == 0 by value   */
+#define NMV_FLAG_CAND_CONSTANT 4u  /* numel >= 2, every bits(c_i) == bits(c_0) */
+#define NMV_FLAG_REF_ALL_ZERO 8u   /* the same rules applied to the reference */
+#define NMV_FLAG_REF_CONSTANT 16u
+
+/* One tensor: a device buffer of prod(shape) elements, contiguous row-major.
+ * `data` must be readable by the current CUDA device (device memory, or
+ * host memory the device can address).  It is borrowed, never written, and
+ * must stay valid until the call returns.  `shape` is host memory with
+ * `rank` entries, each >= 0 (it may be NULL when rank == 0; a rank-0 tensor
+ * has one element). */
+typedef struct nmv_tensor {
+    const void *data;
+    int32_t dtype;        /* nmv_dtype */
+    int32_t rank;         /* 0 .. NMV_MAX_RANK */
+    const int64_t *shape;
+} nmv_tensor;
+
+/* One validation case: the check Validate(K, R, T, tau) of Section 3.2 on
+ * one output pair.  The forensics view the tensors as the 2-D matrix
+ * [M, N] with M = prod(shape[:-1]) and N = shape[-1] (rank 1: M = 1; rank 0:
+ * [1, 1]); element i sits at row i / N, column i % N. */
+typedef struct nmv_case {
+    nmv_tensor cand;            /* candidate output (the repaired kernel's) */
+    nmv_tensor ref;             /* reference output; same dtype and shape   */
+    const nmv_tensor *inputs;   /* operator inputs for the pass-through
+                                   check; may be NULL when n_inputs == 0    */
+    int32_t n_inputs;           /* 0 .. NMV_MAX_INPUTS                       */
+    int32_t reserved;           /* must be 0                                */
+    double rtol, atol;          /* tau: finite and >= 0                     */
+    int64_t tile_rows;          /* localisation tile, 1 .. NMV_MAX_TILE     */
+    int64_t tile_cols;
+    int64_t first_k;            /* mismatch records to return, 0 .. NMV_MAX_FIRST_K */
+} nmv_case;
+
+/* Result of one case.  All arrays live in one host block owned by the
+ * library until nmv_result_free(). */
+typedef struct nmv_result {
+    int32_t status;             /* NMV_OK                                   */
+    int32_t rank;
+    int64_t numel;
+    int32_t pass;               /* 1 iff mismatch == 0 (torch.allclose)     */
+    uint32_t flags;             /* NMV_FLAG_* bits                          */
+    int64_t mismatch;           /* #{i : !pass(i)}; match rate = 1 - mismatch/numel */
+    int64_t cand_nan, cand_posinf, cand_neginf;
+    int64_t ref_nan, ref_posinf, ref_neginf;
+    int64_t n_finite_pairs;     /* #{i : c_i and r_i both finite}           */
+    /* Over the both-finite pairs, with d = fl64(c - r):                    */
+    double max_abs;             /* max |d|; 0.0 when there is no such pair  */
+    double max_rel;             /* max fl64(|d| / |r|) over r != 0          */
+    double sse;                 /* sum of d^2 (relative error <= 1e-9)      */
+    int64_t argmax_abs;         /* lowest index attaining max_abs, or -1    */
+    int64_t argmax_rel;         /* lowest index attaining max_rel, or -1    */
+    /* Localisation of the mismatches on the [M, N] view:                   */
+    int64_t grid_rows, grid_cols;   /* ceil(M/tile_rows), ceil(N/tile_cols); 0 when numel == 0 */
+    int64_t tile_rows, tile_cols;
+    int64_t *tile_hist;         /* [grid_rows * grid_cols] row-major: mismatches per tile */
+    int64_t *row_prof;          /* [tile_rows]: mismatches per (row % tile_rows) */
+    int64_t *col_prof;          /* [tile_cols]: mismatches per (col % tile_cols) */
+    /* The first min(first_k, mismatch) mismatches in ascending index order: */
+    int64_t k_out;
+    int64_t *fk_index;          /* [k_out] linear indices                  */
+    int64_t *fk_coords;         /* [k_out * rank] row-major coordinates      */
+    double *fk_cand;            /* [k_out] candidate values widened to fp64  */
+    double *fk_ref;             /* [k_out] reference values widened to fp64  */
+    /* Pass-through check:                                                  */
+    int32_t n_inputs;
+    int32_t passthrough_input;  /* lowest input that raised CAND_EQ_INPUT, or -1 */
+    int64_t *input_eq;          /* [n_inputs]; -1 for an input of another dtype or numel */
+} nmv_result;
+
+/* Validate one case on `cuda_stream` (a cudaStream_t; NULL = the legacy
+ * default stream).  Synchronous: returns after the stream has produced the
+ * result.  On NMV_OK, *out points to one nmv_result to be released with
+ * nmv_result_free().  On any error, *out is NULL, nothing stays allocated
+ * and nmv_last_error() describes the failure. */
+int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out);
+
+/* Validate n independent cases (a full-coverage sweep, Section 4.3) in one
+ * call: one descriptor upload, one launch of each kernel, one copy back.
+ * Results are identical, bit for bit, to n nmv_validate calls.  Every case
+ * is checked before any work starts; an invalid case fails the whole call
+ * (the message names its index).  On NMV_OK, *out points to an array of n
+ * results released by ONE nmv_result_free(*out) call. */
+int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
+                       nmv_result **out);
+
+/* Release what one nmv_validate / nmv_validate_batch call returned.  NULL
+ * is accepted. */
+void nmv_result_free(nmv_result *r);
+
+/* Static text for a status code. */
+const char *nmv_status_string(int status);
+
+/* Text of the last failure on the calling thread ("" if none). */
+const char *nmv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NMV_H */

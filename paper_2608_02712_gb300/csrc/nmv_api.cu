@@ -1,0 +1,706 @@
+// nmv_api.cu -- host side of libnmv: argument checks, work planning, the
+// cached device workspace, launches and the result arena.  Implements the C
+// ABI declared in include/nmv.h.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "nmv_internal.h"
+
+namespace nmv {
+template <int DT>
+struct ScanOps {
+  static cudaError_t prepare(int nin, size_t smem);
+  static int occupancy(int nin, size_t smem);
+  static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
+                            const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
+                            Partial *partials, int32_t *seg_count, uint32_t *seg_list, uint8_t *out,
+                            uint32_t *g_thr);
+};
+cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *,
+                            const uint32_t *, uint8_t *, int, cudaStream_t);
+
+cudaError_t scan_prepare(int dt, int nin, size_t smem) {
+  switch (dt) {
+    case NMV_F32: return ScanOps<NMV_F32>::prepare(nin, smem);
+    case NMV_F16: return ScanOps<NMV_F16>::prepare(nin, smem);
+    case NMV_BF16: return ScanOps<NMV_BF16>::prepare(nin, smem);
+    default: return ScanOps<NMV_I32>::prepare(nin, smem);
+  }
+}
+
+int scan_occupancy(int dt, int nin, size_t smem) {
+  switch (dt) {
+    case NMV_F32: return ScanOps<NMV_F32>::occupancy(nin, smem);
+    case NMV_F16: return ScanOps<NMV_F16>::occupancy(nin, smem);
+    case NMV_BF16: return ScanOps<NMV_BF16>::occupancy(nin, smem);
+    default: return ScanOps<NMV_I32>::occupancy(nin, smem);
+  }
+}
+
+cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
+                        const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
+                        Partial *partials, int32_t *seg_count, uint32_t *seg_list, uint8_t *out,
+                        uint32_t *g_thr) {
+  switch (dt) {
+    case NMV_F32:
+      return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+                                      partials, seg_count, seg_list, out, g_thr);
+    case NMV_F16:
+      return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+                                      partials, seg_count, seg_list, out, g_thr);
+    case NMV_BF16:
+      return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+                                       partials, seg_count, seg_list, out, g_thr);
+    default:
+      return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+                                      partials, seg_count, seg_list, out, g_thr);
+  }
+}
+}  // namespace nmv
+
+using namespace nmv;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const std::string &msg) {
+  g_err = msg;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char *what) {
+  return fail(NMV_ECUDA, std::string(what) + ": " + cudaGetErrorString(e));
+}
+
+// Host-side fault injection for tests of the error paths:
+// NMV_FAULT_INJECT=alloc|launch|d2h makes that step report a failure.
+bool injected(const char *step) {
+  const char *v = std::getenv("NMV_FAULT_INJECT");
+  return v && std::strstr(v, step) != nullptr;
+}
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceState {
+  bool probed = false;
+  int status = NMV_OK;
+  int sms = 0;
+  size_t smem_optin = 0;
+  size_t smem_set[4][3] = {};  // dynamic smem opted in per kernel instantiation
+  void *ws = nullptr;
+  size_t ws_size = 0;
+  void *pinned = nullptr;
+  size_t pinned_size = 0;
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+float f32_down(double x) {
+  float f = (float)x;
+  if ((double)f > x) f = std::nextafter(f, -INFINITY);
+  return f;
+}
+
+float f32_up(double x) {
+  float f = (float)x;
+  if ((double)f < x) f = std::nextafter(f, INFINITY);
+  return f;
+}
+
+bool valid_dtype(int32_t dt) { return dt >= NMV_F32 && dt <= NMV_I32; }
+
+// numel of a tensor, or -1 if its shape is invalid.
+int64_t tensor_numel(const nmv_tensor &t) {
+  if (t.rank < 0 || t.rank > NMV_MAX_RANK) return -1;
+  if (t.rank > 0 && t.shape == nullptr) return -1;
+  int64_t n = 1;
+  for (int d = 0; d < t.rank; ++d) {
+    const int64_t s = t.shape[d];
+    if (s < 0) return -1;
+    if (s != 0 && n > (int64_t(1) << 62) / s) return -1;
+    n *= s;
+  }
+  return n;
+}
+
+struct Geo {
+  int64_t numel, M, N, GR, GC;
+  int dt, eb, vec;
+  size_t out_size, hist_off, rowp_off, colp_off, fk_off;
+};
+
+int check_tensor(const nmv_tensor &t, const char *what, int64_t *numel) {
+  if (!valid_dtype(t.dtype)) return fail(NMV_EINVAL, std::string(what) + ": unknown dtype");
+  const int64_t n = tensor_numel(t);
+  if (n < 0) return fail(NMV_EINVAL, std::string(what) + ": invalid rank or shape");
+  if (n > 0 && t.data == nullptr) return fail(NMV_EINVAL, std::string(what) + ": NULL data");
+  *numel = n;
+  return NMV_OK;
+}
+
+int check_case(const nmv_case &c, Geo *g) {
+  int64_t nc = 0, nr = 0;
+  int rc = check_tensor(c.cand, "cand", &nc);
+  if (rc) return rc;
+  rc = check_tensor(c.ref, "ref", &nr);
+  if (rc) return rc;
+  if (c.cand.dtype != c.ref.dtype) return fail(NMV_EINVAL, "cand and ref dtypes differ");
+  if (c.cand.rank != c.ref.rank) return fail(NMV_EINVAL, "cand and ref ranks differ");
+  for (int d = 0; d < c.cand.rank; ++d)
+    if (c.cand.shape[d] != c.ref.shape[d]) return fail(NMV_EINVAL, "cand and ref shapes differ");
+  if (c.n_inputs < 0 || c.n_inputs > NMV_MAX_INPUTS)
+    return fail(NMV_EINVAL, "n_inputs out of range [0, NMV_MAX_INPUTS]");
+  if (c.n_inputs > 0 && c.inputs == nullptr) return fail(NMV_EINVAL, "inputs is NULL");
+  for (int j = 0; j < c.n_inputs; ++j) {
+    int64_t ni = 0;
+    rc = check_tensor(c.inputs[j], "input", &ni);
+    if (rc) return rc;
+  }
+  if (c.reserved != 0) return fail(NMV_EINVAL, "reserved must be 0");
+  if (!std::isfinite(c.rtol) || !std::isfinite(c.atol) || c.rtol < 0 || c.atol < 0)
+    return fail(NMV_EINVAL, "rtol and atol must be finite and >= 0");
+  if (c.tile_rows < 1 || c.tile_cols < 1 || c.tile_rows > NMV_MAX_TILE || c.tile_cols > NMV_MAX_TILE)
+    return fail(NMV_EINVAL, "tile_rows and tile_cols must lie in [1, NMV_MAX_TILE]");
+  if (c.first_k < 0 || c.first_k > NMV_MAX_FIRST_K)
+    return fail(NMV_EINVAL, "first_k out of range [0, NMV_MAX_FIRST_K]");
+  g->numel = nc;
+  g->dt = c.cand.dtype;
+  g->eb = elem_bytes(g->dt);
+  g->vec = vec_elems(g->dt);
+  if (c.cand.rank == 0) {
+    g->M = 1;
+    g->N = 1;
+  } else {
+    g->N = c.cand.shape[c.cand.rank - 1];
+    g->M = 1;
+    for (int d = 0; d + 1 < c.cand.rank; ++d) g->M *= c.cand.shape[d];
+  }
+  if (nc == 0) {
+    g->GR = 0;
+    g->GC = 0;
+  } else {
+    g->GR = (g->M + c.tile_rows - 1) / c.tile_rows;
+    g->GC = (g->N + c.tile_cols - 1) / c.tile_cols;
+    if (g->GR > NMV_MAX_HIST_BINS / g->GC)
+      return fail(NMV_EINVAL, "tile grid exceeds NMV_MAX_HIST_BINS bins");
+  }
+  size_t off = align_up(sizeof(OutHeader), 256);
+  g->hist_off = off;
+  off = align_up(off + (size_t)(g->GR * g->GC) * 8, 256);
+  g->rowp_off = off;
+  off = align_up(off + (size_t)c.tile_rows * 8, 256);
+  g->colp_off = off;
+  off = align_up(off + (size_t)c.tile_cols * 8, 256);
+  g->fk_off = off;
+  off = align_up(off + (size_t)c.first_k * 24, 256);
+  g->out_size = off;
+  return NMV_OK;
+}
+
+int probe_device(int *dev_out, DeviceState **st_out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(NMV_EUNSUPPORTED, "device ordinal out of range");
+  DeviceState &s = g_dev[dev];
+  if (!s.probed) {
+    cudaDeviceProp p;
+    e = cudaGetDeviceProperties(&p, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+    s.probed = true;
+    if (!(p.major == 10 && p.minor == 3)) {
+      s.status = NMV_EUNSUPPORTED;
+    } else {
+      s.sms = p.multiProcessorCount;
+      s.smem_optin = p.sharedMemPerBlockOptin;
+    }
+  }
+  if (s.status != NMV_OK) return fail(s.status, "libnmv is built for sm_103 (GB300) only");
+  *dev_out = dev;
+  *st_out = &s;
+  return NMV_OK;
+}
+
+int ensure_workspace(DeviceState &s, size_t ws, size_t pinned) {
+  if (injected("alloc")) return fail(NMV_ENOMEM, "injected allocation failure");
+  if (ws > s.ws_size) {
+    if (s.ws) cudaFree(s.ws);
+    s.ws = nullptr;
+    s.ws_size = 0;
+    size_t want = std::max(ws, s.ws_size * 2);
+    cudaError_t e = cudaMalloc(&s.ws, want);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      s.ws = nullptr;
+      return fail(NMV_ENOMEM, std::string("cudaMalloc workspace: ") + cudaGetErrorString(e));
+    }
+    s.ws_size = want;
+  }
+  if (pinned > s.pinned_size) {
+    if (s.pinned) cudaFreeHost(s.pinned);
+    s.pinned = nullptr;
+    s.pinned_size = 0;
+    size_t want = std::max(pinned, s.pinned_size * 2);
+    cudaError_t e = cudaHostAlloc(&s.pinned, want, cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      s.pinned = nullptr;
+      return fail(NMV_ENOMEM, std::string("cudaHostAlloc staging: ") + cudaGetErrorString(e));
+    }
+    s.pinned_size = want;
+  }
+  return NMV_OK;
+}
+
+struct Plan {
+  std::vector<Piece> pieces;
+  std::vector<int64_t> block_piece;
+  size_t smem = 0;
+};
+
+void piece_window(const nmv_case &c, const Geo &g, Piece &p) {
+  const int64_t th = c.tile_rows, tw = c.tile_cols;
+  const int64_t r0 = p.begin / g.N, r1 = (p.end - 1) / g.N;
+  int64_t wr, wc;
+  if (r0 == r1) {
+    p.tr0 = r0 / th;
+    p.tc0 = (p.begin % g.N) / tw;
+    wr = 1;
+    wc = ((p.end - 1) % g.N) / tw - p.tc0 + 1;
+  } else {
+    p.tr0 = r0 / th;
+    p.tc0 = 0;
+    wr = r1 / th - p.tr0 + 1;
+    wc = g.GC;
+  }
+  if (wr > 0 && wc > 0 && wr <= kHistCap / wc) {
+    p.wr = (int32_t)wr;
+    p.wc = (int32_t)wc;
+  } else {
+    p.wr = 0;
+    p.wc = 0;
+  }
+  p.prof_smem = (th <= kProfCap && tw <= kProfCap) ? 1 : 0;
+}
+
+// Shared-memory words of the scan kernel's head (class counters and the
+// generic input path's pass-through counters).
+constexpr size_t kShHeadWords = 16;
+
+size_t piece_smem(const nmv_case &c, const Piece &p) {
+  size_t words = kShHeadWords;
+  if (p.prof_smem) words += (size_t)(c.tile_rows + c.tile_cols);
+  words += (size_t)p.wr * (size_t)p.wc;
+  return words * 4;
+}
+
+// Split the concatenated bytes of the cases `ids` into `grid` balanced block
+// ranges; cut them at case boundaries (and at kMaxPiece) into pieces whose
+// element boundaries are multiples of the case's vector width.
+void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::vector<int64_t> &ids,
+               int grid, Plan &plan) {
+  const int64_t n = (int64_t)ids.size();
+  std::vector<int64_t> off(n + 1, 0);
+  for (int64_t i = 0; i < n; ++i) off[i + 1] = off[i] + geo[ids[i]].numel * geo[ids[i]].eb;
+  const int64_t total = off[n];
+  std::vector<int64_t> sc(grid + 1), se(grid + 1);
+  int64_t ci = 0;
+  for (int b = 0; b <= grid; ++b) {
+    const int64_t x = (b == grid) ? total : (int64_t)((__int128)total * b / grid);
+    while (ci < n && off[ci + 1] <= x) ++ci;
+    if (ci >= n || b == grid) {
+      sc[b] = n;
+      se[b] = 0;
+      continue;
+    }
+    const Geo &g = geo[ids[ci]];
+    int64_t e = (x - off[ci]) / g.eb;
+    e = e / g.vec * g.vec;
+    sc[b] = ci;
+    se[b] = e;
+  }
+  plan.pieces.clear();
+  plan.block_piece.assign(grid + 1, 0);
+  plan.smem = 0;
+  for (int b = 0; b < grid; ++b) {
+    plan.block_piece[b] = (int64_t)plan.pieces.size();
+    for (int64_t c = sc[b]; c <= std::min(sc[b + 1], n - 1); ++c) {
+      const Geo &g = geo[ids[c]];
+      if (g.numel == 0) continue;
+      const int64_t beg = (c == sc[b]) ? se[b] : 0;
+      const int64_t end = (c == sc[b + 1]) ? se[b + 1] : g.numel;
+      for (int64_t s = beg; s < end; s += kMaxPiece) {
+        Piece p;
+        std::memset(&p, 0, sizeof(p));
+        p.begin = s;
+        p.end = std::min(end, s + kMaxPiece);
+        p.case_id = (int32_t)ids[c];
+        piece_window(cases[ids[c]], g, p);
+        plan.smem = std::max(plan.smem, piece_smem(cases[ids[c]], p));
+        plan.pieces.push_back(p);
+      }
+    }
+  }
+  plan.block_piece[grid] = (int64_t)plan.pieces.size();
+}
+
+// Cases that share an element type and an input-count class run in one
+// launch of the matching kernel instantiation.
+struct Group {
+  int dt = 0, nin = 0;
+  std::vector<int64_t> ids;
+  Plan plan;
+  int grid = 0;
+  size_t smem = 0;
+  int64_t piece_base = 0;
+  int64_t bp_base = 0;
+};
+
+int nin_class(const nmv_case &c, const Geo &g) {
+  int ne = 0;
+  for (int j = 0; j < c.n_inputs; ++j) {
+    const nmv_tensor &x = c.inputs[j];
+    if (x.dtype == c.cand.dtype && tensor_numel(x) == g.numel && g.numel > 0) ++ne;
+  }
+  return ne == 0 ? 0 : (ne == 1 ? 1 : -1);
+}
+
+void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
+  std::memset(&d, 0, sizeof(d));
+  d.cand = c.cand.data;
+  d.ref = c.ref.data;
+  d.n_inputs = c.n_inputs;
+  d.dtype = g.dt;
+  bool aligned = ((uintptr_t)c.cand.data % 16 == 0) && ((uintptr_t)c.ref.data % 16 == 0);
+  int ne = 0;
+  for (int j = 0; j < c.n_inputs; ++j) {
+    const nmv_tensor &x = c.inputs[j];
+    if (x.dtype == c.cand.dtype && tensor_numel(x) == g.numel && g.numel > 0) {
+      d.in_ptr[ne] = x.data;
+      d.in_slot[ne] = j;
+      aligned = aligned && ((uintptr_t)x.data % 16 == 0);
+      ++ne;
+    }
+  }
+  d.n_elig = ne;
+  d.vec_ok = aligned ? 1 : 0;
+  d.numel = g.numel;
+  d.M = g.M;
+  d.N = g.N > 0 ? g.N : 1;
+  d.th = c.tile_rows;
+  d.tw = c.tile_cols;
+  d.GR = g.GR;
+  d.GC = g.GC;
+  d.dN = make_div((uint64_t)d.N);
+  d.dth = make_div((uint64_t)d.th);
+  d.dtw = make_div((uint64_t)d.tw);
+  d.rtol = c.rtol;
+  d.atol = c.atol;
+  // fp32 pre-filter coefficients (margins of 2^-20; see nmv_kernels.cu)
+  const bool filter = c.rtol <= 0.5 && c.atol <= 0x1p100;
+  d.filter_ok = filter ? 1 : 0;
+  if (filter) {
+    d.lo_r = f32_down(c.rtol * (1.0 - 0x1p-20));
+    d.lo_a = f32_down(c.atol * (1.0 - 0x1p-20));
+    d.hi_r = f32_up(c.rtol * (1.0 + 0x1p-20));
+    d.hi_a = f32_up(c.atol * (1.0 + 0x1p-20));
+  } else {
+    d.lo_r = 0.f;
+    d.lo_a = -1.f;          // never sure-pass
+    d.hi_r = 0.f;
+    d.hi_a = INFINITY;      // never sure-fail
+  }
+  d.first_k = c.first_k;
+  d.hist_off = (int64_t)g.hist_off;
+  d.rowp_off = (int64_t)g.rowp_off;
+  d.colp_off = (int64_t)g.colp_off;
+  d.fk_off = (int64_t)g.fk_off;
+}
+
+int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
+  if (out == nullptr) return fail(NMV_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (cases == nullptr && n > 0) return fail(NMV_EINVAL, "cases is NULL");
+  if (n < 0 || n > NMV_MAX_CASES) return fail(NMV_EINVAL, "case count out of range");
+  std::vector<Geo> geo((size_t)n);
+  for (int64_t i = 0; i < n; ++i) {
+    const int rc = check_case(cases[i], &geo[i]);
+    if (rc) {
+      char buf[64];
+      std::snprintf(buf, sizeof buf, "case %lld: ", (long long)i);
+      g_err = buf + g_err;
+      return rc;
+    }
+  }
+  if (n == 0) return NMV_OK;
+
+  std::lock_guard<std::mutex> lock(g_mu);
+  int dev = -1;
+  DeviceState *S = nullptr;
+  int rc = probe_device(&dev, &S);
+  if (rc) return rc;
+  cudaStream_t st = (cudaStream_t)stream;
+
+  // ---- plan: one group per (element type, input class), each with a
+  // full grid of its own, launched back to back on the stream.
+  std::vector<Group> groups;
+  {
+    int slot[4][3];
+    for (auto &row : slot)
+      for (int &v : row) v = -1;
+    for (int64_t i = 0; i < n; ++i) {
+      if (geo[i].numel == 0) continue;
+      const int nin = nin_class(cases[i], geo[i]);
+      int &gi = slot[geo[i].dt][nin + 1];
+      if (gi < 0) {
+        gi = (int)groups.size();
+        groups.emplace_back();
+        groups.back().dt = geo[i].dt;
+        groups.back().nin = nin;
+      }
+      groups[gi].ids.push_back(i);
+    }
+  }
+  int64_t np = 0, nbp = 0;
+  for (Group &G : groups) {
+    int64_t total_bytes = 0;
+    size_t prof_smem = kShHeadWords * 4;
+    for (int64_t i : G.ids) {
+      total_bytes += geo[i].numel * geo[i].eb;
+      if (cases[i].tile_rows <= kProfCap && cases[i].tile_cols <= kProfCap)
+        prof_smem = std::max(prof_smem, (size_t)(kShHeadWords + cases[i].tile_rows + cases[i].tile_cols) * 4);
+    }
+    size_t guess = prof_smem;
+    for (int attempt = 0; attempt < 3; ++attempt) {
+      const size_t want = std::min(std::max(guess, (size_t)1024), S->smem_optin);
+      size_t &set = S->smem_set[G.dt][G.nin + 1];
+      if (want > set) {
+        cudaError_t e = scan_prepare(G.dt, G.nin, want);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+        set = want;
+      }
+      int occ = scan_occupancy(G.dt, G.nin, want);
+      if (occ < 1) occ = 1;
+      int64_t g = (int64_t)S->sms * occ;
+      g = std::min(g, std::max<int64_t>(1, total_bytes / 16384));
+      G.grid = (int)g;
+      make_plan(cases, geo, G.ids, G.grid, G.plan);
+      G.smem = std::max(G.plan.smem, (size_t)1024);
+      if (G.plan.smem <= want) break;
+      guess = G.plan.smem;
+    }
+    if (G.smem > S->smem_optin)
+      return fail(NMV_EINVAL, "localisation maps need more shared memory than the device has");
+    size_t &set = S->smem_set[G.dt][G.nin + 1];
+    if (G.smem > set) {
+      cudaError_t e = scan_prepare(G.dt, G.nin, G.smem);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+      set = G.smem;
+    }
+    G.piece_base = np;
+    G.bp_base = nbp;
+    np += (int64_t)G.plan.pieces.size();
+    nbp += G.grid + 1;
+  }
+
+  // ---- descriptors (pieces of a case are contiguous within its group)
+  std::vector<CaseDesc> desc((size_t)n);
+  std::vector<Piece> all_pieces;
+  std::vector<int64_t> all_bp;
+  all_pieces.reserve((size_t)np);
+  all_bp.reserve((size_t)nbp);
+  size_t out_size = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    fill_desc(cases[i], geo[i], desc[i]);
+    desc[i].out_off = (int64_t)out_size;
+    out_size += geo[i].out_size;
+    desc[i].piece_begin = 0;
+    desc[i].piece_end = 0;
+  }
+  for (Group &G : groups) {
+    for (size_t k = 0; k < G.plan.pieces.size(); ++k) {
+      const Piece &p = G.plan.pieces[k];
+      const int64_t gid = G.piece_base + (int64_t)k;
+      CaseDesc &d = desc[p.case_id];
+      if (d.piece_end == 0) d.piece_begin = gid;
+      d.piece_end = gid + 1;
+      all_pieces.push_back(p);
+    }
+    all_bp.insert(all_bp.end(), G.plan.block_piece.begin(), G.plan.block_piece.end());
+  }
+
+  // ---- workspace layout
+  const size_t sz_cases = align_up(sizeof(CaseDesc) * n, 256);
+  const size_t sz_pieces = align_up(sizeof(Piece) * std::max<int64_t>(np, 1), 256);
+  const size_t sz_bp = align_up(sizeof(int64_t) * std::max<int64_t>(nbp, 1), 256);
+  const size_t table = sz_cases + sz_pieces + sz_bp;
+  const size_t sz_part = align_up(sizeof(Partial) * std::max<int64_t>(np, 1), 256);
+  const size_t sz_segc = align_up(sizeof(int32_t) * kWarps * std::max<int64_t>(np, 1), 256);
+  const size_t sz_segl = align_up(sizeof(uint32_t) * kWarps * kFirstR * std::max<int64_t>(np, 1), 256);
+  const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n, 256);
+  const size_t o_part = table, o_segc = o_part + sz_part, o_segl = o_segc + sz_segc;
+  const size_t o_thr = o_segl + sz_segl, o_out = o_thr + sz_thr;
+  const size_t ws = o_out + out_size;
+  rc = ensure_workspace(*S, ws, table + out_size);
+  if (rc) return rc;
+  uint8_t *W = (uint8_t *)S->ws;
+  uint8_t *H = (uint8_t *)S->pinned;
+  std::memcpy(H, desc.data(), sizeof(CaseDesc) * n);
+  if (np) std::memcpy(H + sz_cases, all_pieces.data(), sizeof(Piece) * np);
+  if (nbp) std::memcpy(H + sz_cases + sz_pieces, all_bp.data(), sizeof(int64_t) * nbp);
+
+  cudaError_t e = cudaMemcpyAsync(W, H, table, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
+  e = cudaMemsetAsync(W + o_thr, 0, sz_thr + out_size, st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  const CaseDesc *d_cases = (const CaseDesc *)W;
+  const Piece *d_pieces = (const Piece *)(W + sz_cases);
+  const int64_t *d_bp = (const int64_t *)(W + sz_cases + sz_pieces);
+  if (injected("launch")) {
+    cudaStreamSynchronize(st);
+    return fail(NMV_ECUDA, "injected launch failure");
+  }
+  for (const Group &G : groups) {
+    e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_bp + G.bp_base,
+                    G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc),
+                    (uint32_t *)(W + o_segl), W + o_out, (uint32_t *)(W + o_thr));
+    if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
+  }
+  e = launch_finalize(d_cases, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc),
+                      (const uint32_t *)(W + o_segl), W + o_out, (int)n, st);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  uint8_t *HO = H + table;
+  e = cudaMemcpyAsync(HO, W + o_out, out_size, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (results)");
+  e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  if (injected("d2h")) return fail(NMV_ECUDA, "injected copy-back failure");
+
+  // ---- result arena
+  size_t bytes = align_up(sizeof(nmv_result) * n, 16);
+  for (int64_t i = 0; i < n; ++i) {
+    const OutHeader *oh = (const OutHeader *)(HO + desc[i].out_off);
+    const nmv_case &c = cases[i];
+    const int64_t k = oh->k_out;
+    bytes += 8 * (size_t)(geo[i].GR * geo[i].GC + c.tile_rows + c.tile_cols);
+    bytes += 8 * (size_t)k * (3 + (size_t)c.cand.rank);
+    bytes += 8 * (size_t)c.n_inputs;
+  }
+  uint8_t *arena = (uint8_t *)std::malloc(bytes);
+  if (!arena) return fail(NMV_ENOMEM, "malloc result arena");
+  nmv_result *res = (nmv_result *)arena;
+  uint8_t *cur = arena + align_up(sizeof(nmv_result) * n, 16);
+  auto take = [&](size_t nbytes) {
+    uint8_t *p = cur;
+    cur += nbytes;
+    return p;
+  };
+  for (int64_t i = 0; i < n; ++i) {
+    const uint8_t *ob = HO + desc[i].out_off;
+    const OutHeader *oh = (const OutHeader *)ob;
+    const nmv_case &c = cases[i];
+    const Geo &g = geo[i];
+    nmv_result &r = res[i];
+    std::memset(&r, 0, sizeof(r));
+    r.status = (int32_t)oh->status;
+    r.rank = c.cand.rank;
+    r.numel = g.numel;
+    r.mismatch = oh->cnt[0];
+    r.cand_nan = oh->cnt[1];
+    r.cand_posinf = oh->cnt[2];
+    r.cand_neginf = oh->cnt[3];
+    r.ref_nan = oh->cnt[4];
+    r.ref_posinf = oh->cnt[5];
+    r.ref_neginf = oh->cnt[6];
+    r.n_finite_pairs = oh->cnt[7];
+    r.pass = r.mismatch == 0;
+    r.flags = oh->flags;
+    r.max_abs = oh->max_abs;
+    r.max_rel = oh->max_rel;
+    r.sse = oh->sse;
+    r.argmax_abs = oh->argmax_abs;
+    r.argmax_rel = oh->argmax_rel;
+    r.grid_rows = g.GR;
+    r.grid_cols = g.GC;
+    r.tile_rows = c.tile_rows;
+    r.tile_cols = c.tile_cols;
+    const size_t nb = (size_t)(g.GR * g.GC);
+    r.tile_hist = (int64_t *)take(8 * nb);
+    std::memcpy(r.tile_hist, ob + g.hist_off, 8 * nb);
+    r.row_prof = (int64_t *)take(8 * (size_t)c.tile_rows);
+    std::memcpy(r.row_prof, ob + g.rowp_off, 8 * (size_t)c.tile_rows);
+    r.col_prof = (int64_t *)take(8 * (size_t)c.tile_cols);
+    std::memcpy(r.col_prof, ob + g.colp_off, 8 * (size_t)c.tile_cols);
+    const int64_t k = oh->k_out;
+    r.k_out = k;
+    r.fk_index = (int64_t *)take(8 * (size_t)k);
+    r.fk_coords = (int64_t *)take(8 * (size_t)k * (size_t)c.cand.rank);
+    r.fk_cand = (double *)take(8 * (size_t)k);
+    r.fk_ref = (double *)take(8 * (size_t)k);
+    const int64_t *fki = (const int64_t *)(ob + g.fk_off);
+    const double *fkc = (const double *)(fki + c.first_k);
+    const double *fkr = fkc + c.first_k;
+    std::memcpy(r.fk_index, fki, 8 * (size_t)k);
+    std::memcpy(r.fk_cand, fkc, 8 * (size_t)k);
+    std::memcpy(r.fk_ref, fkr, 8 * (size_t)k);
+    for (int64_t t = 0; t < k; ++t) {
+      int64_t idx = r.fk_index[t];
+      for (int d = c.cand.rank - 1; d >= 0; --d) {
+        const int64_t s = c.cand.shape[d];
+        r.fk_coords[t * c.cand.rank + d] = s > 0 ? idx % s : 0;
+        idx = s > 0 ? idx / s : 0;
+      }
+    }
+    r.n_inputs = c.n_inputs;
+    r.passthrough_input = oh->passthrough;
+    r.input_eq = (int64_t *)take(8 * (size_t)c.n_inputs);
+    for (int j = 0; j < c.n_inputs; ++j) r.input_eq[j] = oh->input_eq[j];
+  }
+  *out = res;
+  g_err.clear();
+  return NMV_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out) {
+  if (out) *out = nullptr;
+  if (c == nullptr) return fail(NMV_EINVAL, "case is NULL");
+  return run(c, 1, cuda_stream, out);
+}
+
+int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream, nmv_result **out) {
+  return run(cases, n, cuda_stream, out);
+}
+
+void nmv_result_free(nmv_result *r) { std::free(r); }
+
+const char *nmv_status_string(int status) {
+  switch (status) {
+    case NMV_OK: return "ok";
+    case NMV_EINVAL: return "invalid argument";
+    case NMV_ENOMEM: return "out of memory";
+    case NMV_ECUDA: return "CUDA error";
+    case NMV_EUNSUPPORTED: return "unsupported device";
+    default: return "unknown status";
+  }
+}
+
+const char *nmv_last_error(void) { return g_err.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,118 @@
+// nmv_internal.h -- descriptors shared by the host planner (nmv_api.cu) and
+// the kernels (nmv_kernels.cu).  Not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+
+#include "../../include/nmv.h"
+
+#ifdef __CUDACC__
+#define NMV_HD __host__ __device__ __forceinline__
+#else
+#define NMV_HD inline
+#endif
+
+namespace nmv {
+
+// ---- launch geometry ----------------------------------------------------
+constexpr int kWarps = 8;                 // warps per block of the scan kernel
+constexpr int kThreads = kWarps * 32;
+constexpr int kFirstR = 128;              // mismatch offsets kept per segment
+constexpr int kFinThreads = 256;          // threads per block of the finalize kernel
+constexpr int64_t kHistCap = 8192;        // smem tile-histogram window (bins)
+constexpr int64_t kProfCap = 4096;        // smem row / column profile (bins each)
+constexpr int64_t kMaxPiece = int64_t(1) << 30;  // elements per piece (int32 smem counters)
+constexpr int kSseFlush = 64;             // float-float SSE terms per fp64 flush
+
+// Element size in bytes and elements per 16-byte vector.
+NMV_HD int elem_bytes(int dt) { return (dt == NMV_F16 || dt == NMV_BF16) ? 2 : 4; }
+NMV_HD int vec_elems(int dt) { return 16 / elem_bytes(dt); }
+
+// Division of a 64-bit unsigned value by an invariant d >= 1:
+// m = floor((2^64 - 1) / d) gives q0 = mulhi(n, m) in {q - 1, q} for
+// n < 2^63, and one compare fixes it.
+struct Div64 {
+  uint64_t d;
+  uint64_t m;
+};
+
+inline Div64 make_div(uint64_t d) {
+  Div64 r;
+  r.d = d;
+  r.m = ~uint64_t(0) / d;
+  return r;
+}
+
+// One validation case as the kernels see it.
+struct CaseDesc {
+  const void *cand;
+  const void *ref;
+  const void *in_ptr[NMV_MAX_INPUTS];  // eligible inputs only (same dtype, numel)
+  int32_t in_slot[NMV_MAX_INPUTS];     // their index in the caller's input list
+  int32_t n_elig;
+  int32_t n_inputs;                    // caller's input count
+  int32_t dtype;
+  int32_t vec_ok;                      // all buffers 16-byte aligned
+  int32_t filter_ok;                   // the fp32 pre-filter of the predicate is valid
+  int32_t pad0;
+  int64_t numel, M, N, th, tw, GR, GC;
+  Div64 dN, dth, dtw;
+  double rtol, atol;
+  // fp32 pre-filter of the predicate: sure-pass if |s| <= fma_rz(lo_r, |r|, lo_a),
+  // sure-fail if |s| > fma_ru(hi_r, |r|, hi_a) (see element_pass).
+  float lo_r, lo_a, hi_r, hi_a;
+  int64_t first_k;
+  int64_t piece_begin, piece_end;      // this case's pieces
+  int64_t out_off;                     // byte offset of this case's packed result
+  int64_t hist_off, rowp_off, colp_off, fk_off;  // byte offsets inside the packed result
+};
+
+// A contiguous element range of one case processed by one block.  The
+// block's warps split it into kWarps segments (segment_range).
+struct Piece {
+  int64_t begin, end;
+  int64_t tr0, tc0;     // smem tile-histogram window origin (tile coordinates)
+  int32_t wr, wc;       // window extent; wr == 0 -> histogram via global atomics
+  int32_t case_id;
+  int32_t prof_smem;    // 1 -> row / column profiles privatised in smem
+};
+
+// Per-piece partial result, reduced by the finalize kernel.
+struct Partial {
+  int64_t cnt[8];       // mismatch, cnan, cpinf, cninf, rnan, rpinf, rninf, nonfinite pairs
+  double best_abs;
+  double best_rel;
+  double sse;
+  int64_t arg_abs;
+  int64_t arg_rel;
+  uint32_t cacc, racc;  // OR of (bits ^ bits of element 0)
+  int64_t eq[NMV_MAX_INPUTS];
+};
+
+// Header of one case's packed result (followed by the arrays).
+struct OutHeader {
+  int64_t cnt[8];       // as Partial::cnt, but [7] = n_finite_pairs
+  double max_abs, max_rel, sse;
+  int64_t argmax_abs, argmax_rel, k_out;
+  uint32_t flags;
+  int32_t passthrough;
+  int64_t input_eq[NMV_MAX_INPUTS];
+  int64_t status;
+  int64_t pad[3];
+};
+
+// Segment w of a piece [begin, end): a split into kWarps contiguous ranges
+// whose boundaries are multiples of `vec` elements past `begin`.
+NMV_HD void segment_range(int64_t begin, int64_t end, int w, int vec, int64_t *lo,
+                          int64_t *hi) {
+  int64_t len = end - begin;
+  int64_t per = (len + kWarps - 1) / kWarps;
+  per = (per + vec - 1) / vec * vec;
+  int64_t a = per * w, b = per * (w + 1);
+  if (a > len) a = len;
+  if (b > len) b = len;
+  *lo = begin + a;
+  *hi = begin + b;
+}
+
+}  // namespace nmv

@@ -1,0 +1,253 @@
+"""ctypes binding of libnmv.so (include/nmv.h): argument marshalling only.
+
+Every step of the validation runs in the library's CUDA kernels; this module
+turns torch CUDA tensors into ``nmv_tensor`` / ``nmv_case`` structs, calls the
+C ABI, and copies the returned ``nmv_result`` into a dict.  It raises if the
+library is missing: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libnmv.so")
+
+NMV_OK, NMV_EINVAL, NMV_ENOMEM, NMV_ECUDA, NMV_EUNSUPPORTED = 0, -1, -2, -3, -4
+MAX_RANK, MAX_INPUTS = 8, 8
+DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2, torch.int32: 3}
+FLAGS = {"CAND_EQ_INPUT": 1, "CAND_ALL_ZERO": 2, "CAND_CONSTANT": 4,
+         "REF_ALL_ZERO": 8, "REF_CONSTANT": 16}
+
+_i64p = ctypes.POINTER(ctypes.c_int64)
+_f64p = ctypes.POINTER(ctypes.c_double)
+
+
+class Tensor(ctypes.Structure):
+    _fields_ = [("data", ctypes.c_void_p), ("dtype", ctypes.c_int32),
+                ("rank", ctypes.c_int32), ("shape", _i64p)]
+
+
+class Case(ctypes.Structure):
+    _fields_ = [("cand", Tensor), ("ref", Tensor), ("inputs", ctypes.POINTER(Tensor)),
+                ("n_inputs", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("rtol", ctypes.c_double), ("atol", ctypes.c_double),
+                ("tile_rows", ctypes.c_int64), ("tile_cols", ctypes.c_int64),
+                ("first_k", ctypes.c_int64)]
+
+
+class Result(ctypes.Structure):
+    _fields_ = [("status", ctypes.c_int32), ("rank", ctypes.c_int32), ("numel", ctypes.c_int64),
+                ("pass_", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("mismatch", ctypes.c_int64), ("cand_nan", ctypes.c_int64),
+                ("cand_posinf", ctypes.c_int64), ("cand_neginf", ctypes.c_int64),
+                ("ref_nan", ctypes.c_int64), ("ref_posinf", ctypes.c_int64),
+                ("ref_neginf", ctypes.c_int64), ("n_finite_pairs", ctypes.c_int64),
+                ("max_abs", ctypes.c_double), ("max_rel", ctypes.c_double),
+                ("sse", ctypes.c_double), ("argmax_abs", ctypes.c_int64),
+                ("argmax_rel", ctypes.c_int64), ("grid_rows", ctypes.c_int64),
+                ("grid_cols", ctypes.c_int64), ("tile_rows", ctypes.c_int64),
+                ("tile_cols", ctypes.c_int64), ("tile_hist", _i64p), ("row_prof", _i64p),
+                ("col_prof", _i64p), ("k_out", ctypes.c_int64), ("fk_index", _i64p),
+                ("fk_coords", _i64p), ("fk_cand", _f64p), ("fk_ref", _f64p),
+                ("n_inputs", ctypes.c_int32), ("passthrough_input", ctypes.c_int32),
+                ("input_eq", _i64p)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load() -> ctypes.CDLL:
+    """Load libnmv.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    "libnmv.so is not built (run __graft_entry__.build() or "
+                    "python -m paper_2608_02712_gb300._build); there is no fallback")
+            lib = ctypes.CDLL(LIB_PATH)
+            lib.nmv_validate.restype = ctypes.c_int
+            lib.nmv_validate.argtypes = [ctypes.POINTER(Case), ctypes.c_void_p,
+                                         ctypes.POINTER(ctypes.POINTER(Result))]
+            lib.nmv_validate_batch.restype = ctypes.c_int
+            lib.nmv_validate_batch.argtypes = [ctypes.POINTER(Case), ctypes.c_int64,
+                                               ctypes.c_void_p,
+                                               ctypes.POINTER(ctypes.POINTER(Result))]
+            lib.nmv_result_free.restype = None
+            lib.nmv_result_free.argtypes = [ctypes.POINTER(Result)]
+            lib.nmv_status_string.restype = ctypes.c_char_p
+            lib.nmv_status_string.argtypes = [ctypes.c_int]
+            lib.nmv_last_error.restype = ctypes.c_char_p
+            lib.nmv_last_error.argtypes = []
+            _lib = lib
+    return _lib
+
+
+class NmvError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__("nmv status %d: %s" % (status, message))
+        self.status = status
+
+
+def _raise(lib, rc):
+    raise NmvError(rc, (lib.nmv_last_error() or b"").decode() or
+                   lib.nmv_status_string(rc).decode())
+
+
+class _Keep:
+    """Holds the ctypes objects a Case points into."""
+
+    def __init__(self):
+        self.items = []
+
+
+def _tensor(t: torch.Tensor, keep: _Keep, device_only: bool = True) -> Tensor:
+    if t.dtype not in DTYPES:
+        raise TypeError("unsupported dtype %s" % t.dtype)
+    if device_only and not t.is_cuda:
+        raise ValueError("tensors must live on the CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("tensors must be contiguous")
+    shape = (ctypes.c_int64 * max(t.dim(), 1))(*t.shape)
+    keep.items.append(shape)
+    return Tensor(ctypes.c_void_p(t.data_ptr() if t.numel() else 0), DTYPES[t.dtype],
+                  t.dim(), ctypes.cast(shape, _i64p))
+
+
+def make_case(cand, ref, *, inputs=(), rtol, atol, tile=(64, 64), first_k=256,
+              keep: _Keep | None = None) -> tuple[Case, _Keep]:
+    keep = keep or _Keep()
+    c = Case()
+    c.cand = _tensor(cand, keep)
+    c.ref = _tensor(ref, keep)
+    if inputs:
+        arr = (Tensor * len(inputs))(*[_tensor(x, keep) for x in inputs])
+        keep.items.append(arr)
+        c.inputs = ctypes.cast(arr, ctypes.POINTER(Tensor))
+    c.n_inputs = len(inputs)
+    c.reserved = 0
+    c.rtol, c.atol = float(rtol), float(atol)
+    c.tile_rows, c.tile_cols = int(tile[0]), int(tile[1])
+    c.first_k = int(first_k)
+    keep.items.extend([cand, ref, *inputs])
+    return c, keep
+
+
+def _arr(ptr, n, dtype):
+    if n == 0:
+        return np.zeros(0, dtype)
+    return np.ctypeslib.as_array(ptr, shape=(n,)).astype(dtype, copy=True)
+
+
+def result_to_dict(r: Result) -> dict:
+    numel, mismatch = int(r.numel), int(r.mismatch)
+    gr, gc = int(r.grid_rows), int(r.grid_cols)
+    k = int(r.k_out)
+    return {
+        "pass": bool(r.pass_), "numel": numel, "rank": int(r.rank), "mismatch": mismatch,
+        "match_fraction": 1.0 if numel == 0 else (numel - mismatch) / numel,
+        "cand_nan": int(r.cand_nan), "cand_posinf": int(r.cand_posinf),
+        "cand_neginf": int(r.cand_neginf), "ref_nan": int(r.ref_nan),
+        "ref_posinf": int(r.ref_posinf), "ref_neginf": int(r.ref_neginf),
+        "n_finite_pairs": int(r.n_finite_pairs),
+        "max_abs": float(r.max_abs), "argmax_abs": int(r.argmax_abs),
+        "max_rel": float(r.max_rel), "argmax_rel": int(r.argmax_rel), "sse": float(r.sse),
+        "grid_rows": gr, "grid_cols": gc, "tile_rows": int(r.tile_rows),
+        "tile_cols": int(r.tile_cols),
+        "tile_hist": _arr(r.tile_hist, gr * gc, np.int64).reshape(gr, gc),
+        "row_prof": _arr(r.row_prof, int(r.tile_rows), np.int64),
+        "col_prof": _arr(r.col_prof, int(r.tile_cols), np.int64),
+        "k_out": k, "fk_index": _arr(r.fk_index, k, np.int64),
+        "fk_coords": _arr(r.fk_coords, k * int(r.rank), np.int64).reshape(k, int(r.rank)),
+        "fk_cand": _arr(r.fk_cand, k, np.float64), "fk_ref": _arr(r.fk_ref, k, np.float64),
+        "flags": int(r.flags), "input_eq": _arr(r.input_eq, int(r.n_inputs), np.int64),
+        "passthrough_input": int(r.passthrough_input),
+    }
+
+
+def _stream_handle(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def validate(cand: torch.Tensor, ref: torch.Tensor, *, inputs=(), rtol: float, atol: float,
+             tile=(64, 64), first_k: int = 256, stream=None) -> dict:
+    """Validate one candidate/reference pair on the GPU (nmv_validate)."""
+    lib = load()
+    case, keep = make_case(cand, ref, inputs=inputs, rtol=rtol, atol=atol, tile=tile,
+                           first_k=first_k)
+    out = ctypes.POINTER(Result)()
+    rc = lib.nmv_validate(ctypes.byref(case), _stream_handle(stream), ctypes.byref(out))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    try:
+        return result_to_dict(out[0])
+    finally:
+        lib.nmv_result_free(out)
+        del keep
+
+
+def validate_batch(cases, stream=None) -> dict:
+    """Validate many pairs in one call (nmv_validate_batch).  `cases` holds
+    dicts with keys cand, ref, rtol, atol, tile, first_k and optional inputs."""
+    lib = load()
+    keep = _Keep()
+    structs = [make_case(c["cand"], c["ref"], inputs=c.get("inputs", ()), rtol=c["rtol"],
+                         atol=c["atol"], tile=c["tile"], first_k=c["first_k"], keep=keep)[0]
+               for c in cases]
+    arr = (Case * max(len(structs), 1))(*structs)
+    out = ctypes.POINTER(Result)()
+    rc = lib.nmv_validate_batch(arr, len(structs), _stream_handle(stream), ctypes.byref(out))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    try:
+        results = [result_to_dict(out[i]) for i in range(len(structs))]
+    finally:
+        if out:
+            lib.nmv_result_free(out)
+    return {"results": results, "n_pass": sum(int(r["pass"]) for r in results)}
+
+
+class Prepared:
+    """A case marshalled once and called many times (benchmark loops): each
+    call() runs nmv_validate / nmv_validate_batch and frees the result."""
+
+    def __init__(self, cases, stream=None):
+        self.lib = load()
+        self.keep = _Keep()
+        self.structs = [make_case(c["cand"], c["ref"], inputs=c.get("inputs", ()),
+                                  rtol=c["rtol"], atol=c["atol"], tile=c["tile"],
+                                  first_k=c["first_k"], keep=self.keep)[0] for c in cases]
+        self.arr = (Case * len(self.structs))(*self.structs)
+        self.n = len(self.structs)
+        self.stream = _stream_handle(stream)
+        self.out = ctypes.POINTER(Result)()
+
+    def call(self) -> int:
+        if self.n == 1:
+            rc = self.lib.nmv_validate(self.arr, self.stream, ctypes.byref(self.out))
+        else:
+            rc = self.lib.nmv_validate_batch(self.arr, self.n, self.stream, ctypes.byref(self.out))
+        if rc != NMV_OK:
+            _raise(self.lib, rc)
+        self.lib.nmv_result_free(self.out)
+        return rc
+
+    def call_dicts(self) -> list:
+        if self.n == 1:
+            rc = self.lib.nmv_validate(self.arr, self.stream, ctypes.byref(self.out))
+        else:
+            rc = self.lib.nmv_validate_batch(self.arr, self.n, self.stream, ctypes.byref(self.out))
+        if rc != NMV_OK:
+            _raise(self.lib, rc)
+        try:
+            return [result_to_dict(self.out[i]) for i in range(self.n)]
+        finally:
+            self.lib.nmv_result_free(self.out)

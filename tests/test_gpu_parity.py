@@ -1,0 +1,154 @@
+"""GPU parity: the CUDA path (through the C ABI) against the oracle, element
+by element on the same seeded inputs."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from _golden import check, fixture_files, load
+from _parity import assert_same
+from paper_2608_02712_gb300 import validate, validate_batch, workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _gpu(case):
+    dev = lambda t: t.cuda()
+    return validate(dev(case["cand"]), dev(case["ref"]),
+                    inputs=[dev(x) for x in case["inputs"]], rtol=case["rtol"],
+                    atol=case["atol"], tile=case["tile"], first_k=case["first_k"])
+
+
+def _oracle(case):
+    cpu = lambda t: t.cpu()
+    return oracle.validate(cpu(case["cand"]), cpu(case["ref"]),
+                           inputs=[cpu(x) for x in case["inputs"]], rtol=case["rtol"],
+                           atol=case["atol"], tile=case["tile"], first_k=case["first_k"])
+
+
+@pytest.mark.parametrize("path", fixture_files(), ids=lambda p: p.rsplit("/", 1)[-1])
+def test_golden_fixtures_on_gpu(path):
+    case, expect = load(path)
+    check(_gpu(case), expect)
+
+
+@pytest.mark.parametrize("seed", range(300))
+def test_fuzz_parity(seed):
+    case = workloads.fuzz(seed)
+    assert_same(_gpu(case), _oracle(case), case["name"])
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_fuzz_parity_unaligned(seed):
+    """Views that start one element into their buffer (no 16-byte alignment)."""
+    case = workloads.fuzz(1000 + seed)
+    shift = lambda t: torch.cat([t.reshape(-1)[:1], t.reshape(-1)]).cuda()[1:].view(t.shape)
+    c, r = shift(case["cand"]), shift(case["ref"])
+    xs = [shift(x) for x in case["inputs"]]
+    got = validate(c, r, inputs=xs, rtol=case["rtol"], atol=case["atol"], tile=case["tile"],
+                   first_k=case["first_k"])
+    assert_same(got, _oracle(case), case["name"])
+
+
+def test_c1_full():
+    case = workloads.c1(device="cuda")
+    assert_same(_gpu(case), _oracle(case), case["name"])
+
+
+@pytest.mark.parametrize("shape", [(1, 1024, 4096), (3, 1000, 4095), (8, 4096, 4096)])
+def test_c2_parity(shape):
+    case = workloads.c2(device="cuda", shape=shape)
+    assert_same(_gpu(case), _oracle(case), case["name"])
+
+
+@pytest.mark.parametrize("numel", [(1 << 20) + 77, 1 << 28])
+def test_c4_parity(numel):
+    case = workloads.c4(device="cuda", numel=numel)
+    assert_same(_gpu(case), _oracle(case), case["name"])
+
+
+@pytest.mark.parametrize("shape", [(256, 1024), (1024, 4096 + 3)])
+def test_c5_parity_reduced(shape):
+    case = workloads.c5(device="cuda", shape=shape, first_k=4096)
+    assert_same(_gpu(case), _oracle(case), case["name"])
+
+
+def test_c3_batch_parity_and_equal_to_single_calls():
+    cases = workloads.c3(device="cuda", count=96, cap=1 << 20)
+    got = validate_batch(cases)
+    for c, g in zip(cases, got["results"]):
+        assert_same(g, _oracle(c), c["name"])
+        single = _gpu(c)
+        assert_same(single, g, c["name"] + " (single vs batch)")
+    assert got["n_pass"] == sum(int(_oracle(c)["pass"]) for c in cases)
+
+
+def test_mixed_dtype_batch_with_inputs_and_empty_cases():
+    cases = [workloads.fuzz(s) for s in range(60)]
+    cases = [dict(c, cand=c["cand"].cuda(), ref=c["ref"].cuda(),
+                  inputs=[x.cuda() for x in c["inputs"]]) for c in cases]
+    got = validate_batch(cases)
+    for c, g in zip(cases, got["results"]):
+        assert_same(g, _oracle(c), c["name"])
+
+
+def test_deterministic_bits():
+    case = workloads.c2(device="cuda", shape=(2, 2048, 4096))
+    a, b = _gpu(case), _gpu(case)
+    for k in a:
+        if isinstance(a[k], np.ndarray):
+            assert np.array_equal(a[k].view(np.uint8) if a[k].dtype.kind == "f" else a[k],
+                                  b[k].view(np.uint8) if b[k].dtype.kind == "f" else b[k]), k
+        elif isinstance(a[k], float):
+            assert np.float64(a[k]).tobytes() == np.float64(b[k]).tobytes(), k
+        else:
+            assert a[k] == b[k], k
+
+
+def test_first_k_overflowing_segment_lists():
+    """Dense mismatches: every segment list overflows, first-K needs re-reads."""
+    g = torch.Generator(device="cuda").manual_seed(5)
+    ref = torch.randn(3, 777, 1031, generator=g, device="cuda")
+    cand = ref + 1.0
+    for k in (1, 127, 128, 129, 5000, 200000):
+        got = validate(cand, ref, rtol=1e-3, atol=1e-5, tile=(32, 64), first_k=k)
+        want = oracle.validate(cand.cpu(), ref.cpu(), rtol=1e-3, atol=1e-5, tile=(32, 64),
+                               first_k=k)
+        assert_same(got, want, "dense k=%d" % k)
+
+
+def test_exact_tolerance_boundaries_on_gpu():
+    """Elements sitting exactly on, and one ulp either side of, the fp64
+    threshold: the fp32 pre-filter must hand them to the fp64 path."""
+    g = torch.Generator().manual_seed(9)
+    r = torch.randn(4096, generator=g, dtype=torch.float64).to(torch.float32)
+    rtol, atol = 1e-3, 1e-5
+    thr = atol + rtol * r.double().abs()
+    c = (r.double() + thr).to(torch.float32)
+    cases = [c, torch.nextafter(c, torch.full_like(c, float("inf"))),
+             torch.nextafter(c, torch.full_like(c, -float("inf")))]
+    for cc in cases:
+        got = validate(cc.cuda(), r.cuda(), rtol=rtol, atol=atol, tile=(1, 64), first_k=4096)
+        want = oracle.validate(cc, r, rtol=rtol, atol=atol, tile=(1, 64), first_k=4096)
+        assert_same(got, want, "boundary")
+
+
+def test_tiny_and_huge_values_sse():
+    vals = torch.tensor([1e-30, -3e-38, 1e-45, 2e30, -1e38, 3.3e38, 5e-20, 0.0] * 64,
+                        dtype=torch.float32)
+    r = vals
+    c = vals * 1.5
+    got = validate(c.cuda(), r.cuda(), rtol=0.1, atol=0.0, tile=(1, 8), first_k=16)
+    want = oracle.validate(c, r, rtol=0.1, atol=0.0, tile=(1, 8), first_k=16)
+    assert_same(got, want, "extremes")
+    small = torch.tensor([1e-42, 2e-42, 3e-41] * 100, dtype=torch.float32)
+    got = validate(small.cuda() * 2, small.cuda(), rtol=0.0, atol=0.0, tile=(1, 1), first_k=5)
+    want = oracle.validate(small * 2, small, rtol=0.0, atol=0.0, tile=(1, 1), first_k=5)
+    assert_same(got, want, "subnormal sse")
+
+
+def test_exact_equal_tensors_fast():
+    x = torch.randn(1 << 22, device="cuda")
+    got = validate(x, x.clone(), rtol=0, atol=0, tile=(1, 4096), first_k=8)
+    assert got["pass"] and got["mismatch"] == 0 and got["max_abs"] == 0.0
+    assert got["argmax_abs"] == 0 and got["argmax_rel"] == int((x != 0).nonzero()[0])
