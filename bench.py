@@ -1,0 +1,391 @@
+#!/usr/bin/env python
+"""Benchmark: validation throughput on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config c1|c2|c3|c4|c5]
+
+A step is one nmv_validate call (nmv_validate_batch for c3) on one seeded
+synthetic workload resident in HBM; the default workload is the bf16
+[8, 4096, 4096] candidate/reference pair with planted tile faults.  The metric
+is GB/s of candidate + reference bytes read.  Prints ONE JSON line on rank 0.
+
+Under torchrun (N > 1) every rank validates its own replica (independent
+problems, no collective on the data path); the timed region is bracketed by
+a barrier and a device synchronize on every rank and the slowest rank's time
+is used.  ``--impl reference`` times the CPU oracle (the reference arm: one
+host core, a bounded sample of the same workload per step).
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "validation GB/s (cand+ref bytes read) and % of GB300 HBM peak, 1 GPU"
+L2_BYTES = 129 * 1024 * 1024
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="c2", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--c2-batch", type=int, default=8,
+                    help="leading dimension of the c2 workload (8 = full size); smaller "
+                         "values give the small cases used for profiler captures")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------- workloads
+def make_cases(config: str, device, seed_shift: int = 0, c2_batch: int = 8):
+    from paper_2608_02712_gb300 import workloads as W
+    if config == "c1":
+        return [W.c1(seed=0 + seed_shift, device=device)]
+    if config == "c2":
+        return [W.c2(seed=1 + seed_shift, device=device, shape=(c2_batch, 4096, 4096))]
+    if config == "c3":
+        return W.c3(seed=2 + seed_shift, device=device)
+    if config == "c4":
+        return [W.c4(seed=3 + seed_shift, device=device)]
+    return [W.c5(seed=4 + seed_shift, device=device)]
+
+
+def case_bytes(c, with_inputs=False):
+    b = c["cand"].numel() * c["cand"].element_size() * 2
+    if with_inputs:
+        b += sum(x.numel() * x.element_size() for x in c["inputs"])
+    return b
+
+
+def describe(config, cases):
+    c = cases[0]
+    if config == "c3":
+        name = "c3_batch%d_rank1-5_fp32/fp16/bf16" % len(cases)
+        return {"workload": name, "cases": len(cases),
+                "elements": int(sum(x["cand"].numel() for x in cases)),
+                "tolerance": "torch.testing defaults per dtype", "tile": [64, 64],
+                "first_k": 256}
+    return {"workload": c["name"], "shape": list(c["cand"].shape),
+            "dtype_in": str(c["cand"].dtype).split(".")[-1], "rtol": c["rtol"],
+            "atol": c["atol"], "tile": list(c["tile"]), "first_k": c["first_k"],
+            "inputs": len(c["inputs"])}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """Samples SM clock and throttle reasons through NVML while running."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, device_index: int):
+        self.samples, self.reasons, self.max_mhz = [], set(), None
+        self._stop = threading.Event()
+        self._nvml = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                return
+            handle = ctypes.c_void_p()
+            import torch
+            bus = None
+            try:
+                p = torch.cuda.get_device_properties(device_index)
+                bus = "%08x:%02x:%02x.0" % (p.pci_domain_id, p.pci_bus_id, p.pci_device_id)
+            except Exception:
+                bus = None
+            ok = bus is not None and nv.nvmlDeviceGetHandleByPciBusId_v2(
+                bus.encode(), ctypes.byref(handle)) == 0
+            if not ok and nv.nvmlDeviceGetHandleByIndex_v2(device_index, ctypes.byref(handle)) != 0:
+                return
+            self._nv, self._h = nv, handle
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(handle, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = mx.value
+            self._nvml = True
+        except OSError:
+            self._nvml = None
+
+    def sample(self):
+        if not self._nvml:
+            return
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        if self._nv.nvmlDeviceGetClockInfo(self._h, 1, ctypes.byref(clk)) == 0:
+            self.samples.append(clk.value)
+        if self._nv.nvmlDeviceGetCurrentClocksEventReasons(self._h, ctypes.byref(rs)) == 0:
+            for bit, name in self.REASONS.items():
+                if rs.value & bit:
+                    self.reasons.add(name)
+
+    def _run(self):
+        while not self._stop.is_set():
+            self.sample()
+            time.sleep(0.02)
+
+    def __enter__(self):
+        self.sample()
+        self._t = threading.Thread(target=self._run, daemon=True)
+        self._t.start()
+        return self
+
+    def __exit__(self, *a):
+        self._stop.set()
+        self._t.join()
+        self.sample()
+
+    def report(self):
+        if not self._nvml:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvml unavailable"]}
+        return {"sm_mhz": statistics.median(self.samples) if self.samples else None,
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(self.reasons),
+                "samples": len(self.samples)}
+
+
+# ---------------------------------------------------------------- peaks
+def measured_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs)"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def profiled_traffic(config: str):
+    """DRAM bytes per scan launch from the committed ncu summary, when it was
+    taken on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "scan_kernel_%s_traffic.txt" % config)
+    src = os.path.join(ROOT, "paper_2608_02712_gb300", "csrc", "nmv_scan.cuh")
+    try:
+        info = {}
+        for line in open(path):
+            if ":" in line and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                info[k.strip()] = v.strip()
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        if info.get("kernel_source_sha256") != digest:
+            return None
+        return int(info["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+# ------------------------------------------------------------ reference
+def oracle_step_time(cases, rows):
+    """Run the oracle on the first `rows` rows of the [M, N] view of case 0."""
+    import oracle
+    c = cases[0]
+    n = c["cand"].shape[-1]
+    cv = c["cand"].reshape(-1, n)[:rows]
+    rv = c["ref"].reshape(-1, n)[:rows]
+    t0 = time.perf_counter()
+    oracle.validate(cv, rv, rtol=c["rtol"], atol=c["atol"], tile=c["tile"],
+                    first_k=c["first_k"])
+    return time.perf_counter() - t0, cv.numel() * cv.element_size() * 2
+
+
+def host_copy(cases):
+    return [dict(c, cand=c["cand"].cpu(), ref=c["ref"].cpu(),
+                 inputs=[x.cpu() for x in c["inputs"]]) for c in cases]
+
+
+def cpu_baseline(cases_host, budget_s=12.0):
+    """The oracle as it stands, on one host core, on a bounded row sample."""
+    n_rows = cases_host[0]["cand"].reshape(-1, cases_host[0]["cand"].shape[-1]).shape[0]
+    rows = min(n_rows, 256)
+    t, b = oracle_step_time(cases_host, rows)
+    rows = int(min(n_rows, max(rows, rows * budget_s / max(t, 1e-6))))
+    t, b = oracle_step_time(cases_host, rows)
+    return {"value": b / t / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": "first %d rows of the [M, N] view (%d bytes of cand+ref), one pass, "
+                      "%.1f s" % (rows, b, t)}
+
+
+def run_reference(args, rank, world):
+    import torch
+    if rank != 0:
+        return None
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    cases = host_copy(make_cases(args.config if args.config != "c3" else "c2", dev,
+                                 c2_batch=args.c2_batch))
+    n_rows = cases[0]["cand"].reshape(-1, cases[0]["cand"].shape[-1]).shape[0]
+    t, _ = oracle_step_time(cases, 64)
+    per_step = 150.0 / max(1, args.steps + args.warmup)
+    rows = int(min(n_rows, max(1, 64 * per_step / max(t, 1e-6))))
+    for _ in range(args.warmup):
+        oracle_step_time(cases, rows)
+    times, nbytes = [], 0
+    for _ in range(args.steps):
+        dt, nbytes = oracle_step_time(cases, rows)
+        times.append(dt)
+    total = sum(times)
+    value = nbytes * args.steps / total / 1e9
+    sample = "first %d rows of the [M, N] view per step (%d bytes of cand+ref)" % (rows, nbytes)
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": describe(args.config, cases),
+        "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+# ------------------------------------------------------------------ ours
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    import paper_2608_02712_gb300 as nmv
+    from paper_2608_02712_gb300 import nmv as nmvmod
+
+    torch.cuda.set_device(local_rank)
+    cases = make_cases(args.config, "cuda", seed_shift=0, c2_batch=args.c2_batch)
+    torch.cuda.synchronize()
+    nbytes = sum(case_bytes(c) for c in cases)
+    algo_bytes = sum(case_bytes(c, with_inputs=True) for c in cases)
+    stream = torch.cuda.current_stream()
+    prep = nmv.Prepared(cases, stream=stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    for _ in range(max(3, args.warmup)):
+        prep.call()
+    nmvmod.profile_enable(True)
+    scan_ms, launches = [], 0
+    sampler = ClockSampler(local_rank)
+    barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with sampler:
+        ev0.record(stream)
+        for _ in range(args.steps):
+            prep.call()
+            pr = nmvmod.profile_last()
+            scan_ms.append(pr["scan_ms"])
+            launches += pr["kernel_launches"]
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    nmvmod.profile_enable(False)
+    ms_per_step = elapsed_ms / args.steps
+    value = world * nbytes / (ms_per_step * 1e-3) / 1e9
+
+    # e2e: pinned host buffers -> device copies -> validate -> results back
+    host = [dict(c, cand=c["cand"].cpu().pin_memory(), ref=c["ref"].cpu().pin_memory(),
+                 inputs=[x.cpu().pin_memory() for x in c["inputs"]]) for c in cases]
+    dev_bufs = [dict(c, cand=torch.empty_like(c["cand"]), ref=torch.empty_like(c["ref"]),
+                     inputs=[torch.empty_like(x) for x in c["inputs"]]) for c in cases]
+    prep2 = nmv.Prepared(dev_bufs, stream=stream)
+    copied = sum(case_bytes(c, with_inputs=True) for c in cases)
+
+    def e2e_step():
+        for h, d in zip(host, dev_bufs):
+            d["cand"].copy_(h["cand"], non_blocking=True)
+            d["ref"].copy_(h["ref"], non_blocking=True)
+            for hx, dx in zip(h["inputs"], d["inputs"]):
+                dx.copy_(hx, non_blocking=True)
+        prep2.call()
+
+    for _ in range(2):
+        e2e_step()
+    nmvmod.profile_enable(True)
+    e2e_step()
+    pr_e2e = nmvmod.profile_last()
+    lib_h2d, lib_d2h = pr_e2e["h2d_bytes"], pr_e2e["d2h_bytes"]
+    nmvmod.profile_enable(False)
+    ke = max(1, min(args.e2e_steps, args.steps))
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(ke):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / ke
+    if world > 1:
+        t = torch.tensor([e2e_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    if rank != 0:
+        return None
+    peak, peak_src = measured_peak()
+    scan_mean = statistics.fmean(scan_ms)
+    achieved = algo_bytes / (scan_mean * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f32+f64", "data": "synthetic",
+        "config": dict(describe(args.config, cases),
+                       l2="inputs (%d B) larger than the %d B L2; no flush between steps"
+                          % (algo_bytes, L2_BYTES) if algo_bytes > L2_BYTES else
+                          "inputs smaller than L2 (cache-warm)",
+                       parallelism="replicas" if world > 1 else "1 GPU",
+                       pct_of_hbm_peak=100.0 * value / world / peak),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": profiled_traffic(args.config),
+                     "kernel": "scan_kernel", "peak_source": peak_src,
+                     "algorithmic_bytes_per_launch": algo_bytes,
+                     "scan_ms_mean": scan_mean, "scan_ms_min": min(scan_ms),
+                     "slow_steps": pr["slow_steps"], "light_steps": pr["light_steps"],
+                     "exact_abs": pr["exact_abs"],
+                     "exact_rel": pr["exact_rel"], "exact_pred": pr["exact_pred"]},
+        "e2e": {"value": world * nbytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+                "h2d_bytes_per_step": copied + lib_h2d, "d2h_bytes_per_step": lib_d2h,
+                "ms_per_step": e2e_ms},
+        "gpu_launches": launches,
+        "clocks": sampler.report(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(host_copy(cases))
+    return line
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        if world > 1:
+            import torch
+            import torch.distributed as dist
+            torch.cuda.set_device(local_rank)
+            dist.init_process_group("nccl")
+        line = run_ours(args, rank, world, local_rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+    if line is not None:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

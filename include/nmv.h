@@ -167,6 +167,31 @@ const char *nmv_status_string(int status);
 /* Text of the last failure on the calling thread ("" if none). */
 const char *nmv_last_error(void);
 
+/* Launch profile, for measuring the kernels against their roofline (the
+ * paper's forensics "compiles and profiles" a kernel, Section 4; this is the
+ * library's own profile).  While enabled (on != 0), every call records CUDA
+ * events on its stream around its scan-kernel launches and around its
+ * finalize launch, and counts the scan pass's exact-path work.
+ * nmv_profile_last() fills *out for the last successful call on any thread;
+ * it returns NMV_EINVAL if profiling was off for that call or out is NULL. */
+typedef struct nmv_profile {
+    double scan_ms;            /* scan-kernel launches, stream time          */
+    double finalize_ms;        /* finalize launch, stream time               */
+    int64_t kernel_launches;   /* kernels the call launched                  */
+    int64_t h2d_bytes;         /* bytes the library copied host to device    */
+    int64_t d2h_bytes;         /* bytes the library copied device to host    */
+    int64_t slow_steps;        /* warp steps that took the exact path        */
+    int64_t light_steps;       /* warp steps that only updated the maxima    */
+    int64_t exact_abs;         /* fp64 evaluations of a max |d| candidate    */
+    int64_t exact_rel;         /* fp64 evaluations of a max |d|/|r| candidate */
+    int64_t exact_pred;        /* fp64 evaluations of the predicate          */
+    int64_t slow_cycles;       /* SM clock cycles warps spent in exact steps  */
+    int64_t light_cycles;      /* SM clock cycles warps spent in light steps  */
+} nmv_profile;
+
+void nmv_profile_enable(int on);
+int nmv_profile_last(nmv_profile *out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <cstddef>
 #include <cstdint>
 #include <cstdio>
 #include <cstdlib>
@@ -22,11 +23,13 @@ struct ScanOps {
   static int occupancy(int nin, size_t smem);
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
-                            Partial *partials, int32_t *seg_count, uint32_t *seg_list, uint8_t *out,
-                            uint32_t *g_thr);
+                            Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
+                            unsigned long long *stats);
 };
-cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *,
-                            const uint32_t *, uint8_t *, int, cudaStream_t);
+cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
+                            int, cudaStream_t);
+cudaError_t launch_sse64(const CaseDesc *cd, double *part, double *dst, cudaStream_t st);
+constexpr int kSseBlocksHost = 1024;  // scratch doubles of launch_sse64
 
 cudaError_t scan_prepare(int dt, int nin, size_t smem) {
   switch (dt) {
@@ -48,21 +51,21 @@ int scan_occupancy(int dt, int nin, size_t smem) {
 
 cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                         const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
-                        Partial *partials, int32_t *seg_count, uint32_t *seg_list, uint8_t *out,
-                        uint32_t *g_thr) {
+                        Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
+                        unsigned long long *stats) {
   switch (dt) {
     case NMV_F32:
       return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, seg_count, seg_list, out, g_thr);
+                                      partials, batch_count, out, g_thr, stats);
     case NMV_F16:
       return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, seg_count, seg_list, out, g_thr);
+                                      partials, batch_count, out, g_thr, stats);
     case NMV_BF16:
       return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                       partials, seg_count, seg_list, out, g_thr);
+                                       partials, batch_count, out, g_thr, stats);
     default:
       return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, seg_count, seg_list, out, g_thr);
+                                      partials, batch_count, out, g_thr, stats);
   }
 }
 }  // namespace nmv
@@ -105,6 +108,19 @@ struct DeviceState {
 
 std::mutex g_mu;
 DeviceState g_dev[kMaxDevices];
+
+// Launch timing (nmv_profile_enable / nmv_profile_last), guarded by g_mu.
+struct Profile {
+  bool on = false;
+  bool valid = false;
+  nmv_profile last{};
+  cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+  int ev_dev = -1;
+} g_prof;
+
+// The packed results start with a call header holding the scan pass's
+// exact-path counters (filled when profiling is on).
+constexpr size_t kCallHeader = 256;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -522,21 +538,29 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   std::vector<int64_t> all_bp;
   all_pieces.reserve((size_t)np);
   all_bp.reserve((size_t)nbp);
-  size_t out_size = 0;
+  size_t out_size = kCallHeader;
   for (int64_t i = 0; i < n; ++i) {
     fill_desc(cases[i], geo[i], desc[i]);
     desc[i].out_off = (int64_t)out_size;
     out_size += geo[i].out_size;
-    desc[i].piece_begin = 0;
-    desc[i].piece_end = 0;
+    desc[i].piece_begin = desc[i].piece_end = 0;
+    desc[i].batch_begin = desc[i].batch_end = 0;
   }
+  int64_t n_batches = 0;
   for (Group &G : groups) {
     for (size_t k = 0; k < G.plan.pieces.size(); ++k) {
-      const Piece &p = G.plan.pieces[k];
+      Piece p = G.plan.pieces[k];
       const int64_t gid = G.piece_base + (int64_t)k;
       CaseDesc &d = desc[p.case_id];
-      if (d.piece_end == 0) d.piece_begin = gid;
+      p.batch_base = n_batches;
+      const int64_t nb = piece_batches(p.begin, p.end, G.dt);
+      if (d.piece_end == 0) {
+        d.piece_begin = gid;
+        d.batch_begin = n_batches;
+      }
       d.piece_end = gid + 1;
+      n_batches += nb;
+      d.batch_end = n_batches;
       all_pieces.push_back(p);
     }
     all_bp.insert(all_bp.end(), G.plan.block_piece.begin(), G.plan.block_piece.end());
@@ -548,11 +572,11 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   const size_t sz_bp = align_up(sizeof(int64_t) * std::max<int64_t>(nbp, 1), 256);
   const size_t table = sz_cases + sz_pieces + sz_bp;
   const size_t sz_part = align_up(sizeof(Partial) * std::max<int64_t>(np, 1), 256);
-  const size_t sz_segc = align_up(sizeof(int32_t) * kWarps * std::max<int64_t>(np, 1), 256);
-  const size_t sz_segl = align_up(sizeof(uint32_t) * kWarps * kFirstR * std::max<int64_t>(np, 1), 256);
+  const size_t sz_segc = align_up(sizeof(int32_t) * std::max<int64_t>(n_batches, 1), 256);
   const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n, 256);
-  const size_t o_part = table, o_segc = o_part + sz_part, o_segl = o_segc + sz_segc;
-  const size_t o_thr = o_segl + sz_segl, o_out = o_thr + sz_thr;
+  const size_t sz_sse = align_up(sizeof(double) * kSseBlocksHost, 256);
+  const size_t o_part = table, o_segc = o_part + sz_part;
+  const size_t o_sse = o_segc + sz_segc, o_thr = o_sse + sz_sse, o_out = o_thr + sz_thr;
   const size_t ws = o_out + out_size;
   rc = ensure_workspace(*S, ws, table + out_size);
   if (rc) return rc;
@@ -573,21 +597,74 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     cudaStreamSynchronize(st);
     return fail(NMV_ECUDA, "injected launch failure");
   }
+  const bool prof = g_prof.on;
+  unsigned long long *d_stats = prof ? (unsigned long long *)(W + o_out) : nullptr;
+  if (prof) {
+    if (g_prof.ev_dev != dev) {
+      for (cudaEvent_t &x : g_prof.ev) {
+        if (x) cudaEventDestroy(x);
+        x = nullptr;
+      }
+      for (cudaEvent_t &x : g_prof.ev) {
+        e = cudaEventCreate(&x);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+      }
+      g_prof.ev_dev = dev;
+    }
+    g_prof.valid = false;
+    cudaEventRecord(g_prof.ev[0], st);
+  }
   for (const Group &G : groups) {
     e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_bp + G.bp_base,
-                    G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc),
-                    (uint32_t *)(W + o_segl), W + o_out, (uint32_t *)(W + o_thr));
+                    G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out,
+                    (uint32_t *)(W + o_thr), d_stats);
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
+  if (prof) cudaEventRecord(g_prof.ev[1], st);
   e = launch_finalize(d_cases, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc),
-                      (const uint32_t *)(W + o_segl), W + o_out, (int)n, st);
+                      W + o_out, (int)n, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  if (prof) cudaEventRecord(g_prof.ev[2], st);
   uint8_t *HO = H + table;
   e = cudaMemcpyAsync(HO, W + o_out, out_size, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (results)");
   e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   if (injected("d2h")) return fail(NMV_ECUDA, "injected copy-back failure");
+  // Cases whose differences are all tiny (max |d| < 2^-38): the fp32 squares
+  // of the scan pass may have lost terms, so their SSE is recomputed in fp64.
+  for (int64_t i = 0; i < n; ++i) {
+    OutHeader *oh = (OutHeader *)(HO + desc[i].out_off);
+    if (oh->max_abs > 0.0 && oh->max_abs < 0x1p-38) {
+      double *dst = (double *)(W + o_out + desc[i].out_off + offsetof(OutHeader, sse));
+      e = launch_sse64(d_cases + i, (double *)(W + o_sse), dst, st);
+      if (e != cudaSuccess) return cuda_fail(e, "fp64 SSE launch");
+      e = cudaMemcpyAsync(&oh->sse, dst, sizeof(double), cudaMemcpyDeviceToHost, st);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fp64 SSE)");
+      e = cudaStreamSynchronize(st);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (fp64 SSE)");
+    }
+  }
+  if (prof) {
+    float a = 0.f, b = 0.f;
+    cudaEventElapsedTime(&a, g_prof.ev[0], g_prof.ev[1]);
+    cudaEventElapsedTime(&b, g_prof.ev[1], g_prof.ev[2]);
+    const unsigned long long *st4 = (const unsigned long long *)HO;  // scan counters
+    nmv_profile &P = g_prof.last;
+    P.scan_ms = a;
+    P.finalize_ms = b;
+    P.kernel_launches = (int64_t)groups.size() + 1;
+    P.h2d_bytes = (int64_t)table;
+    P.d2h_bytes = (int64_t)out_size;
+    P.slow_steps = (int64_t)st4[0];
+    P.light_steps = (int64_t)st4[4];
+    P.exact_abs = (int64_t)st4[1];
+    P.exact_rel = (int64_t)st4[2];
+    P.exact_pred = (int64_t)st4[3];
+    P.slow_cycles = (int64_t)st4[5];
+    P.light_cycles = (int64_t)st4[6];
+    g_prof.valid = true;
+  }
 
   // ---- result arena
   size_t bytes = align_up(sizeof(nmv_result) * n, 16);
@@ -702,5 +779,19 @@ const char *nmv_status_string(int status) {
 }
 
 const char *nmv_last_error(void) { return g_err.c_str(); }
+
+void nmv_profile_enable(int on) {
+  std::lock_guard<std::mutex> lock(g_mu);
+  g_prof.on = on != 0;
+  g_prof.valid = false;
+}
+
+int nmv_profile_last(nmv_profile *out) {
+  std::lock_guard<std::mutex> lock(g_mu);
+  if (!out) return fail(NMV_EINVAL, "NULL output pointer");
+  if (!g_prof.valid) return fail(NMV_EINVAL, "no profiled call");
+  *out = g_prof.last;
+  return NMV_OK;
+}
 
 }  // extern "C"

@@ -1,7 +1,9 @@
 // nmv_finalize.cu -- one block per case: reduce the piece partials of the
-// scan pass in piece order (deterministic), derive the degenerate-output
-// flags, and write the first-K mismatch records: copied from the per-segment
-// offset lists, or found by re-reading a segment whose list overflowed.
+// scan pass (fixed order, so the result is bit-identical run to run), derive
+// the degenerate-output flags, and write the first-K mismatch records:
+// copied from the per-segment offset lists, or found by re-reading a segment
+// whose list overflowed.  Also the fp64 SSE re-pass for cases whose
+// differences are all tiny (see nmv_scan.cuh).
 #include "nmv_scan.cuh"
 
 namespace nmv {
@@ -19,22 +21,42 @@ __device__ __forceinline__ double widen_any(uint32_t b, int dt) {
   }
 }
 
-// Exclusive block-wide prefix sum of v; *total = the block's sum.
-__device__ __forceinline__ int block_excl_scan(int v, int *total, int *sh /*[kFinThreads/32 + 1]*/) {
+// The predicate with the scan pass's fp32 pre-filter (same decision).
+template <int DT>
+__device__ __forceinline__ bool pass_elem(const CaseDesc &cd, uint32_t cb, uint32_t rb) {
+  const float cf = to_f32<DT>(cb), rf = to_f32<DT>(rb);
+  if constexpr (Tr<DT>::kInt) {
+    if (cb == rb) return true;
+    const long long d = (long long)(int32_t)cb - (long long)(int32_t)rb;
+    const float as = fabsf(__ll2float_rn(d)), ar = fabsf(rf);
+    if (as <= __fmaf_rz(cd.lo_r, ar, cd.lo_a)) return true;
+    if (as > __fmaf_ru(cd.hi_r, ar, cd.hi_a)) return false;
+  } else {
+    if (cf == rf) return true;
+    if (!(isfinite(cf) && isfinite(rf))) return false;
+    const float as = fabsf(__fsub_rn(cf, rf)), ar = fabsf(rf);
+    if (as <= __fmaf_rz(cd.lo_r, ar, cd.lo_a)) return true;
+    if (as > __fmaf_ru(cd.hi_r, ar, cd.hi_a)) return false;
+  }
+  return pass64(to_f64<DT>(cb), to_f64<DT>(rb), cd.rtol, cd.atol);
+}
+
+// Exclusive block-wide prefix sum of a 64-bit v; *total = the block's sum.
+__device__ __forceinline__ int64_t block_excl_scan64(int64_t v, int64_t *total, int64_t *sh) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int incl = v;
+  int64_t incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    const int64_t t = __shfl_up_sync(0xffffffffu, incl, o);
     if (lane >= o) incl += t;
   }
   __syncthreads();
   if (lane == 31) sh[warp] = incl;
   __syncthreads();
   if (threadIdx.x == 0) {
-    int acc = 0;
+    int64_t acc = 0;
     for (int w = 0; w < kFinThreads / 32; ++w) {
-      const int t = sh[w];
+      const int64_t t = sh[w];
       sh[w] = acc;
       acc += t;
     }
@@ -54,81 +76,135 @@ __device__ void write_record(const CaseDesc &cd, uint8_t *o, int64_t pos, int64_
   fk_r[pos] = widen_any(ld_elem(cd.ref, idx, cd.dtype), cd.dtype);
 }
 
-// Re-read segment [lo, hi) and write its first `needed` mismatches at
-// record positions pos0, pos0 + 1, ...  (the whole block, E elements per
-// thread, block-wide ordered compaction).
-__device__ void reread_segment(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t hi, int64_t pos0,
-                               int64_t needed, int *sh) {
+// Re-read elements [lo, hi) with one warp and write the first `needed`
+// mismatches at record positions pos0, pos0 + 1, ...  (E consecutive
+// elements per lane, warp-wide ordered compaction).
+template <int DT>
+__device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t hi, int64_t pos0,
+                            int64_t needed) {
   constexpr int E = 8;
+  constexpr int EB = Tr<DT>::EB;
+  const int lane = threadIdx.x & 31;
   int64_t found = 0;
-  for (int64_t base = lo; base < hi && found < needed; base += (int64_t)kFinThreads * E) {
-    const int64_t i0 = base + (int64_t)threadIdx.x * E;
+  for (int64_t base = lo; base < hi && found < needed; base += 32 * E) {
+    const int64_t i0 = base + (int64_t)lane * E;
     uint32_t mask = 0;
+#pragma unroll
     for (int k = 0; k < E; ++k) {
       const int64_t i = i0 + k;
-      if (i < hi) {
-        const double c = widen_any(ld_elem(cd.cand, i, cd.dtype), cd.dtype);
-        const double r = widen_any(ld_elem(cd.ref, i, cd.dtype), cd.dtype);
-        if (!pass64(c, r, cd.rtol, cd.atol)) mask |= 1u << k;
-      }
+      if (i < hi && !pass_elem<DT>(cd, ld_one<EB>(cd.cand, i), ld_one<EB>(cd.ref, i))) mask |= 1u << k;
     }
-    int total;
-    const int excl = block_excl_scan(__popc(mask), &total, sh);
-    int64_t pos = found + excl;
+    const int cnt = __popc(mask);
+    int incl = cnt;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, d);
+      if (lane >= d) incl += t;
+    }
+    int64_t pos = found + incl - cnt;
     while (mask) {
       const int k = __ffs(mask) - 1;
       mask &= mask - 1;
       if (pos < needed) write_record(cd, o, pos0 + pos, i0 + k);
       ++pos;
     }
-    found += total;
+    found += __shfl_sync(0xffffffffu, incl, 31);
   }
+}
+
+// Element range of global batch g of a case (its pieces are ordered by
+// batch_base).
+__device__ __forceinline__ void batch_range(const CaseDesc &cd, const Piece *pieces, int64_t g, int64_t *lo,
+                                            int64_t *hi) {
+  int64_t a = cd.piece_begin, b = cd.piece_end - 1;
+  while (a < b) {
+    const int64_t mid = (a + b + 1) / 2;
+    if (pieces[mid].batch_base <= g) a = mid;
+    else b = mid - 1;
+  }
+  const Piece &pc = pieces[a];
+  const int64_t be = batch_elems(cd.dtype);
+  *lo = pc.begin + (g - pc.batch_base) * be;
+  *hi = *lo + be < pc.end ? *lo + be : pc.end;
+}
+
+struct Red {
+  int64_t cnt[8];
+  Best ba, br;
+  double sse;
+  uint32_t cacc, racc;
+  int64_t eq[NMV_MAX_INPUTS];
+};
+
+__device__ __forceinline__ void red_add(Red &a, const Red &b) {
+  for (int k = 0; k < 8; ++k) a.cnt[k] += b.cnt[k];
+  best_offer(a.ba, b.ba.v, b.ba.i);
+  best_offer(a.br, b.br.v, b.br.i);
+  a.sse = __dadd_rn(a.sse, b.sse);
+  a.cacc |= b.cacc;
+  a.racc |= b.racc;
+  for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] += b.eq[j];
 }
 
 __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *__restrict__ cases,
                                                                const Piece *__restrict__ pieces,
                                                                const Partial *__restrict__ partials,
-                                                               const int32_t *__restrict__ seg_count,
-                                                               const uint32_t *__restrict__ seg_list,
+                                                               const int32_t *__restrict__ batch_count,
                                                                uint8_t *out) {
   const CaseDesc &cd = cases[blockIdx.x];
   uint8_t *o = out + cd.out_off;
   OutHeader *H = (OutHeader *)o;
-  __shared__ int sh_scan[kFinThreads / 32 + 1];
+  __shared__ int64_t sh_scan[kFinThreads / 32 + 1];
   __shared__ int64_t sh_mism;
-  __shared__ int64_t sh_re[kFinThreads][3];
-  __shared__ int sh_nre;
+  constexpr int kItems = 512;
+  __shared__ int64_t sh_item[kItems][3];
+  constexpr int kRed = 64;
+  __shared__ Red sh_red[kRed];
 
-  // ---- 1. reduce the partials of this case in piece order
-  if (threadIdx.x == 0) {
-    int64_t cnt[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    Best ba = {-1.0, INT64_MAX}, br = {-1.0, INT64_MAX};
-    double sse = 0.0;
-    uint32_t cacc = 0, racc = 0;
-    int64_t eq[NMV_MAX_INPUTS] = {0, 0, 0, 0, 0, 0, 0, 0};
-    for (int64_t p = cd.piece_begin; p < cd.piece_end; ++p) {
+  // ---- 1. reduce the partials: thread t < kRed takes pieces t, t + kRed,
+  // ... in order, then a fixed pairwise tree over those threads.
+  {
+    Red a;
+    for (int k = 0; k < 8; ++k) a.cnt[k] = 0;
+    a.ba = {-1.0, INT64_MAX};
+    a.br = {-1.0, INT64_MAX};
+    a.sse = 0.0;
+    a.cacc = a.racc = 0;
+    for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] = 0;
+    for (int64_t p = cd.piece_begin + threadIdx.x; threadIdx.x < kRed && p < cd.piece_end; p += kRed) {
       const Partial &Q = partials[p];
-      for (int k = 0; k < 8; ++k) cnt[k] += Q.cnt[k];
-      best_offer(ba, Q.best_abs, Q.arg_abs);
-      best_offer(br, Q.best_rel, Q.arg_rel);
-      sse = __dadd_rn(sse, Q.sse);
-      cacc |= Q.cacc;
-      racc |= Q.racc;
-      for (int j = 0; j < NMV_MAX_INPUTS; ++j) eq[j] += Q.eq[j];
+      Red b;
+      for (int k = 0; k < 8; ++k) b.cnt[k] = Q.cnt[k];
+      b.ba = {Q.best_abs, Q.arg_abs};
+      b.br = {Q.best_rel, Q.arg_rel};
+      b.sse = Q.sse;
+      b.cacc = Q.cacc;
+      b.racc = Q.racc;
+      for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = Q.eq[j];
+      red_add(a, b);
     }
-    for (int k = 0; k < 7; ++k) H->cnt[k] = cnt[k];
-    H->cnt[7] = cd.numel - cnt[7];  // n_finite_pairs
-    H->max_abs = ba.v < 0.0 ? 0.0 : ba.v;
-    H->argmax_abs = ba.v < 0.0 ? -1 : ba.i;
-    H->max_rel = br.v < 0.0 ? 0.0 : br.v;
-    H->argmax_rel = br.v < 0.0 ? -1 : br.i;
-    H->sse = sse;
-    H->k_out = cnt[0] < cd.first_k ? cnt[0] : cd.first_k;
+    if (threadIdx.x < kRed) sh_red[threadIdx.x] = a;
+    __syncthreads();
+    for (int half = kRed / 2; half > 0; half >>= 1) {
+      if (threadIdx.x < half) red_add(sh_red[threadIdx.x], sh_red[threadIdx.x + half]);
+      __syncthreads();
+    }
+  }
+  if (threadIdx.x == 0) {
+    const Red &a = sh_red[0];
+    for (int k = 0; k < 7; ++k) H->cnt[k] = a.cnt[k];
+    H->cnt[7] = cd.numel - a.cnt[7];  // n_finite_pairs
+    H->max_abs = a.ba.v < 0.0 ? 0.0 : a.ba.v;
+    H->argmax_abs = a.ba.v < 0.0 ? -1 : a.ba.i;
+    H->max_rel = a.br.v < 0.0 ? 0.0 : a.br.v;
+    H->argmax_rel = a.br.v < 0.0 ? -1 : a.br.i;
+    H->sse = a.sse;
+    H->k_out = a.cnt[0] < cd.first_k ? a.cnt[0] : cd.first_k;
     // degenerate-output flags
     uint32_t flags = 0;
     int32_t pt = -1;
     for (int j = 0; j < NMV_MAX_INPUTS; ++j) H->input_eq[j] = -1;
-    for (int j = 0; j < cd.n_elig; ++j) H->input_eq[cd.in_slot[j]] = eq[j];
+    for (int j = 0; j < cd.n_elig; ++j) H->input_eq[cd.in_slot[j]] = a.eq[j];
     const int64_t thr = cd.numel >= 100 ? (cd.numel + 99) / 100 : 1;
     for (int j = 0; j < cd.n_inputs; ++j) {
       if (H->input_eq[j] >= thr) {
@@ -140,8 +216,8 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
       const bool two = elem_bytes(cd.dtype) == 2;
       const uint32_t c0 = ld_elem(cd.cand, 0, cd.dtype), r0 = ld_elem(cd.ref, 0, cd.dtype);
       const uint32_t mag = cd.dtype == NMV_I32 ? 0xffffffffu : (two ? 0x7fffu : 0x7fffffffu);
-      const uint32_t cfold = two ? ((cacc | (cacc >> 16)) & 0xffffu) : cacc;
-      const uint32_t rfold = two ? ((racc | (racc >> 16)) & 0xffffu) : racc;
+      const uint32_t cfold = two ? ((a.cacc | (a.cacc >> 16)) & 0xffffu) : a.cacc;
+      const uint32_t rfold = two ? ((a.racc | (a.racc >> 16)) & 0xffffu) : a.racc;
       if ((c0 & mag) == 0 && (cfold & mag) == 0) flags |= NMV_FLAG_CAND_ALL_ZERO;
       if ((r0 & mag) == 0 && (rfold & mag) == 0) flags |= NMV_FLAG_REF_ALL_ZERO;
       if (cd.numel >= 2 && cfold == 0) flags |= NMV_FLAG_CAND_CONSTANT;
@@ -150,56 +226,118 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
     H->flags = flags;
     H->passthrough = pt;
     H->status = 0;
-    sh_mism = cnt[0];
+    sh_mism = a.cnt[0];
   }
   __syncthreads();
 
-  // ---- 2. first-K records, segment by segment in index order
+  // ---- 2. first-K records.  Thread t sums the counts of a contiguous
+  // chunk of the case's batches; a block scan places the chunks; every
+  // batch holding records below K becomes an item (batch, first record
+  // position, records wanted), and the warps re-read the items' batches.
   const int64_t K = cd.first_k;
   if (K == 0 || sh_mism == 0) return;
-  const int vec = vec_elems(cd.dtype);
-  const int64_t s0 = cd.piece_begin * kWarps, s1 = cd.piece_end * kWarps;
-  int64_t carry = 0;
-  for (int64_t sb = s0; sb < s1 && carry < K; sb += kFinThreads) {
-    const int64_t s = sb + threadIdx.x;
-    const int cnt = s < s1 ? seg_count[s] : 0;
-    int total;
-    const int excl = block_excl_scan(cnt, &total, sh_scan);
-    if (threadIdx.x == 0) sh_nre = 0;
-    __syncthreads();
-    const int64_t prefix = carry + excl;
-    if (cnt > 0 && prefix < K) {
-      const int64_t needed = (K - prefix) < cnt ? (K - prefix) : cnt;
-      const Piece &pc = pieces[s / kWarps];
-      int64_t lo, hi;
-      segment_range(pc.begin, pc.end, (int)(s % kWarps), vec, &lo, &hi);
-      if (needed <= kFirstR) {
-        for (int64_t j = 0; j < needed; ++j) write_record(cd, o, prefix + j, lo + seg_list[s * kFirstR + j]);
-      } else {
-        const int slot = atomicAdd(&sh_nre, 1);
-        sh_re[slot][0] = s;
-        sh_re[slot][1] = prefix;
-        sh_re[slot][2] = needed;
+  const int64_t B0 = cd.batch_begin, B1 = cd.batch_end;
+  const int64_t cs = (B1 - B0 + kFinThreads - 1) / kFinThreads;
+  const int64_t c0 = B0 + (int64_t)threadIdx.x * cs;
+  const int64_t c1 = c0 + cs < B1 ? c0 + cs : B1;
+  int64_t sum = 0;
+  for (int64_t g = c0; g < c1; ++g) sum += batch_count[g];
+  int64_t total;
+  const int64_t pre = block_excl_scan64(sum, &total, sh_scan);
+  int64_t mine = 0;
+  {
+    int64_t pos = pre;
+    for (int64_t g = c0; g < c1 && pos < K; ++g) {
+      const int64_t n = batch_count[g];
+      if (n > 0) {
+        ++mine;
+        pos += n;
+      }
+    }
+  }
+  int64_t n_items;
+  const int64_t ioff = block_excl_scan64(mine, &n_items, sh_scan);
+  const int warp = threadIdx.x >> 5;
+  for (int64_t r0 = 0; r0 < n_items; r0 += kItems) {
+    int64_t it = ioff, pos = pre;
+    for (int64_t g = c0; g < c1 && pos < K && it < r0 + kItems; ++g) {
+      const int64_t n = batch_count[g];
+      if (n > 0) {
+        if (it >= r0) {
+          sh_item[it - r0][0] = g;
+          sh_item[it - r0][1] = pos;
+          sh_item[it - r0][2] = n < K - pos ? n : K - pos;
+        }
+        ++it;
+        pos += n;
       }
     }
     __syncthreads();
-    const int nre = sh_nre;
-    for (int t = 0; t < nre; ++t) {
-      const int64_t s2 = sh_re[t][0];
-      const Piece &pc = pieces[s2 / kWarps];
+    const int64_t m = n_items - r0 < kItems ? n_items - r0 : kItems;
+    for (int64_t j = warp; j < m; j += kFinThreads / 32) {
       int64_t lo, hi;
-      segment_range(pc.begin, pc.end, (int)(s2 % kWarps), vec, &lo, &hi);
-      reread_segment(cd, o, lo, hi, sh_re[t][1], sh_re[t][2], sh_scan);
+      batch_range(cd, pieces, sh_item[j][0], &lo, &hi);
+      switch (cd.dtype) {
+        case NMV_F32: reread_warp<NMV_F32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        case NMV_F16: reread_warp<NMV_F16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        case NMV_BF16: reread_warp<NMV_BF16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        default: reread_warp<NMV_I32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+      }
     }
-    carry += total;
     __syncthreads();
   }
 }
 
+// ---- fp64 SSE re-pass: block b sums its contiguous range in index order per
+// thread, then a fixed tree; sse64_final adds the block sums in order.
+constexpr int kSseBlocks = 1024;
+
+__global__ void __launch_bounds__(kFinThreads) sse64_kernel(const CaseDesc *__restrict__ cd_p, double *part) {
+  const CaseDesc &cd = *cd_p;
+  __shared__ double sh[kFinThreads];
+  const int64_t per_block = (cd.numel + gridDim.x - 1) / gridDim.x;
+  const int64_t b0 = (int64_t)blockIdx.x * per_block;
+  const int64_t b1 = b0 + per_block < cd.numel ? b0 + per_block : cd.numel;
+  const int64_t per_thr = (per_block + kFinThreads - 1) / kFinThreads;
+  const int64_t t0 = b0 + (int64_t)threadIdx.x * per_thr;
+  const int64_t t1 = t0 + per_thr < b1 ? t0 + per_thr : b1;
+  double acc = 0.0;
+  for (int64_t i = t0; i < t1; ++i) {
+    const double c = widen_any(ld_elem(cd.cand, i, cd.dtype), cd.dtype);
+    const double r = widen_any(ld_elem(cd.ref, i, cd.dtype), cd.dtype);
+    if (isfinite(c) && isfinite(r)) {
+      const double d = __dsub_rn(c, r);
+      acc = __dadd_rn(acc, __dmul_rn(d, d));
+    }
+  }
+  sh[threadIdx.x] = acc;
+  __syncthreads();
+  for (int half = kFinThreads / 2; half > 0; half >>= 1) {
+    if (threadIdx.x < half) sh[threadIdx.x] = __dadd_rn(sh[threadIdx.x], sh[threadIdx.x + half]);
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) part[blockIdx.x] = sh[0];
+}
+
+__global__ void sse64_final(const double *part, int n, double *dst) {
+  if (threadIdx.x == 0 && blockIdx.x == 0) {
+    double acc = 0.0;
+    for (int b = 0; b < n; ++b) acc = __dadd_rn(acc, part[b]);
+    *dst = acc;
+  }
+}
+
 cudaError_t launch_finalize(const CaseDesc *cases, const Piece *pieces, const Partial *partials,
-                            const int32_t *seg_count, const uint32_t *seg_list, uint8_t *out,
-                            int n_cases, cudaStream_t st) {
-  finalize_kernel<<<n_cases, kFinThreads, 0, st>>>(cases, pieces, partials, seg_count, seg_list, out);
+                            const int32_t *batch_count, uint8_t *out, int n_cases, cudaStream_t st) {
+  finalize_kernel<<<n_cases, kFinThreads, 0, st>>>(cases, pieces, partials, batch_count, out);
+  return cudaGetLastError();
+}
+
+// Recompute one case's SSE in fp64 into *dst (device).  `part` holds
+// kSseBlocks doubles of scratch.
+cudaError_t launch_sse64(const CaseDesc *cd, double *part, double *dst, cudaStream_t st) {
+  sse64_kernel<<<kSseBlocks, kFinThreads, 0, st>>>(cd, part);
+  sse64_final<<<1, 32, 0, st>>>(part, kSseBlocks, dst);
   return cudaGetLastError();
 }
 

@@ -1,5 +1,5 @@
 // nmv_internal.h -- descriptors shared by the host planner (nmv_api.cu) and
-// the kernels (nmv_kernels.cu).  Not part of the public ABI.
+// the kernels (nmv_scan.cuh, nmv_finalize.cu).  Not part of the public ABI.
 #pragma once
 
 #include <cstdint>
@@ -17,12 +17,10 @@ namespace nmv {
 // ---- launch geometry ----------------------------------------------------
 constexpr int kWarps = 8;                 // warps per block of the scan kernel
 constexpr int kThreads = kWarps * 32;
-constexpr int kFirstR = 128;              // mismatch offsets kept per segment
 constexpr int kFinThreads = 256;          // threads per block of the finalize kernel
 constexpr int64_t kHistCap = 8192;        // smem tile-histogram window (bins)
 constexpr int64_t kProfCap = 4096;        // smem row / column profile (bins each)
 constexpr int64_t kMaxPiece = int64_t(1) << 30;  // elements per piece (int32 smem counters)
-constexpr int kSseFlush = 64;             // float-float SSE terms per fp64 flush
 
 // Element size in bytes and elements per 16-byte vector.
 NMV_HD int elem_bytes(int dt) { return (dt == NMV_F16 || dt == NMV_BF16) ? 2 : 4; }
@@ -59,18 +57,21 @@ struct CaseDesc {
   Div64 dN, dth, dtw;
   double rtol, atol;
   // fp32 pre-filter of the predicate: sure-pass if |s| <= fma_rz(lo_r, |r|, lo_a),
-  // sure-fail if |s| > fma_ru(hi_r, |r|, hi_a) (see element_pass).
+  // sure-fail if |s| > fma_ru(hi_r, |r|, hi_a) (see nmv_scan.cuh).
   float lo_r, lo_a, hi_r, hi_a;
   int64_t first_k;
   int64_t piece_begin, piece_end;      // this case's pieces
+  int64_t batch_begin, batch_end;      // this case's batches (global batch indices)
   int64_t out_off;                     // byte offset of this case's packed result
   int64_t hist_off, rowp_off, colp_off, fk_off;  // byte offsets inside the packed result
 };
 
-// A contiguous element range of one case processed by one block.  The
-// block's warps split it into kWarps segments (segment_range).
+// A contiguous element range of one case processed by one block.  It is
+// cut into batches of batch_elems(dtype) elements (the last one may be
+// shorter); warp w of the block takes batches w, w + kWarps, ... in order.
 struct Piece {
   int64_t begin, end;
+  int64_t batch_base;   // global index of the piece's first batch
   int64_t tr0, tc0;     // smem tile-histogram window origin (tile coordinates)
   int32_t wr, wc;       // window extent; wr == 0 -> histogram via global atomics
   int32_t case_id;
@@ -101,18 +102,12 @@ struct OutHeader {
   int64_t pad[3];
 };
 
-// Segment w of a piece [begin, end): a split into kWarps contiguous ranges
-// whose boundaries are multiples of `vec` elements past `begin`.
-NMV_HD void segment_range(int64_t begin, int64_t end, int w, int vec, int64_t *lo,
-                          int64_t *hi) {
-  int64_t len = end - begin;
-  int64_t per = (len + kWarps - 1) / kWarps;
-  per = (per + vec - 1) / vec * vec;
-  int64_t a = per * w, b = per * (w + 1);
-  if (a > len) a = len;
-  if (b > len) b = len;
-  *lo = begin + a;
-  *hi = begin + b;
+// Steps of one warp per batch, and elements per batch.
+constexpr int kUnroll = 4;
+NMV_HD int64_t batch_elems(int dt) { return (int64_t)32 * vec_elems(dt) * kUnroll; }
+NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt) {
+  const int64_t be = batch_elems(dt);
+  return (end - begin + be - 1) / be;
 }
 
 }  // namespace nmv

@@ -32,6 +32,16 @@ class Tensor(ctypes.Structure):
                 ("rank", ctypes.c_int32), ("shape", _i64p)]
 
 
+class Profile(ctypes.Structure):
+    _fields_ = [("scan_ms", ctypes.c_double), ("finalize_ms", ctypes.c_double),
+                ("kernel_launches", ctypes.c_int64), ("h2d_bytes", ctypes.c_int64),
+                ("d2h_bytes", ctypes.c_int64), ("slow_steps", ctypes.c_int64),
+                ("light_steps", ctypes.c_int64),
+                ("exact_abs", ctypes.c_int64), ("exact_rel", ctypes.c_int64),
+                ("exact_pred", ctypes.c_int64), ("slow_cycles", ctypes.c_int64),
+                ("light_cycles", ctypes.c_int64)]
+
+
 class Case(ctypes.Structure):
     _fields_ = [("cand", Tensor), ("ref", Tensor), ("inputs", ctypes.POINTER(Tensor)),
                 ("n_inputs", ctypes.c_int32), ("reserved", ctypes.c_int32),
@@ -85,6 +95,10 @@ def load() -> ctypes.CDLL:
             lib.nmv_status_string.argtypes = [ctypes.c_int]
             lib.nmv_last_error.restype = ctypes.c_char_p
             lib.nmv_last_error.argtypes = []
+            lib.nmv_profile_enable.restype = None
+            lib.nmv_profile_enable.argtypes = [ctypes.c_int]
+            lib.nmv_profile_last.restype = ctypes.c_int
+            lib.nmv_profile_last.argtypes = [ctypes.POINTER(Profile)]
             _lib = lib
     return _lib
 
@@ -251,3 +265,18 @@ class Prepared:
             return [result_to_dict(self.out[i]) for i in range(self.n)]
         finally:
             self.lib.nmv_result_free(self.out)
+
+
+def profile_enable(on: bool = True) -> None:
+    """Record CUDA events around the kernels of every following call."""
+    load().nmv_profile_enable(1 if on else 0)
+
+
+def profile_last() -> dict:
+    """Launch profile of the last profiled call (see nmv_profile in nmv.h)."""
+    lib = load()
+    p = Profile()
+    rc = lib.nmv_profile_last(ctypes.byref(p))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    return {name: getattr(p, name) for name, _ in Profile._fields_}

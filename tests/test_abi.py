@@ -40,7 +40,8 @@ def test_exports_every_declared_symbol(lib):
 def test_struct_layout_matches_header(tmp_path):
     from paper_2608_02712_gb300 import nmv
     prog = tmp_path / "layout.c"
-    fields = {"nmv_tensor": nmv.Tensor, "nmv_case": nmv.Case, "nmv_result": nmv.Result}
+    fields = {"nmv_tensor": nmv.Tensor, "nmv_case": nmv.Case, "nmv_result": nmv.Result,
+              "nmv_profile": nmv.Profile}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "nmv.h"', 'int main(void){']
     for cname, py in fields.items():
         lines.append('printf("%s sizeof %%zu\\n", sizeof(%s));' % (cname, cname))
@@ -61,6 +62,14 @@ def test_struct_layout_matches_header(tmp_path):
         assert got[(cname, "sizeof")] == ctypes.sizeof(py), cname
         for fname, _ in py._fields_:
             assert got[(cname, fname)] == getattr(py, fname).offset, (cname, fname)
+
+
+def test_profile_last_without_a_profiled_call(lib):
+    from paper_2608_02712_gb300 import nmv
+    assert lib.nmv_profile_last(None) == -1
+    nmv.profile_enable(False)
+    out = nmv.Profile()
+    assert lib.nmv_profile_last(ctypes.byref(out)) == -1
 
 
 def test_status_strings(lib):
