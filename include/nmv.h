@@ -169,11 +169,18 @@ const char *nmv_last_error(void);
 
 /* Launch profile, for measuring the kernels against their roofline (the
  * paper's forensics "compiles and profiles" a kernel, Section 4; this is the
- * library's own profile).  While enabled (on != 0), every call records CUDA
- * events on its stream around its scan-kernel launches and around its
- * finalize launch, and counts the scan pass's exact-path work.
- * nmv_profile_last() fills *out for the last successful call on any thread;
- * it returns NMV_EINVAL if profiling was off for that call or out is NULL. */
+ * library's own profile).  nmv_profile_enable(mode) applies to every
+ * following call on any thread; mode is a set of NMV_PROFILE_* bits (0 =
+ * off).  NMV_PROFILE_TIMING records CUDA events on the call's stream around
+ * its scan-kernel launches and around its finalize launch.
+ * NMV_PROFILE_COUNTERS makes the scan kernel count its exact-path work
+ * (atomic counters and clock reads, which slow it down; the counter fields
+ * are 0 without it).  nmv_profile_last() fills *out for the last successful
+ * profiled call; it returns NMV_EINVAL if there is none since the last
+ * nmv_profile_enable() or out is NULL. */
+#define NMV_PROFILE_TIMING 1
+#define NMV_PROFILE_COUNTERS 2
+
 typedef struct nmv_profile {
     double scan_ms;            /* scan-kernel launches, stream time          */
     double finalize_ms;        /* finalize launch, stream time               */
@@ -189,7 +196,7 @@ typedef struct nmv_profile {
     int64_t light_cycles;      /* SM clock cycles warps spent in light steps  */
 } nmv_profile;
 
-void nmv_profile_enable(int on);
+void nmv_profile_enable(int mode);
 int nmv_profile_last(nmv_profile *out);
 
 #ifdef __cplusplus

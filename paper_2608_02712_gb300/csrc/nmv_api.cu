@@ -111,7 +111,7 @@ DeviceState g_dev[kMaxDevices];
 
 // Launch timing (nmv_profile_enable / nmv_profile_last), guarded by g_mu.
 struct Profile {
-  bool on = false;
+  int mode = 0;  // NMV_PROFILE_* bits
   bool valid = false;
   nmv_profile last{};
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
@@ -425,7 +425,7 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.dtw = make_div((uint64_t)d.tw);
   d.rtol = c.rtol;
   d.atol = c.atol;
-  // fp32 pre-filter coefficients (margins of 2^-20; see nmv_kernels.cu)
+  // fp32 pre-filter coefficients (margins of 2^-20; see nmv_scan.cuh)
   const bool filter = c.rtol <= 0.5 && c.atol <= 0x1p100;
   d.filter_ok = filter ? 1 : 0;
   if (filter) {
@@ -597,8 +597,9 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     cudaStreamSynchronize(st);
     return fail(NMV_ECUDA, "injected launch failure");
   }
-  const bool prof = g_prof.on;
-  unsigned long long *d_stats = prof ? (unsigned long long *)(W + o_out) : nullptr;
+  const bool prof = g_prof.mode != 0;
+  unsigned long long *d_stats =
+      (g_prof.mode & NMV_PROFILE_COUNTERS) ? (unsigned long long *)(W + o_out) : nullptr;
   if (prof) {
     if (g_prof.ev_dev != dev) {
       for (cudaEvent_t &x : g_prof.ev) {
@@ -780,9 +781,9 @@ const char *nmv_status_string(int status) {
 
 const char *nmv_last_error(void) { return g_err.c_str(); }
 
-void nmv_profile_enable(int on) {
+void nmv_profile_enable(int mode) {
   std::lock_guard<std::mutex> lock(g_mu);
-  g_prof.on = on != 0;
+  g_prof.mode = mode & (NMV_PROFILE_TIMING | NMV_PROFILE_COUNTERS);
   g_prof.valid = false;
 }
 

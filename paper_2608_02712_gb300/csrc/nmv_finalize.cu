@@ -1,9 +1,9 @@
 // nmv_finalize.cu -- one block per case: reduce the piece partials of the
 // scan pass (fixed order, so the result is bit-identical run to run), derive
-// the degenerate-output flags, and write the first-K mismatch records:
-// copied from the per-segment offset lists, or found by re-reading a segment
-// whose list overflowed.  Also the fp64 SSE re-pass for cases whose
-// differences are all tiny (see nmv_scan.cuh).
+// the degenerate-output flags, and write the first-K mismatch records, found
+// by re-reading the few batches that hold them (located through the pieces'
+// and then the batches' mismatch counts).  Also the fp64 SSE re-pass for
+// cases whose differences are all tiny (see nmv_scan.cuh).
 #include "nmv_scan.cuh"
 
 namespace nmv {
@@ -67,13 +67,14 @@ __device__ __forceinline__ int64_t block_excl_scan64(int64_t v, int64_t *total, 
   return sh[warp] + incl - v;
 }
 
-__device__ void write_record(const CaseDesc &cd, uint8_t *o, int64_t pos, int64_t idx) {
+__device__ __forceinline__ void write_record(const CaseDesc &cd, uint8_t *o, int64_t pos, int64_t idx,
+                                             uint32_t cb, uint32_t rb) {
   int64_t *fk_index = (int64_t *)(o + cd.fk_off);
   double *fk_c = (double *)(fk_index + cd.first_k);
   double *fk_r = fk_c + cd.first_k;
   fk_index[pos] = idx;
-  fk_c[pos] = widen_any(ld_elem(cd.cand, idx, cd.dtype), cd.dtype);
-  fk_r[pos] = widen_any(ld_elem(cd.ref, idx, cd.dtype), cd.dtype);
+  fk_c[pos] = widen_any(cb, cd.dtype);
+  fk_r[pos] = widen_any(rb, cd.dtype);
 }
 
 // Re-read elements [lo, hi) with one warp and write the first `needed`
@@ -88,12 +89,17 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
   int64_t found = 0;
   for (int64_t base = lo; base < hi && found < needed; base += 32 * E) {
     const int64_t i0 = base + (int64_t)lane * E;
-    uint32_t mask = 0;
+    uint32_t cb[E], rb[E];
 #pragma unroll
     for (int k = 0; k < E; ++k) {
-      const int64_t i = i0 + k;
-      if (i < hi && !pass_elem<DT>(cd, ld_one<EB>(cd.cand, i), ld_one<EB>(cd.ref, i))) mask |= 1u << k;
+      const bool in = i0 + k < hi;
+      cb[k] = in ? ld_one<EB>(cd.cand, i0 + k) : 0u;
+      rb[k] = in ? ld_one<EB>(cd.ref, i0 + k) : 0u;
     }
+    uint32_t mask = 0;
+#pragma unroll
+    for (int k = 0; k < E; ++k)
+      if (i0 + k < hi && !pass_elem<DT>(cd, cb[k], rb[k])) mask |= 1u << k;
     const int cnt = __popc(mask);
     int incl = cnt;
 #pragma unroll
@@ -101,31 +107,55 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
       const int t = __shfl_up_sync(0xffffffffu, incl, d);
       if (lane >= d) incl += t;
     }
-    int64_t pos = found + incl - cnt;
-    while (mask) {
-      const int k = __ffs(mask) - 1;
-      mask &= mask - 1;
-      if (pos < needed) write_record(cd, o, pos0 + pos, i0 + k);
-      ++pos;
+    const int64_t pos = found + incl - cnt;
+#pragma unroll
+    for (int k = 0, j = 0; k < E; ++k) {
+      if ((mask >> k) & 1u) {
+        if (pos + j < needed) write_record(cd, o, pos0 + pos + j, i0 + k, cb[k], rb[k]);
+        ++j;
+      }
     }
     found += __shfl_sync(0xffffffffu, incl, 31);
   }
 }
 
-// Element range of global batch g of a case (its pieces are ordered by
-// batch_base).
-__device__ __forceinline__ void batch_range(const CaseDesc &cd, const Piece *pieces, int64_t g, int64_t *lo,
-                                            int64_t *hi) {
-  int64_t a = cd.piece_begin, b = cd.piece_end - 1;
-  while (a < b) {
-    const int64_t mid = (a + b + 1) / 2;
-    if (pieces[mid].batch_base <= g) a = mid;
-    else b = mid - 1;
-  }
-  const Piece &pc = pieces[a];
+// Records of one piece whose first record has position pos0 (< K): its
+// batches are taken kFinThreads at a time, a block scan of their mismatch
+// counts places them, and each batch holding records below K is re-read by
+// one warp.  Called by the whole block with uniform arguments.
+__device__ void first_k_piece(const CaseDesc &cd, uint8_t *o, const Piece &pc, const int32_t *batch_count,
+                              int64_t pos0, int64_t K, int64_t *sh_scan, int64_t (*sh_item)[3], int *sh_nitems) {
   const int64_t be = batch_elems(cd.dtype);
-  *lo = pc.begin + (g - pc.batch_base) * be;
-  *hi = *lo + be < pc.end ? *lo + be : pc.end;
+  const int64_t nb = piece_batches(pc.begin, pc.end, cd.dtype);
+  const int warp = threadIdx.x >> 5;
+  int64_t pos = pos0;
+  for (int64_t b0 = 0; b0 < nb && pos < K; b0 += kFinThreads) {
+    const int64_t b = b0 + threadIdx.x;
+    const int64_t n = b < nb ? batch_count[pc.batch_base + b] : 0;
+    int64_t total;
+    const int64_t pre = pos + block_excl_scan64(n, &total, sh_scan);
+    if (threadIdx.x == 0) *sh_nitems = 0;
+    __syncthreads();
+    if (n > 0 && pre < K) {
+      const int it = atomicAdd(sh_nitems, 1);
+      sh_item[it][0] = b;
+      sh_item[it][1] = pre;
+      sh_item[it][2] = n < K - pre ? n : K - pre;
+    }
+    __syncthreads();
+    for (int j = warp; j < *sh_nitems; j += kFinThreads / 32) {
+      const int64_t lo = pc.begin + sh_item[j][0] * be;
+      const int64_t hi = lo + be < pc.end ? lo + be : pc.end;
+      switch (cd.dtype) {
+        case NMV_F32: reread_warp<NMV_F32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        case NMV_F16: reread_warp<NMV_F16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        case NMV_BF16: reread_warp<NMV_BF16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+        default: reread_warp<NMV_I32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
+      }
+    }
+    __syncthreads();
+    pos += total;
+  }
 }
 
 struct Red {
@@ -156,13 +186,14 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
   OutHeader *H = (OutHeader *)o;
   __shared__ int64_t sh_scan[kFinThreads / 32 + 1];
   __shared__ int64_t sh_mism;
-  constexpr int kItems = 512;
-  __shared__ int64_t sh_item[kItems][3];
-  constexpr int kRed = 64;
-  __shared__ Red sh_red[kRed];
+  __shared__ int64_t sh_need[kFinThreads];
+  __shared__ int64_t sh_item[kFinThreads][3];
+  __shared__ int sh_nitems;
+  __shared__ Red sh_red[kFinThreads / 32];
 
-  // ---- 1. reduce the partials: thread t < kRed takes pieces t, t + kRed,
-  // ... in order, then a fixed pairwise tree over those threads.
+  // ---- 1. reduce the partials: thread t takes pieces t, t + kFinThreads,
+  // ... in order, then a fixed butterfly within each warp and the warps in
+  // order (the same tree on every run).
   {
     Red a;
     for (int k = 0; k < 8; ++k) a.cnt[k] = 0;
@@ -171,7 +202,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
     a.sse = 0.0;
     a.cacc = a.racc = 0;
     for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] = 0;
-    for (int64_t p = cd.piece_begin + threadIdx.x; threadIdx.x < kRed && p < cd.piece_end; p += kRed) {
+    for (int64_t p = cd.piece_begin + threadIdx.x; p < cd.piece_end; p += kFinThreads) {
       const Partial &Q = partials[p];
       Red b;
       for (int k = 0; k < 8; ++k) b.cnt[k] = Q.cnt[k];
@@ -183,12 +214,35 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = Q.eq[j];
       red_add(a, b);
     }
-    if (threadIdx.x < kRed) sh_red[threadIdx.x] = a;
-    __syncthreads();
-    for (int half = kRed / 2; half > 0; half >>= 1) {
-      if (threadIdx.x < half) red_add(sh_red[threadIdx.x], sh_red[threadIdx.x + half]);
-      __syncthreads();
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      Red b;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) b.cnt[k] = __shfl_xor_sync(0xffffffffu, a.cnt[k], off);
+      b.ba.v = __shfl_xor_sync(0xffffffffu, a.ba.v, off);
+      b.ba.i = __shfl_xor_sync(0xffffffffu, a.ba.i, off);
+      b.br.v = __shfl_xor_sync(0xffffffffu, a.br.v, off);
+      b.br.i = __shfl_xor_sync(0xffffffffu, a.br.i, off);
+      b.sse = __shfl_xor_sync(0xffffffffu, a.sse, off);
+      b.cacc = __shfl_xor_sync(0xffffffffu, a.cacc, off);
+      b.racc = __shfl_xor_sync(0xffffffffu, a.racc, off);
+#pragma unroll
+      for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = __shfl_xor_sync(0xffffffffu, a.eq[j], off);
+      // lanes below the partner add the partner's value second, lanes above
+      // first, so both hold the same bits
+      if ((threadIdx.x & off) == 0) {
+        red_add(a, b);
+      } else {
+        red_add(b, a);
+        a = b;
+      }
     }
+    if ((threadIdx.x & 31) == 0) sh_red[threadIdx.x >> 5] = a;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      for (int w = 1; w < kFinThreads / 32; ++w) red_add(sh_red[0], sh_red[w]);
+    }
+    __syncthreads();
   }
   if (threadIdx.x == 0) {
     const Red &a = sh_red[0];
@@ -230,60 +284,26 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
   }
   __syncthreads();
 
-  // ---- 2. first-K records.  Thread t sums the counts of a contiguous
-  // chunk of the case's batches; a block scan places the chunks; every
-  // batch holding records below K becomes an item (batch, first record
-  // position, records wanted), and the warps re-read the items' batches.
+  // ---- 2. first-K records.  Pieces are taken kFinThreads at a time, one
+  // per thread; a block scan of their mismatch counts gives each piece its
+  // first record position.  Each piece holding records below K is then
+  // scanned the same way over its batch counts, and every batch holding
+  // records below K is re-read by one warp.
   const int64_t K = cd.first_k;
   if (K == 0 || sh_mism == 0) return;
-  const int64_t B0 = cd.batch_begin, B1 = cd.batch_end;
-  const int64_t cs = (B1 - B0 + kFinThreads - 1) / kFinThreads;
-  const int64_t c0 = B0 + (int64_t)threadIdx.x * cs;
-  const int64_t c1 = c0 + cs < B1 ? c0 + cs : B1;
-  int64_t sum = 0;
-  for (int64_t g = c0; g < c1; ++g) sum += batch_count[g];
-  int64_t total;
-  const int64_t pre = block_excl_scan64(sum, &total, sh_scan);
-  int64_t mine = 0;
-  {
-    int64_t pos = pre;
-    for (int64_t g = c0; g < c1 && pos < K; ++g) {
-      const int64_t n = batch_count[g];
-      if (n > 0) {
-        ++mine;
-        pos += n;
-      }
-    }
-  }
-  int64_t n_items;
-  const int64_t ioff = block_excl_scan64(mine, &n_items, sh_scan);
-  const int warp = threadIdx.x >> 5;
-  for (int64_t r0 = 0; r0 < n_items; r0 += kItems) {
-    int64_t it = ioff, pos = pre;
-    for (int64_t g = c0; g < c1 && pos < K && it < r0 + kItems; ++g) {
-      const int64_t n = batch_count[g];
-      if (n > 0) {
-        if (it >= r0) {
-          sh_item[it - r0][0] = g;
-          sh_item[it - r0][1] = pos;
-          sh_item[it - r0][2] = n < K - pos ? n : K - pos;
-        }
-        ++it;
-        pos += n;
-      }
-    }
+  int64_t base = 0;  // records in the pieces before this round
+  for (int64_t q0 = cd.piece_begin; q0 < cd.piece_end && base < K; q0 += kFinThreads) {
+    const int64_t p = q0 + threadIdx.x;
+    const int64_t n = p < cd.piece_end ? partials[p].cnt[0] : 0;
+    int64_t total;
+    const int64_t pre = base + block_excl_scan64(n, &total, sh_scan);
+    sh_need[threadIdx.x] = (n > 0 && pre < K) ? pre : -1;
     __syncthreads();
-    const int64_t m = n_items - r0 < kItems ? n_items - r0 : kItems;
-    for (int64_t j = warp; j < m; j += kFinThreads / 32) {
-      int64_t lo, hi;
-      batch_range(cd, pieces, sh_item[j][0], &lo, &hi);
-      switch (cd.dtype) {
-        case NMV_F32: reread_warp<NMV_F32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
-        case NMV_F16: reread_warp<NMV_F16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
-        case NMV_BF16: reread_warp<NMV_BF16>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
-        default: reread_warp<NMV_I32>(cd, o, lo, hi, sh_item[j][1], sh_item[j][2]); break;
-      }
+    for (int j = 0; j < kFinThreads && q0 + j < cd.piece_end; ++j) {
+      const int64_t pos0 = sh_need[j];
+      if (pos0 >= 0) first_k_piece(cd, o, pieces[q0 + j], batch_count, pos0, K, sh_scan, sh_item, &sh_nitems);
     }
+    base += total;
     __syncthreads();
   }
 }

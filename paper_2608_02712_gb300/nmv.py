@@ -267,9 +267,15 @@ class Prepared:
             self.lib.nmv_result_free(self.out)
 
 
-def profile_enable(on: bool = True) -> None:
-    """Record CUDA events around the kernels of every following call."""
-    load().nmv_profile_enable(1 if on else 0)
+PROFILE_TIMING = 1
+PROFILE_COUNTERS = 2
+
+
+def profile_enable(mode: int = PROFILE_TIMING) -> None:
+    """Profile every following call: PROFILE_TIMING records CUDA events
+    around the kernels, PROFILE_COUNTERS counts the scan's exact-path work
+    (and slows it down); 0 or False turns profiling off."""
+    load().nmv_profile_enable(int(mode))
 
 
 def profile_last() -> dict:
