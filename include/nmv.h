@@ -157,6 +157,48 @@ int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out);
 int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
                        nmv_result **out);
 
+/* ---- validation without allocation --------------------------------------
+ * The paper has no counterpart of this entry point; it is a service of this
+ * library.  nmv_validate may allocate: it grows a cached device workspace
+ * with cudaMalloc and a pinned staging block with cudaHostAlloc when a case
+ * needs more than earlier calls did.  Some callers cannot allow that: a
+ * process whose framework allocator has reserved (nearly) all device memory
+ * up front, so that a library's own cudaMalloc fails or fragments it, and
+ * latency-critical code that must not meet cudaMalloc/cudaFree's implicit
+ * device-wide synchronisation.  nmv_validate_noalloc validates one case like
+ * nmv_validate, with the same kernels and bit-identical results, but calls
+ * no cudaMalloc, cudaFree, cudaHostAlloc or other allocating routine:
+ *
+ *  - its device scratch is one fixed array of NMV_NOALLOC_SCRATCH_BYTES in
+ *    the library's module; every GPU that loads the library holds it until
+ *    the process exits;
+ *  - the caller owns the output: before the call it points out->tile_hist
+ *    [grid_rows * grid_cols], row_prof [tile_rows], col_prof [tile_cols],
+ *    fk_index, fk_cand, fk_ref [first_k], fk_coords [first_k * rank] and
+ *    input_eq [n_inputs] at host arrays of at least those sizes (grid_rows =
+ *    ceil(M / tile_rows), grid_cols = ceil(N / tile_cols), see nmv_case; an
+ *    array whose size is 0 may be NULL).  The call fills them and every
+ *    scalar field of *out, and leaves the pointers as they were.
+ *
+ * A case needs about: 4 bytes per batch of 1024 (16-bit types) or 512
+ * (32-bit types) elements, 8 bytes per histogram bin, 8 * (tile_rows +
+ * tile_cols) + 24 * first_k bytes, and under 1 MiB of descriptors and
+ * partials.  A case that does not fit fails with NMV_EINVAL and a message
+ * giving the bytes it needs (nmv_validate has no such limit).
+ *
+ * The first call on each device looks up the scratch array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture.  All calls share the one array and find the
+ * previous call's contents in it; each call clears what must start at zero.
+ * Calls made through this library are serialised by its lock and return
+ * only after their stream work has finished; calls that did overlap on the
+ * GPU would race on the array.  Profiling (nmv_profile_enable) does not
+ * apply to this entry point.  On error *out's scalar fields are unspecified.
+ */
+#define NMV_NOALLOC_SCRATCH_BYTES (32LL << 20)
+
+int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out);
+
 /* Release what one nmv_validate / nmv_validate_batch call returned.  NULL
  * is accepted. */
 void nmv_result_free(nmv_result *r);

@@ -7,4 +7,4 @@ validation step of the paper's repair engine, Section 3.2, Eq. 1, and
 Sections 4.2-4.3).  ``workloads`` holds the seeded synthetic inputs.
 """
 from .nmv import (FLAGS, NmvError, Prepared, load, validate,  # noqa: F401
-                  validate_batch)
+                  validate_batch, validate_noalloc)

@@ -752,6 +752,235 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   return NMV_OK;
 }
 
+// ---- validation without allocation (nmv_validate_noalloc) ----------------
+// Scratch of the no-allocation entry point: a fixed array in the module's
+// device memory, present on every GPU that loads this library until the
+// process exits.  Host code must not pass `g_noalloc_scratch` itself to a
+// kernel (in host code it names a host-side stand-in); it passes the device
+// address from cudaGetSymbolAddress, looked up once per device.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[NMV_NOALLOC_SCRATCH_BYTES];
+void *g_noalloc_ptr[kMaxDevices];
+
+// Host staging of the descriptors: file-scope arrays, so planning a call
+// allocates nothing either.  Guarded by g_mu.
+constexpr int kNaMaxBlocks = 8192;
+CaseDesc g_na_desc;
+Piece g_na_pieces[kNaMaxBlocks];
+int64_t g_na_bp[kNaMaxBlocks + 1];
+OutHeader g_na_head;
+
+int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
+  if (c == nullptr) return fail(NMV_EINVAL, "case is NULL");
+  if (out == nullptr) return fail(NMV_EINVAL, "out is NULL");
+  Geo g;
+  int rc = check_case(*c, &g);
+  if (rc) return rc;
+  const int64_t n_hist = g.GR * g.GC;
+  if ((n_hist > 0 && out->tile_hist == nullptr) || out->row_prof == nullptr || out->col_prof == nullptr)
+    return fail(NMV_EINVAL, "out->tile_hist, row_prof and col_prof must point to caller arrays");
+  if (c->first_k > 0 && (out->fk_index == nullptr || out->fk_cand == nullptr || out->fk_ref == nullptr ||
+                         (c->cand.rank > 0 && out->fk_coords == nullptr)))
+    return fail(NMV_EINVAL, "out->fk_index, fk_coords, fk_cand and fk_ref must point to caller arrays");
+  if (c->n_inputs > 0 && out->input_eq == nullptr)
+    return fail(NMV_EINVAL, "out->input_eq must point to a caller array");
+
+  std::lock_guard<std::mutex> lock(g_mu);
+  int dev = -1;
+  DeviceState *S = nullptr;
+  rc = probe_device(&dev, &S);
+  if (rc) return rc;
+  if (g_noalloc_ptr[dev] == nullptr) {
+    // First call on this device: look up the scratch array's device address.
+    void *ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress (scratch)");
+    g_noalloc_ptr[dev] = ptr;
+  }
+  uint8_t *W = (uint8_t *)g_noalloc_ptr[dev];
+  cudaStream_t st = (cudaStream_t)stream;
+
+  // ---- plan: the scan kernel's byte-balanced split of one case
+  int grid = 0;
+  int64_t n_pieces = 0;
+  size_t smem = 1024;
+  const int nin = nin_class(*c, g);
+  const int gi = nin + 1;
+  if (g.numel > 0) {
+    size_t prof = kShHeadWords * 4;
+    if (c->tile_rows <= kProfCap && c->tile_cols <= kProfCap)
+      prof = (size_t)(kShHeadWords + c->tile_rows + c->tile_cols) * 4;
+    size_t guess = prof;
+    for (int attempt = 0; attempt < 3; ++attempt) {
+      const size_t want = std::min(std::max(guess, (size_t)1024), S->smem_optin);
+      size_t &set = S->smem_set[g.dt][gi];
+      if (want > set) {
+        cudaError_t e = scan_prepare(g.dt, nin, want);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+        set = want;
+      }
+      int occ = scan_occupancy(g.dt, nin, want);
+      if (occ < 1) occ = 1;
+      int64_t gr = (int64_t)S->sms * occ;
+      gr = std::min(gr, std::max<int64_t>(1, g.numel * g.eb / 16384));
+      gr = std::min<int64_t>(gr, kNaMaxBlocks);
+      grid = (int)gr;
+      const int64_t total = g.numel * g.eb;
+      size_t need = 0;
+      n_pieces = 0;
+      for (int b = 0; b < grid; ++b) {
+        g_na_bp[b] = n_pieces;
+        const int64_t x0 = (int64_t)((__int128)total * b / grid);
+        const int64_t x1 = (int64_t)((__int128)total * (b + 1) / grid);
+        const int64_t e0 = x0 / g.eb / g.vec * g.vec;
+        const int64_t e1 = (b + 1 == grid) ? g.numel : x1 / g.eb / g.vec * g.vec;
+        if (e1 <= e0) continue;
+        if (e1 - e0 > kMaxPiece) return fail(NMV_EINVAL, "case too large for the no-allocation scratch");
+        Piece &pc = g_na_pieces[n_pieces++];
+        std::memset(&pc, 0, sizeof(pc));
+        pc.begin = e0;
+        pc.end = e1;
+        pc.case_id = 0;
+        piece_window(*c, g, pc);
+        need = std::max(need, piece_smem(*c, pc));
+      }
+      g_na_bp[grid] = n_pieces;
+      smem = std::max(need, (size_t)1024);
+      if (need <= want) break;
+      guess = need;
+    }
+    if (smem > S->smem_optin)
+      return fail(NMV_EINVAL, "localisation maps need more shared memory than the device has");
+    size_t &set = S->smem_set[g.dt][gi];
+    if (smem > set) {
+      cudaError_t e = scan_prepare(g.dt, nin, smem);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+      set = smem;
+    }
+  }
+  fill_desc(*c, g, g_na_desc);
+  g_na_desc.out_off = (int64_t)kCallHeader;
+  g_na_desc.piece_begin = 0;
+  g_na_desc.piece_end = n_pieces;
+  int64_t n_batches = 0;
+  for (int64_t k = 0; k < n_pieces; ++k) {
+    g_na_pieces[k].batch_base = n_batches;
+    n_batches += piece_batches(g_na_pieces[k].begin, g_na_pieces[k].end, g.dt);
+  }
+  g_na_desc.batch_begin = 0;
+  g_na_desc.batch_end = n_batches;
+
+  // ---- scratch layout (the same regions as the workspace of nmv_validate)
+  const size_t sz_cases = align_up(sizeof(CaseDesc), 256);
+  const size_t sz_pieces = align_up(sizeof(Piece) * (size_t)std::max<int64_t>(n_pieces, 1), 256);
+  const size_t sz_bp = align_up(sizeof(int64_t) * (size_t)(grid + 1), 256);
+  const size_t o_part = sz_cases + sz_pieces + sz_bp;
+  const size_t sz_part = align_up(sizeof(Partial) * (size_t)std::max<int64_t>(n_pieces, 1), 256);
+  const size_t o_segc = o_part + sz_part;
+  const size_t sz_segc = align_up(sizeof(int32_t) * (size_t)std::max<int64_t>(n_batches, 1), 256);
+  const size_t o_sse = o_segc + sz_segc;
+  const size_t o_thr = o_sse + align_up(sizeof(double) * kSseBlocksHost, 256);
+  const size_t o_out = o_thr + 256;
+  const size_t need = o_out + kCallHeader + g.out_size;
+  if (need > (size_t)NMV_NOALLOC_SCRATCH_BYTES) {
+    char buf[160];
+    std::snprintf(buf, sizeof buf,
+                  "case needs %zu bytes of scratch; the no-allocation scratch holds %lld (use nmv_validate)",
+                  need, (long long)NMV_NOALLOC_SCRATCH_BYTES);
+    return fail(NMV_EINVAL, buf);
+  }
+
+  // ---- upload, clear, launch
+  cudaError_t e = cudaMemcpyAsync(W, &g_na_desc, sizeof(CaseDesc), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && n_pieces > 0)
+    e = cudaMemcpyAsync(W + sz_cases, g_na_pieces, sizeof(Piece) * (size_t)n_pieces, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && grid > 0)
+    e = cudaMemcpyAsync(W + sz_cases + sz_pieces, g_na_bp, sizeof(int64_t) * (size_t)(grid + 1),
+                        cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
+  // The scratch keeps the previous call's contents: the thresholds and the
+  // packed result (maps and counters are accumulated) must start at zero.
+  // Partials and batch counts are written in full by the scan kernel.
+  e = cudaMemsetAsync(W + o_thr, 0, 256 + kCallHeader + g.out_size, st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  const CaseDesc *d_case = (const CaseDesc *)W;
+  const Piece *d_pieces = (const Piece *)(W + sz_cases);
+  if (grid > 0) {
+    e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (const int64_t *)(W + sz_cases + sz_pieces), 0,
+                    (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr);
+    if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
+  }
+  e = launch_finalize(d_case, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc), W + o_out,
+                      1, st);
+  if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
+  const uint8_t *ob = W + o_out + kCallHeader;
+  e = cudaMemcpyAsync(&g_na_head, ob, sizeof(OutHeader), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (result header)");
+  if (g_na_head.max_abs > 0.0 && g_na_head.max_abs < 0x1p-38) {
+    // the fp64 SSE re-pass for cases whose differences are all tiny
+    double *dst = (double *)(W + o_out + kCallHeader + offsetof(OutHeader, sse));
+    e = launch_sse64(d_case, (double *)(W + o_sse), dst, st);
+    if (e != cudaSuccess) return cuda_fail(e, "fp64 SSE launch");
+    e = cudaMemcpyAsync(&g_na_head.sse, dst, sizeof(double), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fp64 SSE)");
+  }
+  const int64_t k = g_na_head.k_out;
+  if (n_hist > 0) e = cudaMemcpyAsync(out->tile_hist, ob + g.hist_off, 8 * (size_t)n_hist, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(out->row_prof, ob + g.rowp_off, 8 * (size_t)c->tile_rows, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(out->col_prof, ob + g.colp_off, 8 * (size_t)c->tile_cols, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess && k > 0) {
+    const uint8_t *fki = ob + g.fk_off;
+    e = cudaMemcpyAsync(out->fk_index, fki, 8 * (size_t)k, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(out->fk_cand, fki + 8 * (size_t)c->first_k, 8 * (size_t)k, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(out->fk_ref, fki + 16 * (size_t)c->first_k, 8 * (size_t)k, cudaMemcpyDeviceToHost, st);
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (results)");
+
+  // ---- scalar fields; the caller's array pointers stay as they were
+  const OutHeader &oh = g_na_head;
+  out->status = (int32_t)oh.status;
+  out->rank = c->cand.rank;
+  out->numel = g.numel;
+  out->mismatch = oh.cnt[0];
+  out->cand_nan = oh.cnt[1];
+  out->cand_posinf = oh.cnt[2];
+  out->cand_neginf = oh.cnt[3];
+  out->ref_nan = oh.cnt[4];
+  out->ref_posinf = oh.cnt[5];
+  out->ref_neginf = oh.cnt[6];
+  out->n_finite_pairs = oh.cnt[7];
+  out->pass = out->mismatch == 0;
+  out->flags = oh.flags;
+  out->max_abs = oh.max_abs;
+  out->max_rel = oh.max_rel;
+  out->sse = oh.sse;
+  out->argmax_abs = oh.argmax_abs;
+  out->argmax_rel = oh.argmax_rel;
+  out->grid_rows = g.GR;
+  out->grid_cols = g.GC;
+  out->tile_rows = c->tile_rows;
+  out->tile_cols = c->tile_cols;
+  out->k_out = k;
+  for (int64_t t = 0; t < k; ++t) {
+    int64_t idx = out->fk_index[t];
+    for (int d = c->cand.rank - 1; d >= 0; --d) {
+      const int64_t sd = c->cand.shape[d];
+      out->fk_coords[t * c->cand.rank + d] = sd > 0 ? idx % sd : 0;
+      idx = sd > 0 ? idx / sd : 0;
+    }
+  }
+  out->n_inputs = c->n_inputs;
+  out->passthrough_input = oh.passthrough;
+  for (int j = 0; j < c->n_inputs; ++j) out->input_eq[j] = oh.input_eq[j];
+  g_err.clear();
+  return NMV_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -764,6 +993,10 @@ int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out) {
 
 int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream, nmv_result **out) {
   return run(cases, n, cuda_stream, out);
+}
+
+int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out) {
+  return run_noalloc(c, cuda_stream, out);
 }
 
 void nmv_result_free(nmv_result *r) { std::free(r); }

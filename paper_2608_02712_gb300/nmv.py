@@ -99,6 +99,9 @@ def load() -> ctypes.CDLL:
             lib.nmv_profile_enable.argtypes = [ctypes.c_int]
             lib.nmv_profile_last.restype = ctypes.c_int
             lib.nmv_profile_last.argtypes = [ctypes.POINTER(Profile)]
+            lib.nmv_validate_noalloc.restype = ctypes.c_int
+            lib.nmv_validate_noalloc.argtypes = [ctypes.POINTER(Case), ctypes.c_void_p,
+                                                 ctypes.POINTER(Result)]
             _lib = lib
     return _lib
 
@@ -227,6 +230,44 @@ def validate_batch(cases, stream=None) -> dict:
         if out:
             lib.nmv_result_free(out)
     return {"results": results, "n_pass": sum(int(r["pass"]) for r in results)}
+
+
+def validate_noalloc(cand: torch.Tensor, ref: torch.Tensor, *, inputs=(), rtol: float,
+                     atol: float, tile=(64, 64), first_k: int = 256, stream=None) -> dict:
+    """Validate one pair through nmv_validate_noalloc, the entry point that
+    allocates no device or pinned memory (its scratch is a fixed array in the
+    library; see nmv.h).  The output arrays are host arrays owned here."""
+    lib = load()
+    case, keep = make_case(cand, ref, inputs=inputs, rtol=rtol, atol=atol, tile=tile,
+                           first_k=first_k)
+    shape = list(cand.shape)
+    n = cand.shape[-1] if cand.dim() else 1
+    m = cand.numel() // n if (cand.dim() and n) else (0 if cand.numel() == 0 else 1)
+    if cand.numel() == 0:
+        gr = gc = 0
+    else:
+        gr, gc = -(-m // int(tile[0])), -(-n // int(tile[1]))
+    k = int(first_k)
+    bufs = {
+        "tile_hist": np.zeros(max(gr * gc, 1), np.int64),
+        "row_prof": np.zeros(int(tile[0]), np.int64),
+        "col_prof": np.zeros(int(tile[1]), np.int64),
+        "fk_index": np.zeros(max(k, 1), np.int64),
+        "fk_coords": np.zeros(max(k * len(shape), 1), np.int64),
+        "fk_cand": np.zeros(max(k, 1), np.float64),
+        "fk_ref": np.zeros(max(k, 1), np.float64),
+        "input_eq": np.zeros(max(len(inputs), 1), np.int64),
+    }
+    r = Result()
+    for name, arr in bufs.items():
+        ctype = ctypes.c_double if arr.dtype == np.float64 else ctypes.c_int64
+        setattr(r, name, arr.ctypes.data_as(ctypes.POINTER(ctype)))
+    rc = lib.nmv_validate_noalloc(ctypes.byref(case), _stream_handle(stream), ctypes.byref(r))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    out = result_to_dict(r)
+    del keep, bufs
+    return out
 
 
 class Prepared:
