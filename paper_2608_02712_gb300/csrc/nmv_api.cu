@@ -24,7 +24,7 @@ struct ScanOps {
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
-                            unsigned long long *stats);
+                            unsigned long long *stats, uint32_t *err);
 };
 cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
                             int, cudaStream_t);
@@ -52,20 +52,20 @@ int scan_occupancy(int dt, int nin, size_t smem) {
 cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                         const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
                         Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
-                        unsigned long long *stats) {
+                        unsigned long long *stats, uint32_t *err) {
   switch (dt) {
     case NMV_F32:
       return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, batch_count, out, g_thr, stats);
+                                      partials, batch_count, out, g_thr, stats, err);
     case NMV_F16:
       return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, batch_count, out, g_thr, stats);
+                                      partials, batch_count, out, g_thr, stats, err);
     case NMV_BF16:
       return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                       partials, batch_count, out, g_thr, stats);
+                                       partials, batch_count, out, g_thr, stats, err);
     default:
       return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
-                                      partials, batch_count, out, g_thr, stats);
+                                      partials, batch_count, out, g_thr, stats, err);
   }
 }
 }  // namespace nmv
@@ -119,8 +119,11 @@ struct Profile {
 } g_prof;
 
 // The packed results start with a call header holding the scan pass's
-// exact-path counters (filled when profiling is on).
+// exact-path counters (filled when profiling is on) and, at byte
+// kCallErrOff, the scan kernel's error word (nonzero: a bulk copy into
+// shared memory did not complete within the kernel's wait limit).
 constexpr size_t kCallHeader = 256;
+constexpr size_t kCallErrOff = 128;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -325,7 +328,7 @@ size_t piece_smem(const nmv_case &c, const Piece &p) {
 
 // Split the concatenated bytes of the cases `ids` into `grid` balanced block
 // ranges; cut them at case boundaries (and at kMaxPiece) into pieces whose
-// element boundaries are multiples of the case's vector width.
+// element boundaries are multiples of the case's batch (batch_elems).
 void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::vector<int64_t> &ids,
                int grid, Plan &plan) {
   const int64_t n = (int64_t)ids.size();
@@ -344,7 +347,7 @@ void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::ve
     }
     const Geo &g = geo[ids[ci]];
     int64_t e = (x - off[ci]) / g.eb;
-    e = e / g.vec * g.vec;
+    e = e / batch_elems(g.dt) * batch_elems(g.dt);
     sc[b] = ci;
     se[b] = e;
   }
@@ -518,7 +521,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       if (G.plan.smem <= want) break;
       guess = G.plan.smem;
     }
-    if (G.smem > S->smem_optin)
+    if (G.smem + ring_bytes(G.nin) > S->smem_optin)
       return fail(NMV_EINVAL, "localisation maps need more shared memory than the device has");
     size_t &set = S->smem_set[G.dt][G.nin + 1];
     if (G.smem > set) {
@@ -618,7 +621,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   for (const Group &G : groups) {
     e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_bp + G.bp_base,
                     G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out,
-                    (uint32_t *)(W + o_thr), d_stats);
+                    (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   if (prof) cudaEventRecord(g_prof.ev[1], st);
@@ -632,6 +635,8 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   if (injected("d2h")) return fail(NMV_ECUDA, "injected copy-back failure");
+  if (*(const uint32_t *)(HO + kCallErrOff) != 0)
+    return fail(NMV_ECUDA, "scan kernel: a bulk copy into shared memory did not complete in time");
   // Cases whose differences are all tiny (max |d| < 2^-38): the fp32 squares
   // of the scan pass may have lost terms, so their SSE is recomputed in fp64.
   for (int64_t i = 0; i < n; ++i) {
@@ -831,8 +836,9 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
         g_na_bp[b] = n_pieces;
         const int64_t x0 = (int64_t)((__int128)total * b / grid);
         const int64_t x1 = (int64_t)((__int128)total * (b + 1) / grid);
-        const int64_t e0 = x0 / g.eb / g.vec * g.vec;
-        const int64_t e1 = (b + 1 == grid) ? g.numel : x1 / g.eb / g.vec * g.vec;
+        const int64_t be = batch_elems(g.dt);
+        const int64_t e0 = x0 / g.eb / be * be;
+        const int64_t e1 = (b + 1 == grid) ? g.numel : x1 / g.eb / be * be;
         if (e1 <= e0) continue;
         if (e1 - e0 > kMaxPiece) return fail(NMV_EINVAL, "case too large for the no-allocation scratch");
         Piece &pc = g_na_pieces[n_pieces++];
@@ -848,7 +854,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
       if (need <= want) break;
       guess = need;
     }
-    if (smem > S->smem_optin)
+    if (smem + ring_bytes(nin) > S->smem_optin)
       return fail(NMV_EINVAL, "localisation maps need more shared memory than the device has");
     size_t &set = S->smem_set[g.dt][gi];
     if (smem > set) {
@@ -906,16 +912,20 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   if (grid > 0) {
     e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (const int64_t *)(W + sz_cases + sz_pieces), 0,
-                    (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr);
+                    (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr,
+                    (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   e = launch_finalize(d_case, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc), W + o_out,
                       1, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   const uint8_t *ob = W + o_out + kCallHeader;
+  uint32_t kerr = 0;
   e = cudaMemcpyAsync(&g_na_head, ob, sizeof(OutHeader), cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(&kerr, W + o_out + kCallErrOff, 4, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (result header)");
+  if (kerr != 0) return fail(NMV_ECUDA, "scan kernel: a bulk copy into shared memory did not complete in time");
   if (g_na_head.max_abs > 0.0 && g_na_head.max_abs < 0x1p-38) {
     // the fp64 SSE re-pass for cases whose differences are all tiny
     double *dst = (double *)(W + o_out + kCallHeader + offsetof(OutHeader, sse));

@@ -2,6 +2,7 @@
 // the kernels (nmv_scan.cuh, nmv_finalize.cu).  Not part of the public ABI.
 #pragma once
 
+#include <cstddef>
 #include <cstdint>
 
 #include "../../include/nmv.h"
@@ -20,7 +21,10 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kFinThreads = 256;          // threads per block of the finalize kernel
 constexpr int64_t kHistCap = 8192;        // smem tile-histogram window (bins)
 constexpr int64_t kProfCap = 4096;        // smem row / column profile (bins each)
-constexpr int64_t kMaxPiece = int64_t(1) << 30;  // elements per piece (int32 smem counters)
+// Elements per piece at most: a multiple of every batch size (so piece
+// boundaries stay on batch boundaries), small enough for int32 shared-memory
+// counters and 32-bit byte offsets within a piece.
+constexpr int64_t kMaxPiece = int64_t(3) << 27;
 
 // Element size in bytes and elements per 16-byte vector.
 NMV_HD int elem_bytes(int dt) { return (dt == NMV_F16 || dt == NMV_BF16) ? 2 : 4; }
@@ -102,12 +106,30 @@ struct OutHeader {
   int64_t pad[3];
 };
 
-// Steps of one warp per batch, and elements per batch.
-constexpr int kUnroll = 4;
-NMV_HD int64_t batch_elems(int dt) { return (int64_t)32 * vec_elems(dt) * kUnroll; }
+// Warp steps (32 lanes x 16 bytes of each tensor) per batch, and elements
+// per batch.  A batch is the unit of the first-K counts and of the warps'
+// shared-memory rings.
+constexpr int kSteps = 3;
+constexpr int kBatchBytes = 32 * 16 * kSteps;  // one tensor's bytes of a batch
+NMV_HD int64_t batch_elems(int dt) { return (int64_t)32 * vec_elems(dt) * kSteps; }
 NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt) {
   const int64_t be = batch_elems(dt);
   return (end - begin + be - 1) / be;
+}
+
+// Ring of each scan warp, by input class (0, 1 or -1 = several inputs read
+// from global memory): stages, tensors staged per batch, and the dynamic
+// shared memory of all rings of a block (stage data, then one 8-byte
+// mbarrier per stage).
+#ifdef __CUDACC__
+#define NMV_CHD __host__ __device__ constexpr
+#else
+#define NMV_CHD constexpr
+#endif
+NMV_CHD int ring_stages(int nin) { return nin == 1 ? 2 : 3; }
+NMV_CHD int ring_streams(int nin) { return nin == 1 ? 3 : 2; }
+NMV_CHD size_t ring_bytes(int nin) {
+  return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * kBatchBytes + 8);
 }
 
 }  // namespace nmv

@@ -55,7 +55,9 @@
 
 namespace nmv {
 
-constexpr int kFlushBatches = 8;
+// The SSE's float-float pairs go to fp64 every kFlushBatches batches (about
+// 32 warp steps, at most 128 terms per pair).
+constexpr int kFlushBatches = (32 + kSteps - 1) / kSteps;
 constexpr float kHuge = 0x1p56f;
 constexpr float kMarginLo = 1.0f - 0x1p-20f;
 
@@ -87,9 +89,9 @@ __device__ __forceinline__ uint32_t ld_one(const void *base, int64_t i) {
   }
 }
 
-__device__ __forceinline__ uint32_t ld_relaxed(const uint32_t *p) {
-  uint32_t v;
-  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p));
+__device__ __forceinline__ uint64_t ld_relaxed64(const uint32_t *p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p));
   return v;
 }
 
@@ -243,11 +245,14 @@ __device__ __forceinline__ T warp_reduce(T v, Op op) {
 // Piece-constant data, in shared memory.
 struct PieceSh {
   CaseDesc cd;
+  int64_t pbegin;  // the piece's first element
   int64_t tr0, tc0;
   int32_t wr, wc, prof_smem, pad;
   int32_t *sh_cls, *sh_row, *sh_col, *sh_hist;
   unsigned long long *g_hist, *g_row, *g_col;
   uint32_t *g_thr;
+  uint32_t *cta_thr;  // [2] the block's view of the case-wide maxima (float bits), in shared memory
+  int32_t *sh_eq;  // [kThreads][NMV_MAX_INPUTS] pass-through counts of the exact paths (inputs only)
   unsigned long long *stats;  // [exact steps, exact abs, exact rel, exact predicate, light steps,
                               //  SM cycles in exact steps, SM cycles in light steps]
 };
@@ -264,7 +269,6 @@ struct LaneSh {
   float r_lo;  // an fp32 strictly below the held |d|/|r| by the 2^-20 margin (-1: none)
   int32_t a_x, r_x;
   uint32_t cacc, racc;
-  int32_t eq[NMV_MAX_INPUTS];
 };
 
 // Warp-uniform state of a batch sweep, in shared memory.
@@ -274,6 +278,7 @@ struct WarpSh {
   float ga, gr;       // the case-wide part at the last merge (-1: none)
   uint32_t pubA, pubR;
   int64_t mism;       // mismatches so far in this batch
+  unsigned long long st[7];  // the warp's profile counters (layout of PieceSh::stats)
 };
 
 __device__ __forceinline__ float pub_thr(uint32_t bits) {
@@ -286,7 +291,21 @@ __device__ __forceinline__ void merge_thr(float wA, float wR, float ga, float gr
   tR = fmaxf(wR, gr);
 }
 
-// fl32 round-down lower bounds of a lane's maxima (-1 when none held).
+// fl32(|s| / |r|) for |r| != 0, within 2^-22 of the quotient: a fast
+// reciprocal in the normal range, an IEEE division otherwise.
+__device__ __forceinline__ float rel32(float as, float ar) {
+  if (ar > 0x1p-125f && ar < 0x1p125f) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(ar));
+    return __fmul_rn(as, r);
+  }
+  return __fdiv_rn(as, ar);
+}
+
+// A strict fp32 lower bound of n / d (n >= 0, d > 0): rel32 is within 2^-22.
+__device__ __forceinline__ float quot_lb(float n, float d) { return __fmul_rz(rel32(n, d), 1.0f - 0x1p-21f); }
+
+// fp32 lower bounds of a lane's maxima (-1 when none held).
 __device__ __forceinline__ float abs_lb(const LaneSh *L) {
   if (L->a_i == INT64_MAX) return -1.f;
   return L->a_x ? L->a_f : __double2float_rd(L->a_v);
@@ -294,7 +313,7 @@ __device__ __forceinline__ float abs_lb(const LaneSh *L) {
 
 __device__ __forceinline__ float rel_lb(const LaneSh *L) {
   if (L->r_i == INT64_MAX) return -1.f;
-  return L->r_x ? __fdiv_rd(L->r_n, L->r_d) : __double2float_rd(L->r_v);
+  return L->r_x ? quot_lb(L->r_n, L->r_d) : __double2float_rd(L->r_v);
 }
 
 // The lane's maxima as fp64 (for the reduction at the end of a piece).
@@ -369,7 +388,7 @@ __device__ __forceinline__ bool offer_rel(LaneSh *L, float as, float ar, bool ex
         L->r_n = as;
         L->r_d = ar;
         L->r_i = idx;
-        L->r_lo = __fmul_rz(__fdiv_rd(as, ar), kMarginLo);
+        L->r_lo = __fmul_rz(quot_lb(as, ar), kMarginLo);
       }
       return win;
     }
@@ -387,40 +406,71 @@ __device__ __forceinline__ bool offer_rel(LaneSh *L, float as, float ar, bool ex
   return win;
 }
 
-// fl32(|s| / |r|) for |r| != 0, within 2^-23 of the quotient: a fast
-// reciprocal in the normal range, an IEEE division otherwise.
-__device__ __forceinline__ float rel32(float as, float ar) {
-  if (ar > 0x1p-125f && ar < 0x1p125f) {
-    float r;
-    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(ar));
-    return __fmul_rn(as, r);
+// Order of two candidates for the maximum of |d|/|r| (true when the first,
+// at a higher index, is strictly larger): exact fractions compared exactly,
+// otherwise the fp64 quotients.
+__device__ __forceinline__ bool rel_gt(float as1, float ar1, bool ex1, double a1, double r1, float as2, float ar2,
+                                       bool ex2, double a2, double r2, unsigned &n_fp64) {
+  if (ex1 && ex2) {
+    const int c = frac_cmp(as1, ar1, as2, ar2);
+    if (c != 2) return c > 0;
   }
-  return __fdiv_rn(as, ar);
+  ++n_fp64;
+  const double q1 = __ddiv_rn(ex1 ? (double)as1 : a1, ex1 ? (double)ar1 : r1);
+  const double q2 = __ddiv_rn(ex2 ? (double)as2 : a2, ex2 ? (double)ar2 : r2);
+  return __double_as_longlong(q1) > __double_as_longlong(q2);
 }
 
 // ------------------------------------------------------------- slow path
 // Localisation maps and the batch's mismatch count for one step: bit k of
-// `mask` is element idx0 + k of this lane.  Row, column and tile
-// coordinates are found once per lane and then advanced element by element.
-__device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_t mask, int64_t idx0) {
+// `mask` is element idx0 + k of this lane.  When every lane's mismatches lie
+// in one row and one tile, and all lanes' in the same ones, the warp adds
+// its total to that histogram bin and row bin with one atomic each;
+// otherwise each lane walks its elements, merging runs of equal bins.
+__device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_t mask, int64_t idx0, int V) {
   const int lane = threadIdx.x & 31;
   const int total = __reduce_add_sync(0xffffffffu, (unsigned)__popc(mask));
   if (total == 0) return;
   const int64_t mism0 = W->mism;
   __syncwarp();
   if (lane == 0) W->mism = mism0 + total;
-  if (mask == 0) return;
   const CaseDesc &cd = P->cd;
   const uint64_t N = cd.dN.d, th = cd.dth.d, tw = cd.dtw.d;
-  uint64_t row = div_q((uint64_t)idx0, N, cd.dN.m);
-  uint64_t col = (uint64_t)idx0 - row * N;
-  uint64_t tr = div_q(row, th, cd.dth.m);
-  uint64_t rp = row - tr * th;
-  uint64_t tc = div_q(col, tw, cd.dtw.m);
-  uint64_t cp = col - tc * tw;
+  uint64_t row = 0, col = 0, tr = 0, rp = 0, tc = 0, cp = 0;
+  int64_t hbin = -1;
+  bool single = false;
+  if (mask) {
+    row = div_q((uint64_t)idx0, N, cd.dN.m);
+    col = (uint64_t)idx0 - row * N;
+    tr = div_q(row, th, cd.dth.m);
+    rp = row - tr * th;
+    tc = div_q(col, tw, cd.dtw.m);
+    cp = col - tc * tw;
+    hbin = P->wr > 0 ? ((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0) : (int64_t)(tr * (uint64_t)cd.GC + tc);
+    single = col + V <= N && cp + V <= tw;
+  }
+  const unsigned act = __ballot_sync(0xffffffffu, mask != 0);
+  const int lead = __ffs(act) - 1;
+  const int64_t hb_l = __shfl_sync(0xffffffffu, hbin, lead);
+  const uint64_t rp_l = __shfl_sync(0xffffffffu, rp, lead);
+  if (__all_sync(0xffffffffu, mask == 0 || (single && hbin == hb_l && rp == rp_l))) {
+    if (lane == lead) {
+      if (P->wr > 0) atomicAdd(&P->sh_hist[hbin], total);
+      else atomicAdd(&P->g_hist[hbin], (unsigned long long)total);
+      if (P->prof_smem) atomicAdd(&P->sh_row[rp], total);
+      else atomicAdd(&P->g_row[rp], (unsigned long long)total);
+    }
+    for (uint32_t m = mask; m; m &= m - 1) {
+      const int k = __ffs(m) - 1;
+      if (P->prof_smem) atomicAdd(&P->sh_col[cp + k], 1);
+      else atomicAdd(&P->g_col[cp + k], 1ull);
+    }
+    return;
+  }
+  if (mask == 0) return;
   uint32_t m = mask;
   int kprev = 0;
-  int64_t hbin = -1, rbin = -1;
+  int64_t hb_cur = -1, rbin = -1;
   int hcnt = 0, rcnt = 0;
   while (m) {
     const int k = __ffs(m) - 1;
@@ -444,12 +494,12 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
     kprev = k;
     const int64_t hb = P->wr > 0 ? ((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0)
                                  : (int64_t)(tr * (uint64_t)cd.GC + tc);
-    if (hb != hbin) {
+    if (hb != hb_cur) {
       if (hcnt) {
-        if (P->wr > 0) atomicAdd(&P->sh_hist[hbin], hcnt);
-        else atomicAdd(&P->g_hist[hbin], (unsigned long long)hcnt);
+        if (P->wr > 0) atomicAdd(&P->sh_hist[hb_cur], hcnt);
+        else atomicAdd(&P->g_hist[hb_cur], (unsigned long long)hcnt);
       }
-      hbin = hb;
+      hb_cur = hb;
       hcnt = 0;
     }
     ++hcnt;
@@ -465,8 +515,8 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
     if (P->prof_smem) atomicAdd(&P->sh_col[cp], 1);
     else atomicAdd(&P->g_col[cp], 1ull);
   }
-  if (P->wr > 0) atomicAdd(&P->sh_hist[hbin], hcnt);
-  else atomicAdd(&P->g_hist[hbin], (unsigned long long)hcnt);
+  if (P->wr > 0) atomicAdd(&P->sh_hist[hb_cur], hcnt);
+  else atomicAdd(&P->g_hist[hb_cur], (unsigned long long)hcnt);
   if (P->prof_smem) atomicAdd(&P->sh_row[rbin], rcnt);
   else atomicAdd(&P->g_row[rbin], (unsigned long long)rcnt);
 }
@@ -486,12 +536,17 @@ __device__ __forceinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpS
   if (lane == 0) {
     W->wA = fa < 0.f ? -1.f : (fa > 0.f ? __uint_as_float(__float_as_uint(fa) - 1u) : 0.f);
     W->wR = fr < 0.f ? -1.f : __fmul_rz(fr, kMarginLo);
+    // Publish improvements to the block, and to the case when they raise
+    // the block's value (the block's value came from the case or from a
+    // warp that published it there).
     if (fa > 0.f && __float_as_uint(fa) > W->pubA) {
-      atomicMax(&P->g_thr[0], __float_as_uint(fa));
+      if (atomicMax(&P->cta_thr[0], __float_as_uint(fa)) < __float_as_uint(fa))
+        atomicMax(&P->g_thr[0], __float_as_uint(fa));
       W->pubA = __float_as_uint(fa);
     }
     if (fr > 0.f && __float_as_uint(fr) > W->pubR) {
-      atomicMax(&P->g_thr[1], __float_as_uint(fr));
+      if (atomicMax(&P->cta_thr[1], __float_as_uint(fr)) < __float_as_uint(fr))
+        atomicMax(&P->g_thr[1], __float_as_uint(fr));
       W->pubR = __float_as_uint(fr);
     }
     merge_thr(W->wA, W->wR, W->ga, W->gr, W->tA, W->tR);
@@ -499,17 +554,19 @@ __device__ __forceinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpS
   __syncwarp();
 }
 
-__device__ __forceinline__ void count_stats(const PieceSh *P, int slot, long long t0, unsigned n_abs,
-                                            unsigned n_rel, unsigned n_pred) {
+// Profile counters of one exact (slot 0) or light (slot 1) step, kept per
+// warp and added to the call's counters once per piece.
+__device__ __forceinline__ void count_stats(WarpSh *W, int slot, long long t0, unsigned n_abs, unsigned n_rel,
+                                            unsigned n_pred) {
   n_abs = __reduce_add_sync(0xffffffffu, n_abs);
   n_rel = __reduce_add_sync(0xffffffffu, n_rel);
   n_pred = __reduce_add_sync(0xffffffffu, n_pred);
   if ((threadIdx.x & 31) == 0) {
-    atomicAdd(&P->stats[slot == 0 ? 0 : 4], 1ull);
-    atomicAdd(&P->stats[slot == 0 ? 5 : 6], (unsigned long long)(clock64() - t0));
-    atomicAdd(&P->stats[1], (unsigned long long)n_abs);
-    atomicAdd(&P->stats[2], (unsigned long long)n_rel);
-    atomicAdd(&P->stats[3], (unsigned long long)n_pred);
+    W->st[slot == 0 ? 0 : 4] += 1;
+    W->st[slot == 0 ? 5 : 6] += (unsigned long long)(clock64() - t0);
+    W->st[1] += n_abs;
+    W->st[2] += n_rel;
+    W->st[3] += n_pred;
   }
 }
 
@@ -592,17 +649,22 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
   // Exact evaluation of the screened candidates.  abs: values below the
   // fp32 predecessor of the step's largest |s| are strictly smaller than it.
   // rel: fl32(|s| / |r|) is within 2^-22 of the quotient, so values below
-  // (1 - 2^-20) of the largest are strictly smaller.
+  // (1 - 2^-20) of the largest are strictly smaller.  The lane's best of
+  // each kind (largest, lowest index on ties) is chosen in registers and
+  // offered once.
   bool changed = false;
   if (candA | candR) {
     const float fA = mA > 0.f ? __uint_as_float(__float_as_uint(mA) - 1u) : mA;
     const float fR = __fmul_rz(mR, kMarginLo);
+    int kA = -1, kR = -1;
+    float bA = 0.f, bRn = 0.f, bRd = 1.f, bRq = 0.f;
+    bool xA = true, xR = true;
+    double aA = 0.0, aR = 0.0, rR = 0.0;
 #pragma unroll
     for (int k = 0; k < V; ++k) {
       const bool ca = ((candA >> k) & 1u) && fabsf(s[k]) >= fA;
       const bool cr = ((candR >> k) & 1u) && rel[k] >= fR;
       if (!(ca || cr)) continue;
-      const int64_t idx = idx0 + k;
       const float as = fabsf(s[k]);
       const uint32_t rb = vbits<DT>(rv, k);
       const float ar = fabsf(to_f32<DT>(rb));
@@ -610,18 +672,40 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
       if constexpr (Tr<DT>::kInt) exact = exact && as < 0x1p24f && ar < 0x1p24f;
       // fl64(|c - r|) from the widened values when c - r is not exact in
       // fp32 (this also covers an fp32 overflow of c - r).
-      double a64 = 0.0;
+      double a64 = (double)as;
       if (!exact) {
         ++n_abs;
         a64 = fabs(__dsub_rn(to_f64<DT>(vbits<DT>(cv, k)), to_f64<DT>(rb)));
       }
-      if (ca) changed |= offer_abs(L, as, exact, a64, idx);
-      if (cr) changed |= offer_rel(L, as, ar, exact, a64, fabs(to_f64<DT>(rb)), rel[k], idx, n_rel);
+      if (ca) {
+        const bool better = kA < 0 || ((exact && xA) ? as > bA
+                                                      : __double_as_longlong(a64) > __double_as_longlong(aA));
+        if (better) {
+          kA = k;
+          bA = as;
+          xA = exact;
+          aA = a64;
+        }
+      }
+      if (cr) {
+        const double r64 = fabs(to_f64<DT>(rb));
+        if (kR < 0 || rel_gt(as, ar, exact, a64, r64, bRn, bRd, xR, aR, rR, n_rel)) {
+          kR = k;
+          bRn = as;
+          bRd = ar;
+          bRq = rel[k];
+          xR = exact;
+          aR = a64;
+          rR = r64;
+        }
+      }
     }
+    if (kA >= 0) changed |= offer_abs(L, bA, xA, aA, idx0 + kA);
+    if (kR >= 0) changed |= offer_rel(L, bRn, bRd, xR, aR, rR, bRq, idx0 + kR, n_rel);
   }
-  if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0);
+  if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0, V);
   if (__any_sync(0xffffffffu, changed)) refresh(P, L, W);
-  if (P->stats) count_stats(P, 0, t_start, n_abs, n_rel, n_pred);
+  if (P->stats) count_stats(W, 0, t_start, n_abs, n_rel, n_pred);
   return sse;
 }
 
@@ -662,29 +746,45 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
   bool changed = false;
   unsigned n_rel = 0;
   if (candA | candR) {
+    // every element here is finite with c - r exact: the lane's best of
+    // each kind is chosen in registers (exact comparisons) and offered once
     const float fA = mA > 0.f ? __uint_as_float(__float_as_uint(mA) - 1u) : mA;
     const float fR = __fmul_rz(mR, kMarginLo);
+    int kA = -1, kR = -1;
+    float bA = 0.f, bRn = 0.f, bRd = 1.f, bRq = 0.f;
+    bool xR = true;
+    double rR = 0.0;
 #pragma unroll
     for (int k = 0; k < V; ++k) {
       const float as = fabsf(s[k]);
-      const bool ca = ((candA >> k) & 1u) && as >= fA;
-      const bool cr = ((candR >> k) & 1u) && rel[k] >= fR;
-      const int64_t idx = idx0 + k;
-      if (ca) changed |= offer_abs(L, as, true, 0.0, idx);
-      if (cr) {
+      if (((candA >> k) & 1u) && as >= fA && (kA < 0 || as > bA)) {
+        kA = k;
+        bA = as;
+      }
+      if (((candR >> k) & 1u) && rel[k] >= fR) {
         const uint32_t rb = vbits<DT>(rv, k);
         const float ar = fabsf(to_f32<DT>(rb));
         const bool exact = !Tr<DT>::kInt || ar < 0x1p24f;
-        changed |= offer_rel(L, as, ar, exact, (double)as, fabs(to_f64<DT>(rb)), rel[k], idx, n_rel);
+        const double r64 = fabs(to_f64<DT>(rb));
+        if (kR < 0 || rel_gt(as, ar, exact, (double)as, r64, bRn, bRd, xR, (double)bRn, rR, n_rel)) {
+          kR = k;
+          bRn = as;
+          bRd = ar;
+          bRq = rel[k];
+          xR = exact;
+          rR = r64;
+        }
       }
     }
+    if (kA >= 0) changed |= offer_abs(L, bA, true, 0.0, idx0 + kA);
+    if (kR >= 0) changed |= offer_rel(L, bRn, bRd, xR, (double)bRn, rR, bRq, idx0 + kR, n_rel);
   }
   if constexpr (!Tr<DT>::kInt) {
 #pragma unroll
     for (int k = 0; k < V; k += 2) ff_pair<Tr<DT>::EB == 4>(sse, make_float2(s[k], s[k + 1]));
   }
   if (__any_sync(0xffffffffu, changed)) refresh(P, L, W);
-  if (P->stats) count_stats(P, 1, t_start, 0, n_rel, 0);
+  if (P->stats) count_stats(W, 1, t_start, 0, n_rel, 0);
   return sse;
 }
 
@@ -704,7 +804,7 @@ __device__ __noinline__ SseAcc tail_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     if constexpr (NIN != 0) {
       for (int j = 0; j < cd.n_elig; ++j) {
         const uint32_t xb = ld_one<EB>(cd.in_ptr[j], i);
-        L->eq[j] += (cb == xb) & (rb != xb);
+        P->sh_eq[threadIdx.x * NMV_MAX_INPUTS + j] += (cb == xb) & (rb != xb);
       }
     }
     if constexpr (EB == 2) {
@@ -732,8 +832,67 @@ __device__ __noinline__ void eq_generic(const PieceSh *P, LaneSh *L, const uint4
       const uint32_t xb = vbits<DT>(x, k);
       add += (vbits<DT>(cv, k) == xb) & (vbits<DT>(rv, k) != xb);
     }
-    L->eq[j] += add;
+    P->sh_eq[threadIdx.x * NMV_MAX_INPUTS + j] += add;
   }
+}
+
+// -------------------------------------------------- the shared-memory ring
+// Each warp streams its own batches into a private ring of shared-memory
+// stages with bulk copies (cp.async.bulk, completion counted in bytes on an
+// mbarrier per stage), kRingStages(nin) - 1 batches ahead of the one it is
+// checking.  Memory parallelism then needs no registers, and the checking
+// loop stays small.
+__device__ __forceinline__ uint32_t smem_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Wait for a stage's copies; gives up after kWaitNs (then the call reports
+// an error instead of hanging the GPU).
+constexpr uint64_t kWaitNs = 2000000000ull;
+
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity) {
+  const uint64_t t0 = global_ns();
+  while (!mbar_try_wait(bar, parity))
+    if (global_ns() - t0 > kWaitNs) return false;
+  return true;
+}
+
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_addr(dst)),
+               "l"(src), "r"(bytes), "r"(smem_addr(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ uint4 lds_v4(const void *p) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(smem_addr(p)));
+  return v;
 }
 
 // ------------------------------------------------------------- fast step
@@ -747,6 +906,7 @@ struct Regs {
   float tRq;     // min(tR, 1/4): also proves c - r exact (see the file comment)
   float ga, gr;  // copy of WarpSh::ga / gr
   float lo_r, lo_a;
+  bool track_c, track_r;  // warp-uniform: the constant / all-zero accumulators still matter
 };
 
 template <int NIN>
@@ -758,21 +918,18 @@ __device__ __forceinline__ void reload_thr(Regs<NIN> &R, const WarpSh *W) {
 
 template <int DT, int NIN>
 __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const uint4 &cv,
-                                     const uint4 &rv, const uint4 *xv, int64_t e) {
+                                     const uint4 &rv, const uint4 &xv, uint32_t erel) {
   constexpr int V = Tr<DT>::V;
-  R.cacc |= (cv.x ^ R.cpat) | (cv.y ^ R.cpat) | (cv.z ^ R.cpat) | (cv.w ^ R.cpat);
-  R.racc |= (rv.x ^ R.rpat) | (rv.y ^ R.rpat) | (rv.z ^ R.rpat) | (rv.w ^ R.rpat);
-  if constexpr (NIN > 0) {
+  if (R.track_c) R.cacc |= (cv.x ^ R.cpat) | (cv.y ^ R.cpat) | (cv.z ^ R.cpat) | (cv.w ^ R.cpat);
+  if (R.track_r) R.racc |= (rv.x ^ R.rpat) | (rv.y ^ R.rpat) | (rv.z ^ R.rpat) | (rv.w ^ R.rpat);
+  if constexpr (NIN == 1) {
 #pragma unroll
-    for (int j = 0; j < NIN; ++j) {
-#pragma unroll
-      for (int k = 0; k < V; ++k) {
-        const uint32_t xb = vbits<DT>(xv[j], k);
-        R.eq[j] += (vbits<DT>(cv, k) == xb) & (vbits<DT>(rv, k) != xb);
-      }
+    for (int k = 0; k < V; ++k) {
+      const uint32_t xb = vbits<DT>(xv, k);
+      R.eq[0] += (vbits<DT>(cv, k) == xb) & (vbits<DT>(rv, k) != xb);
     }
   } else if constexpr (NIN < 0) {
-    eq_generic<DT>(P, L, cv, rv, e);
+    eq_generic<DT>(P, L, cv, rv, P->pbegin + erel);
   }
   bool hard, other;
   if constexpr (Tr<DT>::kInt) {
@@ -785,13 +942,18 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   } else {
     float s[V];
     hard = false;
+    const float2 m1 = make_float2(-1.f, -1.f);
 #pragma unroll
-    for (int k = 0; k < V; ++k) {
-      const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
-      s[k] = __fsub_rn(cf, rf);
-      const float a = __fmaf_rz(R.lo_r, fabsf(rf), R.lo_a);
-      const float b = __fmul_rz(R.tRq, fabsf(rf));
-      hard |= !(fabsf(s[k]) <= min3f(a, b, R.tA));
+    for (int k = 0; k < V; k += 2) {
+      const float2 c2 = make_float2(vdec<DT>(cv, k), vdec<DT>(cv, k + 1));
+      const float2 r2 = make_float2(vdec<DT>(rv, k), vdec<DT>(rv, k + 1));
+      const float2 s2 = __ffma2_rn(r2, m1, c2);  // fl(c - r), one rounding
+      s[k] = s2.x;
+      s[k + 1] = s2.y;
+      const float a0 = __fmaf_rz(R.lo_r, fabsf(r2.x), R.lo_a), a1 = __fmaf_rz(R.lo_r, fabsf(r2.y), R.lo_a);
+      const float b0 = __fmul_rz(R.tRq, fabsf(r2.x)), b1 = __fmul_rz(R.tRq, fabsf(r2.y));
+      hard |= !(fabsf(s2.x) <= min3f(a0, b0, R.tA));
+      hard |= !(fabsf(s2.y) <= min3f(a1, b1, R.tA));
     }
     if (!__any_sync(0xffffffffu, hard)) {
 #pragma unroll
@@ -809,50 +971,129 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
       other |= !(fabsf(s[k]) <= min3f(a, __fmul_rz(0.25f, fabsf(rf)), kHuge));
     }
   }
-  if (__any_sync(0xffffffffu, other)) R.sse = slow_step<DT>(P, L, W, cv, rv, e, V, R.sse);
-  else R.sse = light_step<DT>(P, L, W, cv, rv, e, R.sse);
+  if (__any_sync(0xffffffffu, other)) R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
+  else R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
   reload_thr(R, W);
 }
 
-// Sweep this warp's batches of a piece (each batch_elems elements; the last
-// one may be shorter), writing each batch's mismatch count.  In round r the
-// block's warps take batches r*kWarps .. r*kWarps + kWarps - 1, warp w the
-// one at offset (w - r) mod kWarps: a warp's batches stay in ascending order,
-// and a pattern that repeats every few batches (a faulty column band, say)
-// spreads over all warps instead of landing on the same ones.
+// The j-th batch of warp w in a piece of nb batches is batch j * kWarps +
+// ((w - j) mod kWarps): in round j the block's warps take batches
+// j * kWarps .. j * kWarps + kWarps - 1.  A warp's batches stay in ascending
+// order, and a pattern that repeats every few batches (a faulty column band,
+// say) spreads over all warps instead of landing on the same ones.
+__device__ __forceinline__ int64_t warp_batch(int64_t j, int warp) {
+  return j * kWarps + (int64_t)(((warp - (int)(j % kWarps)) + kWarps) % kWarps);
+}
+
+// Number of batches warp w takes in a piece of nb batches (the j with
+// warp_batch(j, w) < nb).
+__device__ __forceinline__ int64_t warp_batches(int64_t nb, int warp) {
+  const int64_t J = nb / kWarps;
+  const int last = ((warp - (int)(J % kWarps)) % kWarps + kWarps) % kWarps;
+  return J + (last < nb % kWarps ? 1 : 0);
+}
+
+// Issue the copies of one batch, at byte offset `off` of the piece and with
+// `bytes` (whole steps only) per tensor, into a ring stage (lane 0 only).  A
+// ragged rest and the buffers of a case that is not 16-byte aligned
+// (bytes = 0) are read from global memory by tail_step.
+template <int NIN>
+__device__ __forceinline__ void ring_issue(const char *c, const char *r, const char *x, uint32_t off,
+                                           uint32_t bytes, uint8_t *stage, uint64_t *bar) {
+  mbar_arrive_tx(bar, bytes * (NIN == 1 ? 3u : 2u));
+  if (bytes) {
+    bulk_load(stage, c + off, bytes, bar);
+    bulk_load(stage + kBatchBytes, r + off, bytes, bar);
+    if constexpr (NIN == 1) bulk_load(stage + 2 * kBatchBytes, x + off, bytes, bar);
+  }
+}
+
+// Position of a warp in its ring: the stage it checks next and that
+// stage's mbarrier phase.  Carried across pieces.
+struct RingPos {
+  uint32_t stage, phase;
+};
+
+// Sweep this warp's batches of a piece (each batch_elems elements; only a
+// case's last batch may be shorter) through its ring, writing each batch's
+// mismatch count.  Offsets within the piece are 32-bit (a piece holds at
+// most kMaxPiece elements).
 template <int DT, int NIN>
 __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
-                                      int32_t *batch_count) {
+                                      int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
+                                      uint32_t *err) {
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
-  constexpr int BATCH = STEP * kUnroll;
-  constexpr int NX = NIN > 0 ? NIN : 1;
+  constexpr int BATCH = STEP * kSteps;
+  constexpr uint32_t BB = BATCH * EB;  // bytes of one tensor's batch (kBatchBytes)
+  constexpr uint32_t NST = ring_stages(NIN);
+  constexpr int STAGE = ring_streams(NIN) * kBatchBytes;
+  constexpr int kPoll = kWarps;  // batches between a warp's readings of the case-wide maxima
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const CaseDesc &cd = P->cd;
-  const char *cp = (const char *)cd.cand;
-  const char *rp = (const char *)cd.ref;
-  const char *xp[NX];
-#pragma unroll
-  for (int j = 0; j < NX; ++j) xp[j] = (const char *)cd.in_ptr[j];
   const uint32_t *g_thr = P->g_thr;
-  const bool vec_ok = cd.vec_ok != 0;
-  const int64_t nb = (pc.end - pc.begin + BATCH - 1) / BATCH;
+  const uint32_t nb = (uint32_t)((pc.end - pc.begin + BATCH - 1) / BATCH);
+  const uint32_t nj = (uint32_t)warp_batches(nb, warp);
+  const uint32_t mag = Tr<DT>::kInt ? 0xffffffffu : (Tr<DT>::EB == 2 ? 0x7fff7fffu : 0x7fffffffu);
+  const uint32_t pbytes = (uint32_t)((pc.end - pc.begin) * EB);
+  // batches at byte offsets <= full_max are whole and staged (all batches
+  // but a case's last; none when the case is not 16-byte aligned)
+  const int64_t full_max = P->cd.vec_ok ? (int64_t)pbytes - BB : -1;
+  const char *src_c = (const char *)P->cd.cand + pc.begin * EB;
+  const char *src_r = (const char *)P->cd.ref + pc.begin * EB;
+  const char *src_x = NIN == 1 ? (const char *)P->cd.in_ptr[0] + pc.begin * EB : nullptr;
+  int32_t *bcount = batch_count + pc.batch_base;
+  // The j-th batch is j * kWarps + rot_j, rot_j = (warp - j) mod kWarps, so
+  // its offset advances by 7 batches, or by 15 when rot wraps from 0 to 7.
+  // Copies run NST - 1 batches ahead of the check.
+  uint32_t off_i = (uint32_t)warp * BB, rot_i = warp, j_i = 0, st_i = rp.stage;
+  auto issue_next = [&]() {
+    uint32_t bytes = 0;
+    if ((int64_t)off_i <= full_max) {
+      bytes = BB;
+    } else if (P->cd.vec_ok && off_i < pbytes) {
+      bytes = (pbytes - off_i) / (STEP * EB) * (STEP * EB);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    ring_issue<NIN>(src_c, src_r, src_x, off_i, bytes, ring + st_i * STAGE, bars + st_i);
+    off_i += (rot_i == 0 ? 15u : 7u) * BB;
+    rot_i = (rot_i - 1) & (kWarps - 1);
+    st_i = st_i + 1 == NST ? 0 : st_i + 1;
+    ++j_i;
+  };
+  if (lane == 0)
+    while (j_i < NST - 1 && j_i < nj) issue_next();
+  __syncwarp();
+  bool dead = false;
   int flush = 0;
-  for (int64_t r = 0; r * kWarps < nb; ++r) {
-    const int64_t b = r * kWarps + ((warp - r) % kWarps + kWarps) % kWarps;
-    if (b >= nb) continue;
-    const int64_t lo = pc.begin + b * BATCH;
-    const int64_t hi = lo + BATCH < pc.end ? lo + BATCH : pc.end;
-    const uint32_t gA = ld_relaxed(&g_thr[0]);
-    const uint32_t gR = ld_relaxed(&g_thr[1]);
+  uint32_t off = (uint32_t)warp * BB, rot = warp;
+  // The block's view of the case-wide maxima is read every batch; the case's
+  // own value is read by one warp of the block per batch round (each warp
+  // every kPoll batches, its load kPoll batches ahead of its use, so the L2
+  // latency hides and the hot word sees few readers).
+  uint64_t gAR = ld_relaxed64(g_thr);
+  const uint32_t lane_off = (uint32_t)lane * V;
+  for (uint32_t j = 0; j < nj; ++j) {
+    const uint32_t b = off / BB;
+    const uint32_t erel = off / EB;  // element offset of the batch in the piece
+    const uint32_t next = off + (rot == 0 ? 15u : 7u) * BB;
+    rot = (rot - 1) & (kWarps - 1);
+    if (lane == 0 && j_i < nj) issue_next();  // refills the stage released last batch
     if (lane == 0) W->mism = 0;
+    if ((j + warp) % kPoll == 0) {
+      if (lane == 0) {
+        atomicMax(&P->cta_thr[0], (uint32_t)gAR);
+        atomicMax(&P->cta_thr[1], (uint32_t)(gAR >> 32));
+      }
+      gAR = ld_relaxed64(g_thr);
+    }
     {
-      // Case-wide maxima published since the last batch: lane 0's reading,
-      // compared with the warp's register copy, so the branch is uniform.
-      const float ga = __shfl_sync(0xffffffffu, pub_thr(gA), 0);
-      const float gr = __shfl_sync(0xffffffffu, pub_thr(gR), 0);
-      if (__any_sync(0xffffffffu, ga > R.ga || gr > R.gr)) {
+      // lane 0's reading of the block's value, so the branch is uniform
+      uint64_t v = 0;
+      if (lane == 0) v = *(volatile const uint64_t *)P->cta_thr;
+      v = __shfl_sync(0xffffffffu, v, 0);
+      const float ga = pub_thr((uint32_t)v), gr = pub_thr((uint32_t)(v >> 32));
+      if (ga > R.ga || gr > R.gr) {
         __syncwarp();
         if (lane == 0) {
           W->ga = fmaxf(W->ga, ga);
@@ -866,79 +1107,100 @@ __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Re
       }
     }
     __syncwarp();
-    if (vec_ok && hi - lo == BATCH) {
-      uint4 cv[kUnroll], rv[kUnroll];
-      uint4 xv[NIN > 0 ? kUnroll : 1][NX];
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int64_t e = lo + (int64_t)u * STEP + lane * V;
-        cv[u] = ld_v4(cp + e * EB);
-        rv[u] = ld_v4(rp + e * EB);
-        if constexpr (NIN > 0) {
-#pragma unroll
-          for (int j = 0; j < NIN; ++j) xv[u][j] = ld_v4(xp[j] + e * EB);
-        }
-      }
-#pragma unroll
-      for (int u = 0; u < kUnroll; ++u)
-        step<DT, NIN>(P, L, W, R, cv[u], rv[u], xv[NIN > 0 ? u : 0], lo + (int64_t)u * STEP + lane * V);
-    } else {
-      int64_t base = lo;
-      if (vec_ok) {
-        for (; base + STEP <= hi; base += STEP) {
-          const int64_t e = base + lane * V;
-          const uint4 cv = ld_v4(cp + e * EB), rv = ld_v4(rp + e * EB);
-          uint4 xv[NX];
-          if constexpr (NIN > 0) {
-#pragma unroll
-            for (int j = 0; j < NIN; ++j) xv[j] = ld_v4(xp[j] + e * EB);
-          }
-          step<DT, NIN>(P, L, W, R, cv, rv, xv, e);
-        }
-      }
-      for (; base < hi; base += STEP) {
-        const int64_t e = base + lane * V;
-        int64_t n = hi - e;
-        n = n < 0 ? 0 : (n > V ? V : n);
-        R.sse = tail_step<DT, NIN>(P, L, W, e, (int)n, R.sse);
-        reload_thr(R, W);
+    const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
+    if (!dead && !mbar_try_wait(bars + rp.stage, rp.phase)) {
+      if (!mbar_wait_slow(bars + rp.stage, rp.phase)) {
+        dead = true;  // report, and stop waiting (the data of this call is void)
+        if (lane == 0) atomicOr(err, 1u);
       }
     }
-    __syncwarp();
-    if (lane == 0) batch_count[pc.batch_base + b] = (int32_t)W->mism;
+    if (++rp.stage == NST) {
+      rp.stage = 0;
+      rp.phase ^= 1u;
+    }
+    if ((int64_t)off <= full_max) {
+#pragma unroll
+      for (int u = 0; u < kSteps; ++u) {
+        const uint4 cv = lds_v4(stage + u * 512);
+        const uint4 rv = lds_v4(stage + kBatchBytes + u * 512);
+        uint4 xv = make_uint4(0, 0, 0, 0);
+        if constexpr (NIN == 1) xv = lds_v4(stage + 2 * kBatchBytes + u * 512);
+        step<DT, NIN>(P, L, W, R, cv, rv, xv, erel + u * STEP + lane_off);
+      }
+    } else {
+      // the case's last batch, or a case that is not 16-byte aligned
+      const uint32_t pel = pbytes / EB;  // elements in the piece
+      const uint32_t nfull = P->cd.vec_ok ? (pel - erel) / STEP : 0u;
+      for (int u = 0; u < kSteps; ++u) {
+        const uint32_t e = erel + u * STEP + lane_off;
+        if ((uint32_t)u < nfull) {
+          const uint4 cv = lds_v4(stage + u * 512);
+          const uint4 rv = lds_v4(stage + kBatchBytes + u * 512);
+          uint4 xv = make_uint4(0, 0, 0, 0);
+          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * kBatchBytes + u * 512);
+          step<DT, NIN>(P, L, W, R, cv, rv, xv, e);
+        } else if (erel + u * STEP < pel) {
+          const int n = e >= pel ? 0 : (pel - e > (uint32_t)V ? V : (int)(pel - e));
+          R.sse = tail_step<DT, NIN>(P, L, W, P->pbegin + e, n, R.sse);
+          reload_thr(R, W);
+        }
+      }
+    }
+    __syncwarp();  // every lane is done with the stage before it is refilled
+    if (lane == 0) bcount[b] = (int32_t)W->mism;
+    if (R.track_c | R.track_r) {
+      R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
+      R.track_r = R.track_r && !__any_sync(0xffffffffu, (R.racc & mag) != 0u);
+    }
     if (++flush == kFlushBatches) {
       sse_flush(R.sse);
       flush = 0;
     }
+    off = next;
   }
   sse_flush(R.sse);
 }
 
 // ------------------------------------------------------------ the kernel
-// Dynamic shared memory (int32 words): [0, 8) class counters (NaN/+Inf/-Inf
-// of c, of r, non-finite pairs), [8, 16) unused, then the row profile [th],
-// the column profile [tw] and the histogram window.
+// Dynamic shared memory: the warps' rings (ring_bytes(NIN): stage data, then
+// one mbarrier per stage), then int32 words: [0, 8) class counters
+// (NaN/+Inf/-Inf of c, of r, non-finite pairs), [8, 16) unused, the row
+// profile [th], the column profile [tw] and the histogram window.
 constexpr int kShHead = 16;
 
 template <int DT, int NIN>
 __global__ void __launch_bounds__(kThreads, 2)
     scan_kernel(const CaseDesc *__restrict__ cases, const Piece *__restrict__ pieces,
                 const int64_t *__restrict__ block_piece, int64_t piece_base, Partial *partials,
-                int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats) {
+                int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
-  extern __shared__ int32_t smem[];
+  constexpr int NST = ring_stages(NIN);
+  constexpr int STAGE = ring_streams(NIN) * kBatchBytes;
+  extern __shared__ __align__(128) uint8_t dsm[];
   __shared__ PieceSh P;
   __shared__ LaneSh lanes[kThreads];
   __shared__ WarpSh warps[kWarps];
   __shared__ Partial red[kWarps];
+  __shared__ int32_t sh_eq[NIN != 0 ? kThreads * NMV_MAX_INPUTS : 1];
+  __shared__ __align__(8) uint32_t cta_thr[2];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   LaneSh *L = &lanes[threadIdx.x];
   WarpSh *W = &warps[warp];
+  uint8_t *ring = dsm + (size_t)warp * NST * STAGE;
+  uint64_t *bars = (uint64_t *)(dsm + (size_t)kWarps * NST * STAGE) + warp * NST;
+  int32_t *smem = (int32_t *)(dsm + ring_bytes(NIN));
+  if (lane == 0) {
+    for (int s = 0; s < NST; ++s) mbar_init(bars + s);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();
+  RingPos rpos = {0u, 0u};
   const int64_t p0 = block_piece[blockIdx.x], p1 = block_piece[blockIdx.x + 1];
   for (int64_t p = p0; p < p1; ++p) {
     const Piece pc = pieces[p];
     if (threadIdx.x == 0) {
       P.cd = cases[pc.case_id];
+      P.pbegin = pc.begin;
       P.tr0 = pc.tr0;
       P.tc0 = pc.tc0;
       P.wr = pc.wr;
@@ -953,6 +1215,9 @@ __global__ void __launch_bounds__(kThreads, 2)
       P.g_row = (unsigned long long *)(o + P.cd.rowp_off);
       P.g_col = (unsigned long long *)(o + P.cd.colp_off);
       P.g_thr = g_thr + 2 * pc.case_id;
+      P.sh_eq = sh_eq;
+      P.cta_thr = cta_thr;
+      cta_thr[0] = cta_thr[1] = 0;
       P.stats = stats;
     }
     __syncthreads();
@@ -966,11 +1231,14 @@ __global__ void __launch_bounds__(kThreads, 2)
     L->r_lo = -1.f;
     L->cacc = 0;
     L->racc = 0;
-    for (int j = 0; j < NMV_MAX_INPUTS; ++j) L->eq[j] = 0;
+    if constexpr (NIN != 0) {
+      for (int j = 0; j < NMV_MAX_INPUTS; ++j) sh_eq[threadIdx.x * NMV_MAX_INPUTS + j] = 0;
+    }
     if (lane == 0) {
       W->tA = W->tR = W->wA = W->wR = W->ga = W->gr = -1.f;
       W->pubA = W->pubR = 0;
       W->mism = 0;
+      for (int k = 0; k < 7; ++k) W->st[k] = 0;
     }
     __syncthreads();
 
@@ -988,8 +1256,12 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.tA = R.tR = R.tRq = R.ga = R.gr = -1.f;
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
-    sweep<DT, NIN>(&P, L, W, R, pc, batch_count);
+    R.track_c = R.track_r = true;
+    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
     __syncwarp();
+    if (stats && lane == 0)
+      for (int k = 0; k < 7; ++k)
+        if (W->st[k]) atomicAdd(&stats[k], W->st[k]);
 
     // ---- lanes -> warps -> the piece's partial
     const Best a = best_warp(abs_best64(L)), r = best_warp(rel_best64(L));
@@ -999,7 +1271,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     int eqs[NMV_MAX_INPUTS];
 #pragma unroll
     for (int j = 0; j < NMV_MAX_INPUTS; ++j) {
-      int v = L->eq[j];
+      int v = 0;
+      if constexpr (NIN != 0) v = sh_eq[threadIdx.x * NMV_MAX_INPUTS + j];
       if constexpr (NIN > 0) {
         if (j < NIN) v += R.eq[j < NIN ? j : 0];
       }
@@ -1007,11 +1280,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     int64_t mism = 0;
     if (lane == 0) {
-      const int64_t nb = piece_batches(pc.begin, pc.end, DT);
-      for (int64_t rr = 0; rr * kWarps < nb; ++rr) {
-        const int64_t b = rr * kWarps + ((warp - rr) % kWarps + kWarps) % kWarps;
-        if (b < nb) mism += batch_count[pc.batch_base + b];
-      }
+      const int64_t nj = warp_batches(piece_batches(pc.begin, pc.end, DT), warp);
+      for (int64_t j = 0; j < nj; ++j) mism += batch_count[pc.batch_base + warp_batch(j, warp)];
       Partial &w = red[warp];
       w.cnt[0] = mism;
       w.best_abs = a.v;
@@ -1068,7 +1338,9 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
 }
 
-// Launch helpers of one element type (defined in nmv_scan_<dtype>.cu).
+// Launch helpers of one element type (defined in nmv_scan_<dtype>.cu).  The
+// `smem` they take is the localisation part of the dynamic shared memory;
+// they add the rings (ring_bytes).
 template <int DT>
 struct ScanOps {
   static cudaError_t prepare(int nin, size_t smem);
@@ -1076,40 +1348,46 @@ struct ScanOps {
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
-                            unsigned long long *stats);
+                            unsigned long long *stats, uint32_t *err);
 };
 
-#define NMV_DEFINE_SCAN_OPS(DT)                                                                     \
-  template <>                                                                                       \
-  cudaError_t ScanOps<DT>::prepare(int nin, size_t smem) {                                          \
-    if (nin == 0) return cudaFuncSetAttribute(scan_kernel<DT, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-    if (nin == 1) return cudaFuncSetAttribute(scan_kernel<DT, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-    return cudaFuncSetAttribute(scan_kernel<DT, -1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-  }                                                                                                 \
-  template <>                                                                                       \
-  int ScanOps<DT>::occupancy(int nin, size_t smem) {                                                \
-    int n = 0;                                                                                      \
-    cudaError_t e;                                                                                  \
-    if (nin == 0) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, scan_kernel<DT, 0>, kThreads, smem); \
-    else if (nin == 1) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, scan_kernel<DT, 1>, kThreads, smem); \
-    else e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, scan_kernel<DT, -1>, kThreads, smem); \
-    return e == cudaSuccess ? n : 0;                                                                \
-  }                                                                                                 \
-  template <>                                                                                       \
+#define NMV_SCAN_FN(DT, NIN) scan_kernel<DT, NIN>
+#define NMV_SCAN_SMEM(NIN, smem) ((int)((smem) + ring_bytes(NIN)))
+#define NMV_DEFINE_SCAN_OPS(DT)                                                                          \
+  template <>                                                                                            \
+  cudaError_t ScanOps<DT>::prepare(int nin, size_t smem) {                                               \
+    const cudaFuncAttribute A = cudaFuncAttributeMaxDynamicSharedMemorySize;                             \
+    if (nin == 0) return cudaFuncSetAttribute(NMV_SCAN_FN(DT, 0), A, NMV_SCAN_SMEM(0, smem));            \
+    if (nin == 1) return cudaFuncSetAttribute(NMV_SCAN_FN(DT, 1), A, NMV_SCAN_SMEM(1, smem));            \
+    return cudaFuncSetAttribute(NMV_SCAN_FN(DT, -1), A, NMV_SCAN_SMEM(-1, smem));                        \
+  }                                                                                                      \
+  template <>                                                                                            \
+  int ScanOps<DT>::occupancy(int nin, size_t smem) {                                                     \
+    int n = 0;                                                                                           \
+    cudaError_t e;                                                                                       \
+    if (nin == 0)                                                                                        \
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, NMV_SCAN_FN(DT, 0), kThreads, NMV_SCAN_SMEM(0, smem)); \
+    else if (nin == 1)                                                                                   \
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, NMV_SCAN_FN(DT, 1), kThreads, NMV_SCAN_SMEM(1, smem)); \
+    else                                                                                                 \
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, NMV_SCAN_FN(DT, -1), kThreads, NMV_SCAN_SMEM(-1, smem)); \
+    return e == cudaSuccess ? n : 0;                                                                     \
+  }                                                                                                      \
+  template <>                                                                                            \
   cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases, \
-                                  const Piece *pieces, const int64_t *block_piece, int64_t piece_base, \
+                                  const Piece *pieces, const int64_t *block_piece, int64_t piece_base,    \
                                   Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr, \
-                                  unsigned long long *stats) {                                      \
-    if (nin == 0)                                                                                   \
-      scan_kernel<DT, 0><<<grid, kThreads, smem, st>>>(cases, pieces, block_piece, piece_base, partials, \
-                                                       batch_count, out, g_thr, stats);             \
-    else if (nin == 1)                                                                              \
-      scan_kernel<DT, 1><<<grid, kThreads, smem, st>>>(cases, pieces, block_piece, piece_base, partials, \
-                                                       batch_count, out, g_thr, stats);             \
-    else                                                                                            \
-      scan_kernel<DT, -1><<<grid, kThreads, smem, st>>>(cases, pieces, block_piece, piece_base, partials, \
-                                                        batch_count, out, g_thr, stats);            \
-    return cudaGetLastError();                                                                      \
+                                  unsigned long long *stats, uint32_t *err) {                            \
+    if (nin == 0)                                                                                        \
+      NMV_SCAN_FN(DT, 0)<<<grid, kThreads, NMV_SCAN_SMEM(0, smem), st>>>(                               \
+          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+    else if (nin == 1)                                                                                   \
+      NMV_SCAN_FN(DT, 1)<<<grid, kThreads, NMV_SCAN_SMEM(1, smem), st>>>(                               \
+          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+    else                                                                                                 \
+      NMV_SCAN_FN(DT, -1)<<<grid, kThreads, NMV_SCAN_SMEM(-1, smem), st>>>(                              \
+          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+    return cudaGetLastError();                                                                           \
   }
 
 }  // namespace nmv
