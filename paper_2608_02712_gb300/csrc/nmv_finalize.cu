@@ -38,7 +38,7 @@ __device__ __forceinline__ bool pass_elem(const CaseDesc &cd, uint32_t cb, uint3
     if (as <= __fmaf_rz(cd.lo_r, ar, cd.lo_a)) return true;
     if (as > __fmaf_ru(cd.hi_r, ar, cd.hi_a)) return false;
   }
-  return pass64(to_f64<DT>(cb), to_f64<DT>(rb), cd.rtol, cd.atol);
+  return pass64_inl(to_f64<DT>(cb), to_f64<DT>(rb), cd.rtol, cd.atol);
 }
 
 // Exclusive block-wide prefix sum of a 64-bit v; *total = the block's sum.

@@ -144,12 +144,17 @@ __device__ __forceinline__ double to_f64(uint32_t b) {
 
 // The predicate in fp64, written out: (c == r) or (both finite and
 // fl(|fl(c - r)|) <= fl(atol + fl(rtol * |r|))).  No contraction.
-__device__ __forceinline__ bool pass64(double c, double r, double rtol, double atol) {
+__device__ __forceinline__ bool pass64_inl(double c, double r, double rtol, double atol) {
   if (c == r) return true;
   if (!(isfinite(c) && isfinite(r))) return false;
   const double err = fabs(__dsub_rn(c, r));
   const double allowed = __dadd_rn(atol, __dmul_rn(rtol, fabs(r)));
   return err <= allowed;
+}
+
+// The same, out of line (the scan's exact path keeps its code small).
+static __device__ __noinline__ bool pass64(double c, double r, double rtol, double atol) {
+  return pass64_inl(c, r, rtol, atol);
 }
 
 // --------------------------------------------------------------- the SSE
@@ -246,6 +251,7 @@ __device__ __forceinline__ T warp_reduce(T v, Op op) {
 struct PieceSh {
   CaseDesc cd;
   int64_t pbegin;  // the piece's first element
+  uint32_t next_batch;  // the piece's next unclaimed batch
   int64_t tr0, tc0;
   int32_t wr, wc, prof_smem, pad;
   int32_t *sh_cls, *sh_row, *sh_col, *sh_hist;
@@ -278,6 +284,8 @@ struct WarpSh {
   float ga, gr;       // the case-wide part at the last merge (-1: none)
   uint32_t pubA, pubR;
   int64_t mism;       // mismatches so far in this batch
+  int64_t mism_tot;   // mismatches in the warp's batches of this piece
+  uint32_t stage_b[4];  // batch held by each ring stage (kNoBatch: none)
   unsigned long long st[7];  // the warp's profile counters (layout of PieceSh::stats)
 };
 
@@ -422,6 +430,9 @@ __device__ __forceinline__ bool rel_gt(float as1, float ar1, bool ex1, double a1
 }
 
 // ------------------------------------------------------------- slow path
+static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask, uint64_t row, uint64_t col,
+                                                uint64_t tr, uint64_t rp, uint64_t tc, uint64_t cp);
+
 // Localisation maps and the batch's mismatch count for one step: bit k of
 // `mask` is element idx0 + k of this lane.  When every lane's mismatches lie
 // in one row and one tile, and all lanes' in the same ones, the warp adds
@@ -467,7 +478,15 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
     }
     return;
   }
-  if (mask == 0) return;
+  if (mask) record_lane(P, mask, row, col, tr, rp, tc, cp);
+}
+
+// The general case of record_step for one lane: walk its mismatches from
+// the coordinates of its first element, merging runs of equal bins.
+static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask, uint64_t row, uint64_t col,
+                                                uint64_t tr, uint64_t rp, uint64_t tc, uint64_t cp) {
+  const CaseDesc &cd = P->cd;
+  const uint64_t N = cd.dN.d, th = cd.dth.d, tw = cd.dtw.d;
   uint32_t m = mask;
   int kprev = 0;
   int64_t hb_cur = -1, rbin = -1;
@@ -528,7 +547,7 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
 //        (elements not above it are not larger than a maximum at a lower
 //        index of this warp);
 //   rel: fl_rd(max) (1 - 2^-20) rounded toward zero.
-__device__ __forceinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpSh *W) {
+static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpSh *W) {
   const int lane = threadIdx.x & 31;
   const float fa = warp_reduce(abs_lb(L), [](float x, float y) { return fmaxf(x, y); });
   const float fr = warp_reduce(rel_lb(L), [](float x, float y) { return fmaxf(x, y); });
@@ -976,23 +995,6 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   reload_thr(R, W);
 }
 
-// The j-th batch of warp w in a piece of nb batches is batch j * kWarps +
-// ((w - j) mod kWarps): in round j the block's warps take batches
-// j * kWarps .. j * kWarps + kWarps - 1.  A warp's batches stay in ascending
-// order, and a pattern that repeats every few batches (a faulty column band,
-// say) spreads over all warps instead of landing on the same ones.
-__device__ __forceinline__ int64_t warp_batch(int64_t j, int warp) {
-  return j * kWarps + (int64_t)(((warp - (int)(j % kWarps)) + kWarps) % kWarps);
-}
-
-// Number of batches warp w takes in a piece of nb batches (the j with
-// warp_batch(j, w) < nb).
-__device__ __forceinline__ int64_t warp_batches(int64_t nb, int warp) {
-  const int64_t J = nb / kWarps;
-  const int last = ((warp - (int)(J % kWarps)) % kWarps + kWarps) % kWarps;
-  return J + (last < nb % kWarps ? 1 : 0);
-}
-
 // Issue the copies of one batch, at byte offset `off` of the piece and with
 // `bytes` (whole steps only) per tensor, into a ring stage (lane 0 only).  A
 // ragged rest and the buffers of a case that is not 16-byte aligned
@@ -1014,12 +1016,17 @@ struct RingPos {
   uint32_t stage, phase;
 };
 
-// Sweep this warp's batches of a piece (each batch_elems elements; only a
-// case's last batch may be shorter) through its ring, writing each batch's
-// mismatch count.  Offsets within the piece are 32-bit (a piece holds at
-// most kMaxPiece elements).
+constexpr uint32_t kNoBatch = 0xffffffffu;
+
+// Sweep batches of a piece (each batch_elems elements; only a case's last
+// batch may be shorter) through this warp's ring, writing each batch's
+// mismatch count.  Warps claim batches from the block's counter as they
+// issue their copies (NST - 1 batches ahead of the check), so each warp's
+// batches are in ascending order and a warp slowed by exact steps takes
+// fewer.  Offsets within the piece are 32-bit (a piece holds at most
+// kMaxPiece elements).
 template <int DT, int NIN>
-__device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
+__device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
                                       int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
                                       uint32_t *err) {
   constexpr int V = Tr<DT>::V;
@@ -1033,7 +1040,6 @@ __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Re
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t *g_thr = P->g_thr;
   const uint32_t nb = (uint32_t)((pc.end - pc.begin + BATCH - 1) / BATCH);
-  const uint32_t nj = (uint32_t)warp_batches(nb, warp);
   const uint32_t mag = Tr<DT>::kInt ? 0xffffffffu : (Tr<DT>::EB == 2 ? 0x7fff7fffu : 0x7fffffffu);
   const uint32_t pbytes = (uint32_t)((pc.end - pc.begin) * EB);
   // batches at byte offsets <= full_max are whole and staged (all batches
@@ -1043,43 +1049,51 @@ __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Re
   const char *src_r = (const char *)P->cd.ref + pc.begin * EB;
   const char *src_x = NIN == 1 ? (const char *)P->cd.in_ptr[0] + pc.begin * EB : nullptr;
   int32_t *bcount = batch_count + pc.batch_base;
-  // The j-th batch is j * kWarps + rot_j, rot_j = (warp - j) mod kWarps, so
-  // its offset advances by 7 batches, or by 15 when rot wraps from 0 to 7.
-  // Copies run NST - 1 batches ahead of the check.
-  uint32_t off_i = (uint32_t)warp * BB, rot_i = warp, j_i = 0, st_i = rp.stage;
+  // lane 0: claim the next batch into stage st_i and issue its copies
+  uint32_t st_i = rp.stage;
+  bool claiming = true;
   auto issue_next = [&]() {
+    const uint32_t b = claiming ? atomicAdd(&P->next_batch, 1u) : nb;
+    if (b >= nb) {
+      claiming = false;
+      W->stage_b[st_i] = kNoBatch;
+      return;
+    }
+    W->stage_b[st_i] = b;
+    const uint32_t off = b * BB;
     uint32_t bytes = 0;
-    if ((int64_t)off_i <= full_max) {
+    if ((int64_t)off <= full_max) {
       bytes = BB;
-    } else if (P->cd.vec_ok && off_i < pbytes) {
-      bytes = (pbytes - off_i) / (STEP * EB) * (STEP * EB);
+    } else if (P->cd.vec_ok && off < pbytes) {
+      bytes = (pbytes - off) / (STEP * EB) * (STEP * EB);
     }
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    ring_issue<NIN>(src_c, src_r, src_x, off_i, bytes, ring + st_i * STAGE, bars + st_i);
-    off_i += (rot_i == 0 ? 15u : 7u) * BB;
-    rot_i = (rot_i - 1) & (kWarps - 1);
+    ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i);
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
-    ++j_i;
   };
-  if (lane == 0)
-    while (j_i < NST - 1 && j_i < nj) issue_next();
+  if (lane == 0) {
+    for (uint32_t i = 0; i < NST - 1 && claiming; ++i) issue_next();
+    W->mism_tot = 0;
+  }
   __syncwarp();
   bool dead = false;
   int flush = 0;
-  uint32_t off = (uint32_t)warp * BB, rot = warp;
   // The block's view of the case-wide maxima is read every batch; the case's
   // own value is read by one warp of the block per batch round (each warp
   // every kPoll batches, its load kPoll batches ahead of its use, so the L2
   // latency hides and the hot word sees few readers).
   uint64_t gAR = ld_relaxed64(g_thr);
   const uint32_t lane_off = (uint32_t)lane * V;
-  for (uint32_t j = 0; j < nj; ++j) {
-    const uint32_t b = off / BB;
-    const uint32_t erel = off / EB;  // element offset of the batch in the piece
-    const uint32_t next = off + (rot == 0 ? 15u : 7u) * BB;
-    rot = (rot - 1) & (kWarps - 1);
-    if (lane == 0 && j_i < nj) issue_next();  // refills the stage released last batch
-    if (lane == 0) W->mism = 0;
+  for (uint32_t j = 0;; ++j) {
+    const uint32_t b = W->stage_b[rp.stage];
+    if (b == kNoBatch) break;
+    const uint32_t erel = b * BATCH;  // element offset of the batch in the piece
+    const uint32_t off = b * BB;
+    __syncwarp();
+    if (lane == 0) {
+      if (claiming) issue_next();  // refills the stage released last batch
+      W->mism = 0;
+    }
     if ((j + warp) % kPoll == 0) {
       if (lane == 0) {
         atomicMax(&P->cta_thr[0], (uint32_t)gAR);
@@ -1147,7 +1161,10 @@ __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Re
       }
     }
     __syncwarp();  // every lane is done with the stage before it is refilled
-    if (lane == 0) bcount[b] = (int32_t)W->mism;
+    if (lane == 0) {
+      bcount[b] = (int32_t)W->mism;
+      W->mism_tot += W->mism;
+    }
     if (R.track_c | R.track_r) {
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
       R.track_r = R.track_r && !__any_sync(0xffffffffu, (R.racc & mag) != 0u);
@@ -1156,7 +1173,6 @@ __device__ __forceinline__ void sweep(const PieceSh *P, LaneSh *L, WarpSh *W, Re
       sse_flush(R.sse);
       flush = 0;
     }
-    off = next;
   }
   sse_flush(R.sse);
 }
@@ -1201,6 +1217,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (threadIdx.x == 0) {
       P.cd = cases[pc.case_id];
       P.pbegin = pc.begin;
+      P.next_batch = 0;
       P.tr0 = pc.tr0;
       P.tc0 = pc.tc0;
       P.wr = pc.wr;
@@ -1280,8 +1297,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     int64_t mism = 0;
     if (lane == 0) {
-      const int64_t nj = warp_batches(piece_batches(pc.begin, pc.end, DT), warp);
-      for (int64_t j = 0; j < nj; ++j) mism += batch_count[pc.batch_base + warp_batch(j, warp)];
+      mism = W->mism_tot;
       Partial &w = red[warp];
       w.cnt[0] = mism;
       w.best_abs = a.v;
