@@ -604,7 +604,7 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
   float s[V], e[V], rel[V];
   float mA = -1.f, mR = -1.f;
   unsigned n_abs = 0, n_rel = 0, n_pred = 0;
-#pragma unroll
+#pragma unroll 1
   for (int k = 0; k < V; ++k) {
     s[k] = 0.f;
     e[k] = 0.f;
@@ -679,7 +679,7 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     float bA = 0.f, bRn = 0.f, bRd = 1.f, bRq = 0.f;
     bool xA = true, xR = true;
     double aA = 0.0, aR = 0.0, rR = 0.0;
-#pragma unroll
+#pragma unroll 1
     for (int k = 0; k < V; ++k) {
       const bool ca = ((candA >> k) & 1u) && fabsf(s[k]) >= fA;
       const bool cr = ((candR >> k) & 1u) && rel[k] >= fR;
@@ -742,7 +742,7 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
   float s[V], rel[V];
   uint32_t candA = 0, candR = 0;
   float mA = -1.f, mR = -1.f;
-#pragma unroll
+#pragma unroll 1
   for (int k = 0; k < V; ++k) {
     const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
     if constexpr (Tr<DT>::kInt) {
@@ -773,7 +773,7 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
     float bA = 0.f, bRn = 0.f, bRd = 1.f, bRq = 0.f;
     bool xR = true;
     double rR = 0.0;
-#pragma unroll
+#pragma unroll 1
     for (int k = 0; k < V; ++k) {
       const float as = fabsf(s[k]);
       if (((candA >> k) & 1u) && as >= fA && (kA < 0 || as > bA)) {
