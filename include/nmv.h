@@ -236,6 +236,9 @@ typedef struct nmv_profile {
     int64_t exact_pred;        /* fp64 evaluations of the predicate          */
     int64_t slow_cycles;       /* SM clock cycles warps spent in exact steps  */
     int64_t light_cycles;      /* SM clock cycles warps spent in light steps  */
+    int64_t dense_steps;       /* warp steps that only counted and localised
+                                  mismatches (no maximum candidates)         */
+    int64_t dense_cycles;      /* SM clock cycles warps spent in those steps */
 } nmv_profile;
 
 void nmv_profile_enable(int mode);

@@ -669,6 +669,8 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     P.exact_pred = (int64_t)st4[3];
     P.slow_cycles = (int64_t)st4[5];
     P.light_cycles = (int64_t)st4[6];
+    P.dense_steps = (int64_t)st4[7];
+    P.dense_cycles = (int64_t)st4[8];
     g_prof.valid = true;
   }
 

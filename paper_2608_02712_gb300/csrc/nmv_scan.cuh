@@ -260,7 +260,8 @@ struct PieceSh {
   uint32_t *cta_thr;  // [2] the block's view of the case-wide maxima (float bits), in shared memory
   int32_t *sh_eq;  // [kThreads][NMV_MAX_INPUTS] pass-through counts of the exact paths (inputs only)
   unsigned long long *stats;  // [exact steps, exact abs, exact rel, exact predicate, light steps,
-                              //  SM cycles in exact steps, SM cycles in light steps]
+                              //  SM cycles in exact steps, SM cycles in light steps,
+                              //  dense steps, SM cycles in dense steps]
 };
 
 // The maxima one lane holds, in shared memory.
@@ -286,7 +287,7 @@ struct WarpSh {
   int64_t mism;       // mismatches so far in this batch
   int64_t mism_tot;   // mismatches in the warp's batches of this piece
   uint32_t stage_b[4];  // batch held by each ring stage (kNoBatch: none)
-  unsigned long long st[7];  // the warp's profile counters (layout of PieceSh::stats)
+  unsigned long long st[9];  // the warp's profile counters (layout of PieceSh::stats)
 };
 
 __device__ __forceinline__ float pub_thr(uint32_t bits) {
@@ -573,16 +574,16 @@ static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, W
   __syncwarp();
 }
 
-// Profile counters of one exact (slot 0) or light (slot 1) step, kept per
-// warp and added to the call's counters once per piece.
+// Profile counters of one exact (slot 0), light (slot 1) or dense (slot 2)
+// step, kept per warp and added to the call's counters once per piece.
 __device__ __forceinline__ void count_stats(WarpSh *W, int slot, long long t0, unsigned n_abs, unsigned n_rel,
                                             unsigned n_pred) {
   n_abs = __reduce_add_sync(0xffffffffu, n_abs);
   n_rel = __reduce_add_sync(0xffffffffu, n_rel);
   n_pred = __reduce_add_sync(0xffffffffu, n_pred);
   if ((threadIdx.x & 31) == 0) {
-    W->st[slot == 0 ? 0 : 4] += 1;
-    W->st[slot == 0 ? 5 : 6] += (unsigned long long)(clock64() - t0);
+    W->st[slot == 0 ? 0 : (slot == 1 ? 4 : 7)] += 1;
+    W->st[slot == 0 ? 5 : (slot == 1 ? 6 : 8)] += (unsigned long long)(clock64() - t0);
     W->st[1] += n_abs;
     W->st[2] += n_rel;
     W->st[3] += n_pred;
@@ -807,6 +808,34 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
   return sse;
 }
 
+// A step of finite elements whose predicate the fp32 bounds decide and none
+// of which can be a new maximum (|s| <= tA and |s| <= tR |r|, tR uncapped):
+// the dense-mismatch case (an output that is wrong almost everywhere).
+// Only the mismatch count, the localisation maps and the SSE remain; the
+// SSE terms take the exact path's arithmetic (c - r as s + e by TwoSum), so
+// the result does not depend on which path an element took.  Float types.
+template <int DT>
+__device__ __noinline__ SseAcc dense_step(const PieceSh *P, WarpSh *W, uint4 cv, uint4 rv, int64_t idx0,
+                                          SseAcc sse) {
+  constexpr int V = Tr<DT>::V;
+  const long long t_start = P->stats ? clock64() : 0;
+  const float lo_r = P->cd.lo_r, lo_a = P->cd.lo_a;
+  uint32_t mask = 0;
+#pragma unroll
+  for (int k = 0; k < V; ++k) {
+    const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
+    const float sk = __fsub_rn(cf, rf);
+    const float bb = __fsub_rn(sk, cf);
+    const float ek = __fsub_rn(__fsub_rn(cf, __fsub_rn(sk, bb)), __fadd_rn(rf, bb));  // TwoSum(c, -r)
+    if (!(fabsf(sk) <= __fmaf_rz(lo_r, fabsf(rf), lo_a))) mask |= 1u << k;
+    if (k & 1) ff_term(sse.hi.y, sse.lo.y, sk, ek);
+    else ff_term(sse.hi.x, sse.lo.x, sk, ek);
+  }
+  if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0, V);
+  if (P->stats) count_stats(W, 2, t_start, 0, 0, 0);
+  return sse;
+}
+
 // A ragged step: this lane's n (0..V) elements from idx0, loaded one by one.
 template <int DT, int NIN>
 __device__ __noinline__ SseAcc tail_step(const PieceSh *P, LaneSh *L, WarpSh *W, int64_t idx0, int n,
@@ -990,8 +1019,25 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
       other |= !(fabsf(s[k]) <= min3f(a, __fmul_rz(0.25f, fabsf(rf)), kHuge));
     }
   }
-  if (__any_sync(0xffffffffu, other)) R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
-  else R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
+  if (__any_sync(0xffffffffu, other)) {
+    bool dense = false;
+    if constexpr (!Tr<DT>::kInt) {
+      // every element finite, decided by the fp32 bounds, and no candidate
+      // for a maximum (|s| <= tA also rules out NaN and infinities)
+      dense = true;
+#pragma unroll
+      for (int k = 0; k < V; ++k) {
+        const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
+        const float as = fabsf(__fsub_rn(cf, rf)), ar = fabsf(rf);
+        const bool decided = as <= __fmaf_rz(R.lo_r, ar, R.lo_a) || as > __fmaf_ru(P->cd.hi_r, ar, P->cd.hi_a);
+        dense &= decided && as <= R.tA && as <= __fmul_rz(R.tR, ar);
+      }
+    }
+    if (__all_sync(0xffffffffu, dense)) R.sse = dense_step<DT>(P, W, cv, rv, P->pbegin + erel, R.sse);
+    else R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
+  } else {
+    R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
+  }
   reload_thr(R, W);
 }
 
@@ -1255,7 +1301,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       W->tA = W->tR = W->wA = W->wR = W->ga = W->gr = -1.f;
       W->pubA = W->pubR = 0;
       W->mism = 0;
-      for (int k = 0; k < 7; ++k) W->st[k] = 0;
+      for (int k = 0; k < 9; ++k) W->st[k] = 0;
     }
     __syncthreads();
 
@@ -1277,7 +1323,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
     __syncwarp();
     if (stats && lane == 0)
-      for (int k = 0; k < 7; ++k)
+      for (int k = 0; k < 9; ++k)
         if (W->st[k]) atomicAdd(&stats[k], W->st[k]);
 
     // ---- lanes -> warps -> the piece's partial

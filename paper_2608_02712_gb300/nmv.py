@@ -39,7 +39,8 @@ class Profile(ctypes.Structure):
                 ("light_steps", ctypes.c_int64),
                 ("exact_abs", ctypes.c_int64), ("exact_rel", ctypes.c_int64),
                 ("exact_pred", ctypes.c_int64), ("slow_cycles", ctypes.c_int64),
-                ("light_cycles", ctypes.c_int64)]
+                ("light_cycles", ctypes.c_int64), ("dense_steps", ctypes.c_int64),
+                ("dense_cycles", ctypes.c_int64)]
 
 
 class Case(ctypes.Structure):
