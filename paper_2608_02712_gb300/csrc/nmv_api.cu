@@ -22,7 +22,8 @@ struct ScanOps {
   static cudaError_t prepare(int nin, size_t smem);
   static int occupancy(int nin, size_t smem);
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
-                            const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
+                            const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,
+                            int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                             unsigned long long *stats, uint32_t *err);
 };
@@ -50,21 +51,21 @@ int scan_occupancy(int dt, int nin, size_t smem) {
 }
 
 cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
-                        const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
+                        const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
                         Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                         unsigned long long *stats, uint32_t *err) {
   switch (dt) {
     case NMV_F32:
-      return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+      return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
     case NMV_F16:
-      return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+      return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
     case NMV_BF16:
-      return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+      return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
                                        partials, batch_count, out, g_thr, stats, err);
     default:
-      return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, block_piece, piece_base,
+      return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
   }
 }
@@ -286,7 +287,6 @@ int ensure_workspace(DeviceState &s, size_t ws, size_t pinned) {
 
 struct Plan {
   std::vector<Piece> pieces;
-  std::vector<int64_t> block_piece;
   size_t smem = 0;
 };
 
@@ -326,9 +326,10 @@ size_t piece_smem(const nmv_case &c, const Piece &p) {
   return words * 4;
 }
 
-// Split the concatenated bytes of the cases `ids` into `grid` balanced block
+// Split the concatenated bytes of the cases `ids` into `grid` balanced
 // ranges; cut them at case boundaries (and at kMaxPiece) into pieces whose
-// element boundaries are multiples of the case's batch (batch_elems).
+// element boundaries are multiples of the case's batch (batch_elems).  The
+// scan blocks take the pieces dynamically.
 void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::vector<int64_t> &ids,
                int grid, Plan &plan) {
   const int64_t n = (int64_t)ids.size();
@@ -352,10 +353,8 @@ void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::ve
     se[b] = e;
   }
   plan.pieces.clear();
-  plan.block_piece.assign(grid + 1, 0);
   plan.smem = 0;
   for (int b = 0; b < grid; ++b) {
-    plan.block_piece[b] = (int64_t)plan.pieces.size();
     for (int64_t c = sc[b]; c <= std::min(sc[b + 1], n - 1); ++c) {
       const Geo &g = geo[ids[c]];
       if (g.numel == 0) continue;
@@ -373,7 +372,6 @@ void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::ve
       }
     }
   }
-  plan.block_piece[grid] = (int64_t)plan.pieces.size();
 }
 
 // Cases that share an element type and an input-count class run in one
@@ -493,7 +491,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       groups[gi].ids.push_back(i);
     }
   }
-  int64_t np = 0, nbp = 0;
+  int64_t np = 0;
   for (Group &G : groups) {
     int64_t total_bytes = 0;
     size_t prof_smem = kShHeadWords * 4;
@@ -516,7 +514,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       int64_t g = (int64_t)S->sms * occ;
       g = std::min(g, std::max<int64_t>(1, total_bytes / 16384));
       G.grid = (int)g;
-      make_plan(cases, geo, G.ids, G.grid, G.plan);
+      make_plan(cases, geo, G.ids, G.grid * kPiecesPerBlock, G.plan);
       G.smem = std::max(G.plan.smem, (size_t)1024);
       if (G.plan.smem <= want) break;
       guess = G.plan.smem;
@@ -530,17 +528,13 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       set = G.smem;
     }
     G.piece_base = np;
-    G.bp_base = nbp;
     np += (int64_t)G.plan.pieces.size();
-    nbp += G.grid + 1;
   }
 
   // ---- descriptors (pieces of a case are contiguous within its group)
   std::vector<CaseDesc> desc((size_t)n);
   std::vector<Piece> all_pieces;
-  std::vector<int64_t> all_bp;
   all_pieces.reserve((size_t)np);
-  all_bp.reserve((size_t)nbp);
   size_t out_size = kCallHeader;
   for (int64_t i = 0; i < n; ++i) {
     fill_desc(cases[i], geo[i], desc[i]);
@@ -566,17 +560,16 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       d.batch_end = n_batches;
       all_pieces.push_back(p);
     }
-    all_bp.insert(all_bp.end(), G.plan.block_piece.begin(), G.plan.block_piece.end());
   }
 
   // ---- workspace layout
   const size_t sz_cases = align_up(sizeof(CaseDesc) * n, 256);
   const size_t sz_pieces = align_up(sizeof(Piece) * std::max<int64_t>(np, 1), 256);
-  const size_t sz_bp = align_up(sizeof(int64_t) * std::max<int64_t>(nbp, 1), 256);
-  const size_t table = sz_cases + sz_pieces + sz_bp;
+  const size_t table = sz_cases + sz_pieces;
   const size_t sz_part = align_up(sizeof(Partial) * std::max<int64_t>(np, 1), 256);
   const size_t sz_segc = align_up(sizeof(int32_t) * std::max<int64_t>(n_batches, 1), 256);
-  const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n, 256);
+  // published thresholds (2 x u32 per case), then one piece counter per group
+  const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n + sizeof(unsigned long long) * groups.size(), 256);
   const size_t sz_sse = align_up(sizeof(double) * kSseBlocksHost, 256);
   const size_t o_part = table, o_segc = o_part + sz_part;
   const size_t o_sse = o_segc + sz_segc, o_thr = o_sse + sz_sse, o_out = o_thr + sz_thr;
@@ -587,7 +580,6 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   uint8_t *H = (uint8_t *)S->pinned;
   std::memcpy(H, desc.data(), sizeof(CaseDesc) * n);
   if (np) std::memcpy(H + sz_cases, all_pieces.data(), sizeof(Piece) * np);
-  if (nbp) std::memcpy(H + sz_cases + sz_pieces, all_bp.data(), sizeof(int64_t) * nbp);
 
   cudaError_t e = cudaMemcpyAsync(W, H, table, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
@@ -595,7 +587,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   const CaseDesc *d_cases = (const CaseDesc *)W;
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
-  const int64_t *d_bp = (const int64_t *)(W + sz_cases + sz_pieces);
+  unsigned long long *d_ctr = (unsigned long long *)(W + o_thr + sizeof(uint32_t) * 2 * n);
   if (injected("launch")) {
     cudaStreamSynchronize(st);
     return fail(NMV_ECUDA, "injected launch failure");
@@ -618,9 +610,10 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     g_prof.valid = false;
     cudaEventRecord(g_prof.ev[0], st);
   }
-  for (const Group &G : groups) {
-    e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_bp + G.bp_base,
-                    G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out,
+  for (size_t gi = 0; gi < groups.size(); ++gi) {
+    const Group &G = groups[gi];
+    e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_ctr + gi,
+                    (int64_t)G.plan.pieces.size(), G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out,
                     (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
@@ -773,7 +766,6 @@ void *g_noalloc_ptr[kMaxDevices];
 constexpr int kNaMaxBlocks = 8192;
 CaseDesc g_na_desc;
 Piece g_na_pieces[kNaMaxBlocks];
-int64_t g_na_bp[kNaMaxBlocks + 1];
 OutHeader g_na_head;
 
 int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
@@ -829,18 +821,18 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
       if (occ < 1) occ = 1;
       int64_t gr = (int64_t)S->sms * occ;
       gr = std::min(gr, std::max<int64_t>(1, g.numel * g.eb / 16384));
-      gr = std::min<int64_t>(gr, kNaMaxBlocks);
+      gr = std::min<int64_t>(gr, kNaMaxBlocks / kPiecesPerBlock);
       grid = (int)gr;
       const int64_t total = g.numel * g.eb;
+      const int ranges = grid * kPiecesPerBlock;
       size_t need = 0;
       n_pieces = 0;
-      for (int b = 0; b < grid; ++b) {
-        g_na_bp[b] = n_pieces;
-        const int64_t x0 = (int64_t)((__int128)total * b / grid);
-        const int64_t x1 = (int64_t)((__int128)total * (b + 1) / grid);
+      for (int b = 0; b < ranges; ++b) {
+        const int64_t x0 = (int64_t)((__int128)total * b / ranges);
+        const int64_t x1 = (int64_t)((__int128)total * (b + 1) / ranges);
         const int64_t be = batch_elems(g.dt);
         const int64_t e0 = x0 / g.eb / be * be;
-        const int64_t e1 = (b + 1 == grid) ? g.numel : x1 / g.eb / be * be;
+        const int64_t e1 = (b + 1 == ranges) ? g.numel : x1 / g.eb / be * be;
         if (e1 <= e0) continue;
         if (e1 - e0 > kMaxPiece) return fail(NMV_EINVAL, "case too large for the no-allocation scratch");
         Piece &pc = g_na_pieces[n_pieces++];
@@ -851,7 +843,6 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
         piece_window(*c, g, pc);
         need = std::max(need, piece_smem(*c, pc));
       }
-      g_na_bp[grid] = n_pieces;
       smem = std::max(need, (size_t)1024);
       if (need <= want) break;
       guess = need;
@@ -880,8 +871,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   // ---- scratch layout (the same regions as the workspace of nmv_validate)
   const size_t sz_cases = align_up(sizeof(CaseDesc), 256);
   const size_t sz_pieces = align_up(sizeof(Piece) * (size_t)std::max<int64_t>(n_pieces, 1), 256);
-  const size_t sz_bp = align_up(sizeof(int64_t) * (size_t)(grid + 1), 256);
-  const size_t o_part = sz_cases + sz_pieces + sz_bp;
+  const size_t o_part = sz_cases + sz_pieces;
   const size_t sz_part = align_up(sizeof(Partial) * (size_t)std::max<int64_t>(n_pieces, 1), 256);
   const size_t o_segc = o_part + sz_part;
   const size_t sz_segc = align_up(sizeof(int32_t) * (size_t)std::max<int64_t>(n_batches, 1), 256);
@@ -901,19 +891,17 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   cudaError_t e = cudaMemcpyAsync(W, &g_na_desc, sizeof(CaseDesc), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess && n_pieces > 0)
     e = cudaMemcpyAsync(W + sz_cases, g_na_pieces, sizeof(Piece) * (size_t)n_pieces, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess && grid > 0)
-    e = cudaMemcpyAsync(W + sz_cases + sz_pieces, g_na_bp, sizeof(int64_t) * (size_t)(grid + 1),
-                        cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
-  // The scratch keeps the previous call's contents: the thresholds and the
-  // packed result (maps and counters are accumulated) must start at zero.
+  // The scratch keeps the previous call's contents: the thresholds, the piece
+  // counter and the packed result (maps and counters are accumulated) must
+  // start at zero.
   // Partials and batch counts are written in full by the scan kernel.
   e = cudaMemsetAsync(W + o_thr, 0, 256 + kCallHeader + g.out_size, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   const CaseDesc *d_case = (const CaseDesc *)W;
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   if (grid > 0) {
-    e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (const int64_t *)(W + sz_cases + sz_pieces), 0,
+    e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (unsigned long long *)(W + o_thr + 8), n_pieces, 0,
                     (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr,
                     (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");

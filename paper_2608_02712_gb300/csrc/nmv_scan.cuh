@@ -1179,7 +1179,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       rp.phase ^= 1u;
     }
     if ((int64_t)off <= full_max) {
-#pragma unroll
+#pragma unroll 1
       for (int u = 0; u < kSteps; ++u) {
         const uint4 cv = lds_v4(stage + u * 512);
         const uint4 rv = lds_v4(stage + kBatchBytes + u * 512);
@@ -1233,7 +1233,7 @@ constexpr int kShHead = 16;
 template <int DT, int NIN>
 __global__ void __launch_bounds__(kThreads, 2)
     scan_kernel(const CaseDesc *__restrict__ cases, const Piece *__restrict__ pieces,
-                const int64_t *__restrict__ block_piece, int64_t piece_base, Partial *partials,
+                unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base, Partial *partials,
                 int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
@@ -1257,8 +1257,15 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   __syncwarp();
   RingPos rpos = {0u, 0u};
-  const int64_t p0 = block_piece[blockIdx.x], p1 = block_piece[blockIdx.x + 1];
-  for (int64_t p = p0; p < p1; ++p) {
+  // Blocks take pieces from the launch's counter as they finish the last
+  // one, so pieces of uneven cost (a region wrong everywhere next to a clean
+  // one) balance over the blocks.
+  __shared__ int64_t sh_piece;
+  for (;;) {
+    if (threadIdx.x == 0) sh_piece = (int64_t)atomicAdd(piece_ctr, 1ull);
+    __syncthreads();
+    const int64_t p = sh_piece;
+    if (p >= n_pieces) break;
     const Piece pc = pieces[p];
     if (threadIdx.x == 0) {
       P.cd = cases[pc.case_id];
@@ -1280,7 +1287,10 @@ __global__ void __launch_bounds__(kThreads, 2)
       P.g_thr = g_thr + 2 * pc.case_id;
       P.sh_eq = sh_eq;
       P.cta_thr = cta_thr;
-      cta_thr[0] = cta_thr[1] = 0;
+      // the block's view starts from what the case has published so far
+      const uint64_t g = ld_relaxed64(P.g_thr);
+      cta_thr[0] = (uint32_t)g;
+      cta_thr[1] = (uint32_t)(g >> 32);
       P.stats = stats;
     }
     __syncthreads();
@@ -1408,7 +1418,7 @@ struct ScanOps {
   static cudaError_t prepare(int nin, size_t smem);
   static int occupancy(int nin, size_t smem);
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
-                            const Piece *pieces, const int64_t *block_piece, int64_t piece_base,
+                            const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                             unsigned long long *stats, uint32_t *err);
 };
@@ -1437,18 +1447,19 @@ struct ScanOps {
   }                                                                                                      \
   template <>                                                                                            \
   cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases, \
-                                  const Piece *pieces, const int64_t *block_piece, int64_t piece_base,    \
+                                  const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,  \
+                                  int64_t piece_base,                                                     \
                                   Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr, \
                                   unsigned long long *stats, uint32_t *err) {                            \
     if (nin == 0)                                                                                        \
       NMV_SCAN_FN(DT, 0)<<<grid, kThreads, NMV_SCAN_SMEM(0, smem), st>>>(                               \
-          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     else if (nin == 1)                                                                                   \
       NMV_SCAN_FN(DT, 1)<<<grid, kThreads, NMV_SCAN_SMEM(1, smem), st>>>(                               \
-          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     else                                                                                                 \
       NMV_SCAN_FN(DT, -1)<<<grid, kThreads, NMV_SCAN_SMEM(-1, smem), st>>>(                              \
-          cases, pieces, block_piece, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     return cudaGetLastError();                                                                           \
   }
 
