@@ -38,7 +38,7 @@ __device__ __forceinline__ bool pass_elem(const CaseDesc &cd, uint32_t cb, uint3
     if (as <= __fmaf_rz(cd.lo_r, ar, cd.lo_a)) return true;
     if (as > __fmaf_ru(cd.hi_r, ar, cd.hi_a)) return false;
   }
-  return pass64_inl(to_f64<DT>(cb), to_f64<DT>(rb), cd.rtol, cd.atol);
+  return pass64(to_f64<DT>(cb), to_f64<DT>(rb), cd.rtol, cd.atol);
 }
 
 // Exclusive block-wide prefix sum of a 64-bit v; *total = the block's sum.
@@ -77,29 +77,51 @@ __device__ __forceinline__ void write_record(const CaseDesc &cd, uint8_t *o, int
   fk_r[pos] = widen_any(rb, cd.dtype);
 }
 
-// Re-read elements [lo, hi) with one warp and write the first `needed`
-// mismatches at record positions pos0, pos0 + 1, ...  (E consecutive
-// elements per lane, warp-wide ordered compaction).
+// Re-read elements [lo, hi) (one batch, lo batch-aligned) with one warp
+// and write the first `needed` mismatches at record positions pos0, pos0 +
+// 1, ...  Lane l takes the V elements at lo + u * 32V + lV of each warp step
+// u, as the scan does; a 16-byte aligned case loads all of the batch's
+// vectors up front, so the batch costs one memory latency.  Records are
+// placed by a warp-wide ordered compaction, step by step.
 template <int DT>
 __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t hi, int64_t pos0,
                             int64_t needed) {
-  constexpr int E = 8;
+  constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
+  constexpr int STEP = 32 * V;
   const int lane = threadIdx.x & 31;
-  int64_t found = 0;
-  for (int64_t base = lo; base < hi && found < needed; base += 32 * E) {
-    const int64_t i0 = base + (int64_t)lane * E;
-    uint32_t cb[E], rb[E];
+  uint4 cv[kSteps], rv[kSteps];
 #pragma unroll
-    for (int k = 0; k < E; ++k) {
-      const bool in = i0 + k < hi;
-      cb[k] = in ? ld_one<EB>(cd.cand, i0 + k) : 0u;
-      rb[k] = in ? ld_one<EB>(cd.ref, i0 + k) : 0u;
+  for (int u = 0; u < kSteps; ++u) {
+    const int64_t i0 = lo + u * STEP + lane * V;
+    if (cd.vec_ok && i0 + V <= hi) {
+      cv[u] = ld_v4((const char *)cd.cand + i0 * EB);
+      rv[u] = ld_v4((const char *)cd.ref + i0 * EB);
+    } else {
+      uint32_t cw[4] = {0, 0, 0, 0}, rw[4] = {0, 0, 0, 0};
+      for (int k = 0; k < V; ++k) {
+        if (i0 + k >= hi) break;
+        const uint32_t c = ld_one<EB>(cd.cand, i0 + k), r = ld_one<EB>(cd.ref, i0 + k);
+        if constexpr (EB == 2) {
+          cw[k >> 1] |= c << (16 * (k & 1));
+          rw[k >> 1] |= r << (16 * (k & 1));
+        } else {
+          cw[k] = c;
+          rw[k] = r;
+        }
+      }
+      cv[u] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+      rv[u] = make_uint4(rw[0], rw[1], rw[2], rw[3]);
     }
+  }
+  int64_t found = 0;
+#pragma unroll
+  for (int u = 0; u < kSteps; ++u) {
+    const int64_t i0 = lo + u * STEP + lane * V;
     uint32_t mask = 0;
 #pragma unroll
-    for (int k = 0; k < E; ++k)
-      if (i0 + k < hi && !pass_elem<DT>(cd, cb[k], rb[k])) mask |= 1u << k;
+    for (int k = 0; k < V; ++k)
+      if (i0 + k < hi && !pass_elem<DT>(cd, vbits<DT>(cv[u], k), vbits<DT>(rv[u], k))) mask |= 1u << k;
     const int cnt = __popc(mask);
     int incl = cnt;
 #pragma unroll
@@ -108,14 +130,15 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
       if (lane >= d) incl += t;
     }
     const int64_t pos = found + incl - cnt;
-#pragma unroll
-    for (int k = 0, j = 0; k < E; ++k) {
+    for (int k = 0, j = 0; k < V; ++k) {
       if ((mask >> k) & 1u) {
-        if (pos + j < needed) write_record(cd, o, pos0 + pos + j, i0 + k, cb[k], rb[k]);
+        if (pos + j < needed)
+          write_record(cd, o, pos0 + pos + j, i0 + k, vbits<DT>(cv[u], k), vbits<DT>(rv[u], k));
         ++j;
       }
     }
     found += __shfl_sync(0xffffffffu, incl, 31);
+    if (found >= needed) break;
   }
 }
 
@@ -186,7 +209,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
   OutHeader *H = (OutHeader *)o;
   __shared__ int64_t sh_scan[kFinThreads / 32 + 1];
   __shared__ int64_t sh_mism;
-  __shared__ int64_t sh_need[kFinThreads];
+  __shared__ int64_t sh_need[kFinThreads], sh_need_p[kFinThreads];
   __shared__ int64_t sh_item[kFinThreads][3];
   __shared__ int sh_nitems;
   __shared__ Red sh_red[kFinThreads / 32];
@@ -297,11 +320,18 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
     const int64_t n = p < cd.piece_end ? partials[p].cnt[0] : 0;
     int64_t total;
     const int64_t pre = base + block_excl_scan64(n, &total, sh_scan);
-    sh_need[threadIdx.x] = (n > 0 && pre < K) ? pre : -1;
+    // compact the pieces holding records below K, in order
+    const bool need = n > 0 && pre < K;
+    int64_t n_need;
+    const int64_t slot = block_excl_scan64(need ? 1 : 0, &n_need, sh_scan);
+    if (need) {
+      sh_need[slot] = pre;
+      sh_need_p[slot] = p;
+    }
     __syncthreads();
-    for (int j = 0; j < kFinThreads && q0 + j < cd.piece_end; ++j) {
-      const int64_t pos0 = sh_need[j];
-      if (pos0 >= 0) first_k_piece(cd, o, pieces[q0 + j], batch_count, pos0, K, sh_scan, sh_item, &sh_nitems);
+    for (int64_t j = 0; j < n_need; ++j) {
+      const int64_t pos0 = sh_need[j], pj = sh_need_p[j];
+      first_k_piece(cd, o, pieces[pj], batch_count, pos0, K, sh_scan, sh_item, &sh_nitems);
     }
     base += total;
     __syncthreads();

@@ -928,11 +928,21 @@ static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parit
   return true;
 }
 
-__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                   smem_addr(dst)),
-               "l"(src), "r"(bytes), "r"(smem_addr(bar))
-               : "memory");
+// The streamed tensors are read once: their L2 lines are marked
+// evict-first, so they do not push out what is reused (kernel code,
+// descriptors, counters, the next call's metadata).
+__device__ __forceinline__ uint64_t evict_first_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
+__device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(pol)
+      : "memory");
 }
 
 __device__ __forceinline__ uint4 lds_v4(const void *p) {
@@ -1050,9 +1060,10 @@ __device__ __forceinline__ void ring_issue(const char *c, const char *r, const c
                                            uint32_t bytes, uint8_t *stage, uint64_t *bar) {
   mbar_arrive_tx(bar, bytes * (NIN == 1 ? 3u : 2u));
   if (bytes) {
-    bulk_load(stage, c + off, bytes, bar);
-    bulk_load(stage + kBatchBytes, r + off, bytes, bar);
-    if constexpr (NIN == 1) bulk_load(stage + 2 * kBatchBytes, x + off, bytes, bar);
+    const uint64_t pol = evict_first_policy();
+    bulk_load(stage, c + off, bytes, bar, pol);
+    bulk_load(stage + kBatchBytes, r + off, bytes, bar, pol);
+    if constexpr (NIN == 1) bulk_load(stage + 2 * kBatchBytes, x + off, bytes, bar, pol);
   }
 }
 
