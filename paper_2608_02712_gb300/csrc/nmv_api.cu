@@ -331,7 +331,7 @@ size_t piece_smem(const nmv_case &c, const Piece &p) {
 // element boundaries are multiples of the case's batch (batch_elems).  The
 // scan blocks take the pieces dynamically.
 void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::vector<int64_t> &ids,
-               int grid, Plan &plan) {
+               int grid, int nin, Plan &plan) {
   const int64_t n = (int64_t)ids.size();
   std::vector<int64_t> off(n + 1, 0);
   for (int64_t i = 0; i < n; ++i) off[i + 1] = off[i] + geo[ids[i]].numel * geo[ids[i]].eb;
@@ -348,7 +348,7 @@ void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::ve
     }
     const Geo &g = geo[ids[ci]];
     int64_t e = (x - off[ci]) / g.eb;
-    e = e / batch_elems(g.dt) * batch_elems(g.dt);
+    e = e / batch_elems(g.dt, nin) * batch_elems(g.dt, nin);
     sc[b] = ci;
     se[b] = e;
   }
@@ -514,7 +514,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       int64_t g = (int64_t)S->sms * occ;
       g = std::min(g, std::max<int64_t>(1, total_bytes / 16384));
       G.grid = (int)g;
-      make_plan(cases, geo, G.ids, G.grid * kPiecesPerBlock, G.plan);
+      make_plan(cases, geo, G.ids, G.grid * kPiecesPerBlock, G.nin, G.plan);
       G.smem = std::max(G.plan.smem, (size_t)1024);
       if (G.plan.smem <= want) break;
       guess = G.plan.smem;
@@ -550,7 +550,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       const int64_t gid = G.piece_base + (int64_t)k;
       CaseDesc &d = desc[p.case_id];
       p.batch_base = n_batches;
-      const int64_t nb = piece_batches(p.begin, p.end, G.dt);
+      const int64_t nb = piece_batches(p.begin, p.end, G.dt, G.nin);
       if (d.piece_end == 0) {
         d.piece_begin = gid;
         d.batch_begin = n_batches;
@@ -830,7 +830,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
       for (int b = 0; b < ranges; ++b) {
         const int64_t x0 = (int64_t)((__int128)total * b / ranges);
         const int64_t x1 = (int64_t)((__int128)total * (b + 1) / ranges);
-        const int64_t be = batch_elems(g.dt);
+        const int64_t be = batch_elems(g.dt, nin);
         const int64_t e0 = x0 / g.eb / be * be;
         const int64_t e1 = (b + 1 == ranges) ? g.numel : x1 / g.eb / be * be;
         if (e1 <= e0) continue;
@@ -863,7 +863,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   int64_t n_batches = 0;
   for (int64_t k = 0; k < n_pieces; ++k) {
     g_na_pieces[k].batch_base = n_batches;
-    n_batches += piece_batches(g_na_pieces[k].begin, g_na_pieces[k].end, g.dt);
+    n_batches += piece_batches(g_na_pieces[k].begin, g_na_pieces[k].end, g.dt, nin);
   }
   g_na_desc.batch_begin = 0;
   g_na_desc.batch_end = n_batches;

@@ -90,10 +90,15 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
   const int lane = threadIdx.x & 31;
-  uint4 cv[kSteps], rv[kSteps];
+  const int ks = batch_steps(nin_class_of(cd.n_elig));
+  uint4 cv[kMaxSteps], rv[kMaxSteps];
 #pragma unroll
-  for (int u = 0; u < kSteps; ++u) {
+  for (int u = 0; u < kMaxSteps; ++u) {
     const int64_t i0 = lo + u * STEP + lane * V;
+    if (u >= ks) {
+      cv[u] = rv[u] = make_uint4(0, 0, 0, 0);
+      continue;
+    }
     if (cd.vec_ok && i0 + V <= hi) {
       cv[u] = ld_v4((const char *)cd.cand + i0 * EB);
       rv[u] = ld_v4((const char *)cd.ref + i0 * EB);
@@ -116,7 +121,8 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
   }
   int64_t found = 0;
 #pragma unroll
-  for (int u = 0; u < kSteps; ++u) {
+  for (int u = 0; u < kMaxSteps; ++u) {
+    if (u >= ks) break;
     const int64_t i0 = lo + u * STEP + lane * V;
     uint32_t mask = 0;
 #pragma unroll
@@ -148,8 +154,9 @@ __device__ void reread_warp(const CaseDesc &cd, uint8_t *o, int64_t lo, int64_t 
 // one warp.  Called by the whole block with uniform arguments.
 __device__ void first_k_piece(const CaseDesc &cd, uint8_t *o, const Piece &pc, const int32_t *batch_count,
                               int64_t pos0, int64_t K, int64_t *sh_scan, int64_t (*sh_item)[3], int *sh_nitems) {
-  const int64_t be = batch_elems(cd.dtype);
-  const int64_t nb = piece_batches(pc.begin, pc.end, cd.dtype);
+  const int nin = nin_class_of(cd.n_elig);
+  const int64_t be = batch_elems(cd.dtype, nin);
+  const int64_t nb = piece_batches(pc.begin, pc.end, cd.dtype, nin);
   const int warp = threadIdx.x >> 5;
   int64_t pos = pos0;
   for (int64_t b0 = 0; b0 < nb && pos < K; b0 += kFinThreads) {

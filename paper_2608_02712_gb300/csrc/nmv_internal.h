@@ -107,30 +107,34 @@ struct OutHeader {
   int64_t pad[3];
 };
 
-// Warp steps (32 lanes x 16 bytes of each tensor) per batch, and elements
-// per batch.  A batch is the unit of the first-K counts and of the warps'
-// shared-memory rings.
-constexpr int kSteps = 3;
-constexpr int kBatchBytes = 32 * 16 * kSteps;  // one tensor's bytes of a batch
-NMV_HD int64_t batch_elems(int dt) { return (int64_t)32 * vec_elems(dt) * kSteps; }
-NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt) {
-  const int64_t be = batch_elems(dt);
-  return (end - begin + be - 1) / be;
-}
-
-// Ring of each scan warp, by input class (0, 1 or -1 = several inputs read
-// from global memory): stages, tensors staged per batch, and the dynamic
-// shared memory of all rings of a block (stage data, then one 8-byte
-// mbarrier per stage).
 #ifdef __CUDACC__
 #define NMV_CHD __host__ __device__ constexpr
 #else
 #define NMV_CHD constexpr
 #endif
-NMV_CHD int ring_stages(int nin) { return nin == 1 ? 2 : 3; }
+
+// Warp steps (32 lanes x 16 bytes of each tensor) per batch, by input class
+// (0, 1 or -1 = several inputs read from global memory; one staged input
+// leaves shared memory for shorter batches only), and elements per batch.  A
+// batch is the unit of the first-K counts and of the warps' shared-memory
+// rings.
+constexpr int kMaxSteps = 4;
+NMV_CHD int batch_steps(int nin) { return nin == 1 ? 2 : 4; }
+NMV_CHD int batch_bytes(int nin) { return 32 * 16 * batch_steps(nin); }  // one tensor's bytes
+NMV_CHD int nin_class_of(int n_elig) { return n_elig == 0 ? 0 : (n_elig == 1 ? 1 : -1); }
+NMV_HD int64_t batch_elems(int dt, int nin) { return (int64_t)32 * vec_elems(dt) * batch_steps(nin); }
+NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt, int nin) {
+  const int64_t be = batch_elems(dt, nin);
+  return (end - begin + be - 1) / be;
+}
+
+// Ring of each scan warp, by input class: stages, tensors staged per batch,
+// and the dynamic shared memory of all rings of a block (stage data, then
+// one 8-byte mbarrier per stage).
+NMV_CHD int ring_stages(int) { return 2; }
 NMV_CHD int ring_streams(int nin) { return nin == 1 ? 3 : 2; }
 NMV_CHD size_t ring_bytes(int nin) {
-  return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * kBatchBytes + 8);
+  return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * batch_bytes(nin) + 8);
 }
 
 }  // namespace nmv

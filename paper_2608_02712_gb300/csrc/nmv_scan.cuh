@@ -55,9 +55,9 @@
 
 namespace nmv {
 
-// The SSE's float-float pairs go to fp64 every kFlushBatches batches (about
-// 32 warp steps, at most 128 terms per pair).
-constexpr int kFlushBatches = (32 + kSteps - 1) / kSteps;
+// The SSE's float-float pairs go to fp64 every flush_batches(nin) batches
+// (about 32 warp steps, at most 128 terms per pair).
+NMV_CHD int flush_batches(int nin) { return (32 + batch_steps(nin) - 1) / batch_steps(nin); }
 constexpr float kHuge = 0x1p56f;
 constexpr float kMarginLo = 1.0f - 0x1p-20f;
 
@@ -1062,8 +1062,8 @@ __device__ __forceinline__ void ring_issue(const char *c, const char *r, const c
   if (bytes) {
     const uint64_t pol = evict_first_policy();
     bulk_load(stage, c + off, bytes, bar, pol);
-    bulk_load(stage + kBatchBytes, r + off, bytes, bar, pol);
-    if constexpr (NIN == 1) bulk_load(stage + 2 * kBatchBytes, x + off, bytes, bar, pol);
+    bulk_load(stage + batch_bytes(NIN), r + off, bytes, bar, pol);
+    if constexpr (NIN == 1) bulk_load(stage + 2 * batch_bytes(NIN), x + off, bytes, bar, pol);
   }
 }
 
@@ -1089,10 +1089,11 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
-  constexpr int BATCH = STEP * kSteps;
-  constexpr uint32_t BB = BATCH * EB;  // bytes of one tensor's batch (kBatchBytes)
+  constexpr int KS = batch_steps(NIN);
+  constexpr int BATCH = STEP * KS;
+  constexpr uint32_t BB = BATCH * EB;  // bytes of one tensor's batch (batch_bytes)
   constexpr uint32_t NST = ring_stages(NIN);
-  constexpr int STAGE = ring_streams(NIN) * kBatchBytes;
+  constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
   constexpr int kPoll = kWarps;  // batches between a warp's readings of the case-wide maxima
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t *g_thr = P->g_thr;
@@ -1191,24 +1192,24 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     }
     if ((int64_t)off <= full_max) {
 #pragma unroll 1
-      for (int u = 0; u < kSteps; ++u) {
+      for (int u = 0; u < KS; ++u) {
         const uint4 cv = lds_v4(stage + u * 512);
-        const uint4 rv = lds_v4(stage + kBatchBytes + u * 512);
+        const uint4 rv = lds_v4(stage + BB + u * 512);
         uint4 xv = make_uint4(0, 0, 0, 0);
-        if constexpr (NIN == 1) xv = lds_v4(stage + 2 * kBatchBytes + u * 512);
+        if constexpr (NIN == 1) xv = lds_v4(stage + 2 * BB + u * 512);
         step<DT, NIN>(P, L, W, R, cv, rv, xv, erel + u * STEP + lane_off);
       }
     } else {
       // the case's last batch, or a case that is not 16-byte aligned
       const uint32_t pel = pbytes / EB;  // elements in the piece
       const uint32_t nfull = P->cd.vec_ok ? (pel - erel) / STEP : 0u;
-      for (int u = 0; u < kSteps; ++u) {
+      for (int u = 0; u < KS; ++u) {
         const uint32_t e = erel + u * STEP + lane_off;
         if ((uint32_t)u < nfull) {
           const uint4 cv = lds_v4(stage + u * 512);
-          const uint4 rv = lds_v4(stage + kBatchBytes + u * 512);
+          const uint4 rv = lds_v4(stage + BB + u * 512);
           uint4 xv = make_uint4(0, 0, 0, 0);
-          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * kBatchBytes + u * 512);
+          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * BB + u * 512);
           step<DT, NIN>(P, L, W, R, cv, rv, xv, e);
         } else if (erel + u * STEP < pel) {
           const int n = e >= pel ? 0 : (pel - e > (uint32_t)V ? V : (int)(pel - e));
@@ -1226,7 +1227,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
       R.track_r = R.track_r && !__any_sync(0xffffffffu, (R.racc & mag) != 0u);
     }
-    if (++flush == kFlushBatches) {
+    if (++flush == flush_batches(NIN)) {
       sse_flush(R.sse);
       flush = 0;
     }
@@ -1248,7 +1249,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
-  constexpr int STAGE = ring_streams(NIN) * kBatchBytes;
+  constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
   extern __shared__ __align__(128) uint8_t dsm[];
   __shared__ PieceSh P;
   __shared__ LaneSh lanes[kThreads];
