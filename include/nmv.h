@@ -200,7 +200,8 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
 int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out);
 
 /* Release what one nmv_validate / nmv_validate_batch call returned.  NULL
- * is accepted. */
+ * is accepted.  (The block is pinned host memory, which the library keeps
+ * for reuse by later calls.) */
 void nmv_result_free(nmv_result *r);
 
 /* Static text for a status code. */

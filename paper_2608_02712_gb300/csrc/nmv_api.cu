@@ -447,33 +447,56 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.fk_off = (int64_t)g.fk_off;
 }
 
-int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
-  if (out == nullptr) return fail(NMV_EINVAL, "out is NULL");
-  *out = nullptr;
-  if (cases == nullptr && n > 0) return fail(NMV_EINVAL, "cases is NULL");
-  if (n < 0 || n > NMV_MAX_CASES) return fail(NMV_EINVAL, "case count out of range");
-  std::vector<Geo> geo((size_t)n);
-  for (int64_t i = 0; i < n; ++i) {
-    const int rc = check_case(cases[i], &geo[i]);
-    if (rc) {
-      char buf[64];
-      std::snprintf(buf, sizeof buf, "case %lld: ", (long long)i);
-      g_err = buf + g_err;
-      return rc;
-    }
-  }
-  if (n == 0) return NMV_OK;
-
-  std::lock_guard<std::mutex> lock(g_mu);
-  int dev = -1;
-  DeviceState *S = nullptr;
-  int rc = probe_device(&dev, &S);
-  if (rc) return rc;
-  cudaStream_t st = (cudaStream_t)stream;
-
-  // ---- plan: one group per (element type, input class), each with a
-  // full grid of its own, launched back to back on the stream.
+// The plan of the last call on each device: reused when the next call
+// validates the same case set (same buffers, shapes and parameters), so a
+// repeated call skips planning and, while the workspace is unchanged, the
+// descriptor upload.
+struct PlanCache {
+  bool valid = false;
+  std::vector<uint8_t> key;
   std::vector<Group> groups;
+  std::vector<CaseDesc> desc;
+  std::vector<Piece> pieces;
+  int64_t np = 0, n_batches = 0;
+  size_t out_size = 0;
+  void *uploaded_ws = nullptr;  // workspace holding this plan's descriptors
+};
+PlanCache g_plan[kMaxDevices];
+
+// Identity of a case set for the plan cache: every field a plan depends on.
+void case_key(const nmv_case *cases, int64_t n, std::vector<uint8_t> &key) {
+  key.clear();
+  auto put = [&](const void *p, size_t b) {
+    const uint8_t *q = (const uint8_t *)p;
+    key.insert(key.end(), q, q + b);
+  };
+  auto put_t = [&](const nmv_tensor &t) {
+    put(&t.data, sizeof(t.data));
+    put(&t.dtype, 4);
+    put(&t.rank, 4);
+    if (t.rank > 0) put(t.shape, 8 * (size_t)t.rank);
+  };
+  put(&n, 8);
+  for (int64_t i = 0; i < n; ++i) {
+    const nmv_case &c = cases[i];
+    put_t(c.cand);
+    put_t(c.ref);
+    put(&c.n_inputs, 4);
+    for (int j = 0; j < c.n_inputs; ++j) put_t(c.inputs[j]);
+    put(&c.rtol, 8);
+    put(&c.atol, 8);
+    put(&c.tile_rows, 8);
+    put(&c.tile_cols, 8);
+    put(&c.first_k, 8);
+  }
+}
+
+// Plan a case set: groups (one per element type and input class, each with
+// a full grid of its own, launched back to back), pieces and descriptors.
+int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo, DeviceState *S,
+                   PlanCache &C) {
+  C.valid = false;
+  C.groups.clear();
   {
     int slot[4][3];
     for (auto &row : slot)
@@ -483,16 +506,16 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       const int nin = nin_class(cases[i], geo[i]);
       int &gi = slot[geo[i].dt][nin + 1];
       if (gi < 0) {
-        gi = (int)groups.size();
-        groups.emplace_back();
-        groups.back().dt = geo[i].dt;
-        groups.back().nin = nin;
+        gi = (int)C.groups.size();
+        C.groups.emplace_back();
+        C.groups.back().dt = geo[i].dt;
+        C.groups.back().nin = nin;
       }
-      groups[gi].ids.push_back(i);
+      C.groups[gi].ids.push_back(i);
     }
   }
   int64_t np = 0;
-  for (Group &G : groups) {
+  for (Group &G : C.groups) {
     int64_t total_bytes = 0;
     size_t prof_smem = kShHeadWords * 4;
     for (int64_t i : G.ids) {
@@ -531,24 +554,24 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     np += (int64_t)G.plan.pieces.size();
   }
 
-  // ---- descriptors (pieces of a case are contiguous within its group)
-  std::vector<CaseDesc> desc((size_t)n);
-  std::vector<Piece> all_pieces;
-  all_pieces.reserve((size_t)np);
+  // descriptors (pieces of a case are contiguous within its group)
+  C.desc.assign((size_t)n, CaseDesc{});
+  C.pieces.clear();
+  C.pieces.reserve((size_t)np);
   size_t out_size = kCallHeader;
   for (int64_t i = 0; i < n; ++i) {
-    fill_desc(cases[i], geo[i], desc[i]);
-    desc[i].out_off = (int64_t)out_size;
+    fill_desc(cases[i], geo[i], C.desc[i]);
+    C.desc[i].out_off = (int64_t)out_size;
     out_size += geo[i].out_size;
-    desc[i].piece_begin = desc[i].piece_end = 0;
-    desc[i].batch_begin = desc[i].batch_end = 0;
+    C.desc[i].piece_begin = C.desc[i].piece_end = 0;
+    C.desc[i].batch_begin = C.desc[i].batch_end = 0;
   }
   int64_t n_batches = 0;
-  for (Group &G : groups) {
+  for (Group &G : C.groups) {
     for (size_t k = 0; k < G.plan.pieces.size(); ++k) {
       Piece p = G.plan.pieces[k];
       const int64_t gid = G.piece_base + (int64_t)k;
-      CaseDesc &d = desc[p.case_id];
+      CaseDesc &d = C.desc[p.case_id];
       p.batch_base = n_batches;
       const int64_t nb = piece_batches(p.begin, p.end, G.dt, G.nin);
       if (d.piece_end == 0) {
@@ -558,31 +581,156 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
       d.piece_end = gid + 1;
       n_batches += nb;
       d.batch_end = n_batches;
-      all_pieces.push_back(p);
+      C.pieces.push_back(p);
     }
   }
+  C.np = np;
+  C.n_batches = n_batches;
+  C.out_size = out_size;
+  C.uploaded_ws = nullptr;
+  C.valid = true;
+  return NMV_OK;
+}
+
+// ---- result blocks
+// Each call's results live in one pinned host block: the device copies its
+// packed result straight into it and the nmv_result arrays point into that
+// copy.  Released blocks are kept for reuse (a few, the largest first), so a
+// steady stream of calls allocates nothing after the first.
+struct ArenaPool {
+  std::mutex mu;
+  std::vector<std::pair<void *, size_t>> free_blocks;
+  std::vector<std::pair<void *, size_t>> live;
+} g_arenas;
+constexpr size_t kArenaKeep = 8;
+
+void *arena_get(size_t bytes) {
+  {
+    std::lock_guard<std::mutex> lock(g_arenas.mu);
+    size_t best = SIZE_MAX;
+    for (size_t i = 0; i < g_arenas.free_blocks.size(); ++i)
+      if (g_arenas.free_blocks[i].second >= bytes &&
+          (best == SIZE_MAX || g_arenas.free_blocks[i].second < g_arenas.free_blocks[best].second))
+        best = i;
+    if (best != SIZE_MAX) {
+      auto blk = g_arenas.free_blocks[best];
+      g_arenas.free_blocks.erase(g_arenas.free_blocks.begin() + (ptrdiff_t)best);
+      g_arenas.live.push_back(blk);
+      return blk.first;
+    }
+  }
+  void *p = nullptr;
+  const size_t cap = std::max(bytes, (size_t)65536);
+  if (cudaHostAlloc(&p, cap, cudaHostAllocDefault) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lock(g_arenas.mu);
+  g_arenas.live.push_back({p, cap});
+  return p;
+}
+
+void arena_put(void *p) {
+  if (!p) return;
+  void *drop = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_arenas.mu);
+    for (size_t i = 0; i < g_arenas.live.size(); ++i) {
+      if (g_arenas.live[i].first == p) {
+        auto blk = g_arenas.live[i];
+        g_arenas.live.erase(g_arenas.live.begin() + (ptrdiff_t)i);
+        g_arenas.free_blocks.push_back(blk);
+        if (g_arenas.free_blocks.size() > kArenaKeep) {
+          // keep the largest blocks
+          size_t small = 0;
+          for (size_t j = 1; j < g_arenas.free_blocks.size(); ++j)
+            if (g_arenas.free_blocks[j].second < g_arenas.free_blocks[small].second) small = j;
+          drop = g_arenas.free_blocks[small].first;
+          g_arenas.free_blocks.erase(g_arenas.free_blocks.begin() + (ptrdiff_t)small);
+        }
+        break;
+      }
+    }
+  }
+  if (drop) cudaFreeHost(drop);
+}
+
+int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
+  if (out == nullptr) return fail(NMV_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (cases == nullptr && n > 0) return fail(NMV_EINVAL, "cases is NULL");
+  if (n < 0 || n > NMV_MAX_CASES) return fail(NMV_EINVAL, "case count out of range");
+  std::vector<Geo> geo((size_t)n);
+  for (int64_t i = 0; i < n; ++i) {
+    const int rc = check_case(cases[i], &geo[i]);
+    if (rc) {
+      char buf[64];
+      std::snprintf(buf, sizeof buf, "case %lld: ", (long long)i);
+      g_err = buf + g_err;
+      return rc;
+    }
+  }
+  if (n == 0) return NMV_OK;
+
+  std::lock_guard<std::mutex> lock(g_mu);
+  int dev = -1;
+  DeviceState *S = nullptr;
+  int rc = probe_device(&dev, &S);
+  if (rc) return rc;
+  cudaStream_t st = (cudaStream_t)stream;
+
+  // ---- plan (cached for a repeated case set)
+  static thread_local std::vector<uint8_t> key;
+  case_key(cases, n, key);
+  PlanCache &C = g_plan[dev];
+  if (!(C.valid && C.key == key)) {
+    rc = make_call_plan(cases, n, geo, S, C);
+    if (rc) return rc;
+    C.key = key;
+  }
+  const std::vector<Group> &groups = C.groups;
+  const int64_t np = C.np;
+  const size_t out_size = C.out_size;
 
   // ---- workspace layout
   const size_t sz_cases = align_up(sizeof(CaseDesc) * n, 256);
   const size_t sz_pieces = align_up(sizeof(Piece) * std::max<int64_t>(np, 1), 256);
   const size_t table = sz_cases + sz_pieces;
   const size_t sz_part = align_up(sizeof(Partial) * std::max<int64_t>(np, 1), 256);
-  const size_t sz_segc = align_up(sizeof(int32_t) * std::max<int64_t>(n_batches, 1), 256);
+  const size_t sz_segc = align_up(sizeof(int32_t) * std::max<int64_t>(C.n_batches, 1), 256);
   // published thresholds (2 x u32 per case), then one piece counter per group
   const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n + sizeof(unsigned long long) * groups.size(), 256);
   const size_t sz_sse = align_up(sizeof(double) * kSseBlocksHost, 256);
   const size_t o_part = table, o_segc = o_part + sz_part;
   const size_t o_sse = o_segc + sz_segc, o_thr = o_sse + sz_sse, o_out = o_thr + sz_thr;
   const size_t ws = o_out + out_size;
-  rc = ensure_workspace(*S, ws, table + out_size);
+  rc = ensure_workspace(*S, ws, table);
   if (rc) return rc;
   uint8_t *W = (uint8_t *)S->ws;
-  uint8_t *H = (uint8_t *)S->pinned;
-  std::memcpy(H, desc.data(), sizeof(CaseDesc) * n);
-  if (np) std::memcpy(H + sz_cases, all_pieces.data(), sizeof(Piece) * np);
 
-  cudaError_t e = cudaMemcpyAsync(W, H, table, cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
+  // ---- result block: the results, then the device's packed result, then
+  // the first-K coordinates
+  const size_t res_bytes = align_up(sizeof(nmv_result) * n, 256);
+  size_t coord_bytes = 0;
+  for (int64_t i = 0; i < n; ++i) coord_bytes += 8 * (size_t)cases[i].first_k * (size_t)cases[i].cand.rank;
+  uint8_t *arena = (uint8_t *)arena_get(res_bytes + out_size + coord_bytes);
+  if (!arena) return fail(NMV_ENOMEM, "cudaHostAlloc result block");
+  struct ArenaGuard {
+    uint8_t *p;
+    ~ArenaGuard() { arena_put(p); }
+  } guard{arena};
+  uint8_t *HO = arena + res_bytes;
+
+  cudaError_t e = cudaSuccess;
+  const bool upload = C.uploaded_ws != S->ws;
+  if (upload) {
+    uint8_t *H = (uint8_t *)S->pinned;
+    std::memcpy(H, C.desc.data(), sizeof(CaseDesc) * n);
+    if (np) std::memcpy(H + sz_cases, C.pieces.data(), sizeof(Piece) * np);
+    e = cudaMemcpyAsync(W, H, table, cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
+    C.uploaded_ws = S->ws;
+  }
   e = cudaMemsetAsync(W + o_thr, 0, sz_thr + out_size, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   const CaseDesc *d_cases = (const CaseDesc *)W;
@@ -613,8 +761,8 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   for (size_t gi = 0; gi < groups.size(); ++gi) {
     const Group &G = groups[gi];
     e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_ctr + gi,
-                    (int64_t)G.plan.pieces.size(), G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out,
-                    (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
+                    (int64_t)G.plan.pieces.size(), G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc),
+                    W + o_out, (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   if (prof) cudaEventRecord(g_prof.ev[1], st);
@@ -622,7 +770,6 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
                       W + o_out, (int)n, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   if (prof) cudaEventRecord(g_prof.ev[2], st);
-  uint8_t *HO = H + table;
   e = cudaMemcpyAsync(HO, W + o_out, out_size, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (results)");
   e = cudaStreamSynchronize(st);
@@ -633,9 +780,9 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   // Cases whose differences are all tiny (max |d| < 2^-38): the fp32 squares
   // of the scan pass may have lost terms, so their SSE is recomputed in fp64.
   for (int64_t i = 0; i < n; ++i) {
-    OutHeader *oh = (OutHeader *)(HO + desc[i].out_off);
+    OutHeader *oh = (OutHeader *)(HO + C.desc[i].out_off);
     if (oh->max_abs > 0.0 && oh->max_abs < 0x1p-38) {
-      double *dst = (double *)(W + o_out + desc[i].out_off + offsetof(OutHeader, sse));
+      double *dst = (double *)(W + o_out + C.desc[i].out_off + offsetof(OutHeader, sse));
       e = launch_sse64(d_cases + i, (double *)(W + o_sse), dst, st);
       if (e != cudaSuccess) return cuda_fail(e, "fp64 SSE launch");
       e = cudaMemcpyAsync(&oh->sse, dst, sizeof(double), cudaMemcpyDeviceToHost, st);
@@ -653,7 +800,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     P.scan_ms = a;
     P.finalize_ms = b;
     P.kernel_launches = (int64_t)groups.size() + 1;
-    P.h2d_bytes = (int64_t)table;
+    P.h2d_bytes = upload ? (int64_t)table : 0;
     P.d2h_bytes = (int64_t)out_size;
     P.slow_steps = (int64_t)st4[0];
     P.light_steps = (int64_t)st4[4];
@@ -667,28 +814,12 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     g_prof.valid = true;
   }
 
-  // ---- result arena
-  size_t bytes = align_up(sizeof(nmv_result) * n, 16);
-  for (int64_t i = 0; i < n; ++i) {
-    const OutHeader *oh = (const OutHeader *)(HO + desc[i].out_off);
-    const nmv_case &c = cases[i];
-    const int64_t k = oh->k_out;
-    bytes += 8 * (size_t)(geo[i].GR * geo[i].GC + c.tile_rows + c.tile_cols);
-    bytes += 8 * (size_t)k * (3 + (size_t)c.cand.rank);
-    bytes += 8 * (size_t)c.n_inputs;
-  }
-  uint8_t *arena = (uint8_t *)std::malloc(bytes);
-  if (!arena) return fail(NMV_ENOMEM, "malloc result arena");
+  // ---- results: scalar fields, arrays pointing into the packed copy
   nmv_result *res = (nmv_result *)arena;
-  uint8_t *cur = arena + align_up(sizeof(nmv_result) * n, 16);
-  auto take = [&](size_t nbytes) {
-    uint8_t *p = cur;
-    cur += nbytes;
-    return p;
-  };
+  int64_t *coords = (int64_t *)(HO + out_size);
   for (int64_t i = 0; i < n; ++i) {
-    const uint8_t *ob = HO + desc[i].out_off;
-    const OutHeader *oh = (const OutHeader *)ob;
+    uint8_t *ob = HO + C.desc[i].out_off;
+    OutHeader *oh = (OutHeader *)ob;
     const nmv_case &c = cases[i];
     const Geo &g = geo[i];
     nmv_result &r = res[i];
@@ -715,38 +846,29 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     r.grid_cols = g.GC;
     r.tile_rows = c.tile_rows;
     r.tile_cols = c.tile_cols;
-    const size_t nb = (size_t)(g.GR * g.GC);
-    r.tile_hist = (int64_t *)take(8 * nb);
-    std::memcpy(r.tile_hist, ob + g.hist_off, 8 * nb);
-    r.row_prof = (int64_t *)take(8 * (size_t)c.tile_rows);
-    std::memcpy(r.row_prof, ob + g.rowp_off, 8 * (size_t)c.tile_rows);
-    r.col_prof = (int64_t *)take(8 * (size_t)c.tile_cols);
-    std::memcpy(r.col_prof, ob + g.colp_off, 8 * (size_t)c.tile_cols);
+    r.tile_hist = (int64_t *)(ob + g.hist_off);
+    r.row_prof = (int64_t *)(ob + g.rowp_off);
+    r.col_prof = (int64_t *)(ob + g.colp_off);
     const int64_t k = oh->k_out;
     r.k_out = k;
-    r.fk_index = (int64_t *)take(8 * (size_t)k);
-    r.fk_coords = (int64_t *)take(8 * (size_t)k * (size_t)c.cand.rank);
-    r.fk_cand = (double *)take(8 * (size_t)k);
-    r.fk_ref = (double *)take(8 * (size_t)k);
-    const int64_t *fki = (const int64_t *)(ob + g.fk_off);
-    const double *fkc = (const double *)(fki + c.first_k);
-    const double *fkr = fkc + c.first_k;
-    std::memcpy(r.fk_index, fki, 8 * (size_t)k);
-    std::memcpy(r.fk_cand, fkc, 8 * (size_t)k);
-    std::memcpy(r.fk_ref, fkr, 8 * (size_t)k);
+    r.fk_index = (int64_t *)(ob + g.fk_off);
+    r.fk_cand = (double *)(r.fk_index + c.first_k);
+    r.fk_ref = r.fk_cand + c.first_k;
+    r.fk_coords = coords;
     for (int64_t t = 0; t < k; ++t) {
       int64_t idx = r.fk_index[t];
       for (int d = c.cand.rank - 1; d >= 0; --d) {
-        const int64_t s = c.cand.shape[d];
-        r.fk_coords[t * c.cand.rank + d] = s > 0 ? idx % s : 0;
-        idx = s > 0 ? idx / s : 0;
+        const int64_t sd = c.cand.shape[d];
+        coords[t * c.cand.rank + d] = sd > 0 ? idx % sd : 0;
+        idx = sd > 0 ? idx / sd : 0;
       }
     }
+    coords += (size_t)c.first_k * (size_t)c.cand.rank;
     r.n_inputs = c.n_inputs;
     r.passthrough_input = oh->passthrough;
-    r.input_eq = (int64_t *)take(8 * (size_t)c.n_inputs);
-    for (int j = 0; j < c.n_inputs; ++j) r.input_eq[j] = oh->input_eq[j];
+    r.input_eq = oh->input_eq;
   }
+  guard.p = nullptr;  // handed to the caller
   *out = res;
   g_err.clear();
   return NMV_OK;
@@ -999,7 +1121,7 @@ int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out) 
   return run_noalloc(c, cuda_stream, out);
 }
 
-void nmv_result_free(nmv_result *r) { std::free(r); }
+void nmv_result_free(nmv_result *r) { arena_put(r); }
 
 const char *nmv_status_string(int status) {
   switch (status) {

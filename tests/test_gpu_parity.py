@@ -152,3 +152,50 @@ def test_exact_equal_tensors_fast():
     got = validate(x, x.clone(), rtol=0, atol=0, tile=(1, 4096), first_k=8)
     assert got["pass"] and got["mismatch"] == 0 and got["max_abs"] == 0.0
     assert got["argmax_abs"] == 0 and got["argmax_rel"] == int((x != 0).nonzero()[0])
+
+
+def test_repeated_call_on_rewritten_buffers():
+    # The library reuses the plan of a repeated case set (same buffers,
+    # shapes and parameters); the values must still be read afresh.
+    case = workloads.c1()
+    cand, ref = case["cand"].cuda(), case["ref"].cuda()
+    args = dict(rtol=case["rtol"], atol=case["atol"], tile=case["tile"], first_k=case["first_k"])
+    first = validate(cand, ref, **args)
+    assert_same(first, oracle.validate(cand.cpu(), ref.cpu(), **args), "first call")
+    g = torch.Generator().manual_seed(123)
+    cand.copy_(ref + torch.randn(ref.shape, generator=g).cuda() * 0.5)
+    second = validate(cand, ref, **args)
+    assert_same(second, oracle.validate(cand.cpu(), ref.cpu(), **args), "rewritten buffers")
+    assert second["mismatch"] != first["mismatch"]
+    cand.copy_(ref)
+    third = validate(cand, ref, **args)
+    assert third["pass"] and third["k_out"] == 0 and third["tile_hist"].sum() == 0
+
+
+def test_results_stay_valid_until_freed():
+    import ctypes
+    from paper_2608_02712_gb300 import nmv as m
+    lib = m.load()
+    a = workloads.c1()
+    b = workloads.c4(numel=(1 << 16) + 5)
+    keep = []
+    outs = []
+    for case in (a, b, a):
+        c, k = m.make_case(case["cand"].cuda(), case["ref"].cuda(), rtol=case["rtol"], atol=case["atol"],
+                           tile=case["tile"], first_k=case["first_k"])
+        keep.append(k)
+        out = ctypes.POINTER(m.Result)()
+        assert lib.nmv_validate(ctypes.byref(c), None, ctypes.byref(out)) == 0
+        outs.append(out)
+    d = [m.result_to_dict(o[0]) for o in outs]
+    assert_same(d[2], d[0], "same case twice")
+    lib.nmv_result_free(outs[1])
+    # a call after a free reuses the block; the live results do not change
+    c, k = m.make_case(b["cand"].cuda(), b["ref"].cuda(), rtol=b["rtol"], atol=b["atol"], tile=b["tile"],
+                       first_k=b["first_k"])
+    out = ctypes.POINTER(m.Result)()
+    assert lib.nmv_validate(ctypes.byref(c), None, ctypes.byref(out)) == 0
+    assert_same(m.result_to_dict(out[0]), d[1], "reused block")
+    assert_same(m.result_to_dict(outs[0][0]), d[0], "live result after reuse")
+    for o in (outs[0], outs[2], out):
+        lib.nmv_result_free(o)
