@@ -38,10 +38,12 @@
 // the order of their fp64 roundings; only inexact differences fall back to
 // fp64 arithmetic.
 // The SSE is accumulated per lane as two float-float pairs (even and odd
-// elements of each vector) with Knuth's TwoSum, flushed to fp64 every few
-// batches; the exact step feeds the same pairs with the same arithmetic
-// (plus 2 s e for an inexact c - r, e from TwoSum), so the result is
-// bit-identical whichever path an element takes.  Terms with |s| > 2^56 are
+// elements of each vector) with Knuth's TwoSum; the exact step feeds the same
+// pairs with the same arithmetic (plus 2 s e for an inexact c - r, e from
+// TwoSum), so the result does not depend on which path an element takes.
+// Each batch's lane sums are combined by a fixed butterfly and stored per
+// batch, and a piece adds its batches in order: the SSE does not depend on
+// which warp took which batch either, so it is bit-identical run to run.  Terms with |s| > 2^56 are
 // squared in fp64.  When max |d| < 2^-38 the fp32 squares may lose tiny
 // terms; the host then recomputes that case's SSE in fp64 (sse64 kernels).
 #pragma once
@@ -55,9 +57,6 @@
 
 namespace nmv {
 
-// The SSE's float-float pairs go to fp64 every flush_batches(nin) batches
-// (about 32 warp steps, at most 128 terms per pair).
-NMV_CHD int flush_batches(int nin) { return (32 + batch_steps(nin) - 1) / batch_steps(nin); }
 constexpr float kHuge = 0x1p56f;
 constexpr float kMarginLo = 1.0f - 0x1p-20f;
 
@@ -197,17 +196,6 @@ __device__ __forceinline__ void ff_pair(SseAcc &a, float2 s) {
   a.hi = t;
 }
 
-__device__ __forceinline__ void sse_flush(SseAcc &a) {
-  // TwoSum of the two slots' high parts, then two fp64 additions.
-  const float h = __fadd_rn(a.hi.x, a.hi.y);
-  const float hb = __fsub_rn(h, a.hi.x);
-  const float herr = __fadd_rn(__fsub_rn(a.hi.x, __fsub_rn(h, hb)), __fsub_rn(a.hi.y, hb));
-  const float l = __fadd_rn(__fadd_rn(a.lo.x, a.lo.y), herr);
-  a.acc = __dadd_rn(a.acc, __dadd_rn((double)h, (double)l));
-  a.hi = make_float2(0.f, 0.f);
-  a.lo = make_float2(0.f, 0.f);
-}
-
 // ------------------------------------------------------------ reductions
 // Best (value, index): the larger value wins, equal values go to the lower
 // index.  Values are >= 0 or -1 (none), so their bit patterns order as
@@ -244,6 +232,34 @@ __device__ __forceinline__ T warp_reduce(T v, Op op) {
 #pragma unroll
   for (int o = 16; o; o >>= 1) v = op(v, __shfl_xor_sync(0xffffffffu, v, o));
   return v;
+}
+
+// (h, l) += (h2, l2) for float-float pairs: TwoSum of the high parts (its
+// error is exact, so the result does not depend on the operand order).
+__device__ __forceinline__ void ff_add(float &h, float &l, float h2, float l2) {
+  const float t = __fadd_rn(h, h2);
+  const float bp = __fsub_rn(t, h);
+  const float err = __fadd_rn(__fsub_rn(h, __fsub_rn(t, bp)), __fsub_rn(h2, bp));
+  h = t;
+  l = __fadd_rn(__fadd_rn(l, l2), err);
+}
+
+// Store the warp's SSE of one batch (lane 0 writes) and restart the lane
+// accumulators: the lane's two slots, then a butterfly over the warp, after
+// which every lane holds the same bits.
+__device__ __forceinline__ void batch_sse_store(SseAcc &a, BatchSse *dst) {
+  float h = a.hi.x, l = a.lo.x;
+  ff_add(h, l, a.hi.y, a.lo.y);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float h2 = __shfl_xor_sync(0xffffffffu, h, o), l2 = __shfl_xor_sync(0xffffffffu, l, o);
+    ff_add(h, l, h2, l2);
+  }
+  double acc = a.acc;
+  if (__any_sync(0xffffffffu, acc != 0.0)) acc = warp_reduce(acc, [](double x, double y) { return __dadd_rn(x, y); });
+  if ((threadIdx.x & 31) == 0) *dst = BatchSse{h, l, acc};
+  a.hi = a.lo = make_float2(0.f, 0.f);
+  a.acc = 0.0;
 }
 
 // ----------------------------------------------------------------- state
@@ -1074,6 +1090,7 @@ struct RingPos {
 };
 
 constexpr uint32_t kNoBatch = 0xffffffffu;
+constexpr uint32_t kChunk = 4;  // batches a warp claims at once (one SSE sum each)
 
 // Sweep batches of a piece (each batch_elems elements; only a case's last
 // batch may be shorter) through this warp's ring, writing each batch's
@@ -1084,8 +1101,8 @@ constexpr uint32_t kNoBatch = 0xffffffffu;
 // kMaxPiece elements).
 template <int DT, int NIN>
 __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
-                                      int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
-                                      uint32_t *err) {
+                                      int32_t *batch_count, BatchSse *bsse, uint8_t *ring, uint64_t *bars,
+                                      RingPos &rp, uint32_t *err) {
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
@@ -1109,14 +1126,25 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   int32_t *bcount = batch_count + pc.batch_base;
   // lane 0: claim the next batch into stage st_i and issue its copies
   uint32_t st_i = rp.stage;
-  bool claiming = true;
+  bool claiming = true;  // chunks may remain
+  bool live = true;      // the end of the piece has not been marked yet
+  // Batches are claimed kChunk at a time (next_batch counts chunks); a
+  // warp issues a chunk's batches in order before it claims the next.
+  uint32_t i_next = 0, i_left = 0;
   auto issue_next = [&]() {
-    const uint32_t b = claiming ? atomicAdd(&P->next_batch, 1u) : nb;
-    if (b >= nb) {
-      claiming = false;
+    if (i_left == 0 && claiming) {
+      const uint32_t c = atomicAdd(&P->next_batch, 1u);
+      i_next = c * kChunk;
+      i_left = i_next < nb ? (nb - i_next < kChunk ? nb - i_next : kChunk) : 0u;
+      if (i_left == 0) claiming = false;
+    }
+    if (i_left == 0) {
       W->stage_b[st_i] = kNoBatch;
+      live = false;
       return;
     }
+    const uint32_t b = i_next++;
+    --i_left;
     W->stage_b[st_i] = b;
     const uint32_t off = b * BB;
     uint32_t bytes = 0;
@@ -1130,12 +1158,11 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
   };
   if (lane == 0) {
-    for (uint32_t i = 0; i < NST - 1 && claiming; ++i) issue_next();
+    for (uint32_t i = 0; i < NST - 1 && live; ++i) issue_next();
     W->mism_tot = 0;
   }
   __syncwarp();
   bool dead = false;
-  int flush = 0;
   // The block's view of the case-wide maxima is read every batch; the case's
   // own value is read by one warp of the block per batch round (each warp
   // every kPoll batches, its load kPoll batches ahead of its use, so the L2
@@ -1149,7 +1176,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     const uint32_t off = b * BB;
     __syncwarp();
     if (lane == 0) {
-      if (claiming) issue_next();  // refills the stage released last batch
+      if (live) issue_next();  // refills the stage released last batch
       W->mism = 0;
     }
     if ((j + warp) % kPoll == 0) {
@@ -1227,12 +1254,10 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
       R.track_r = R.track_r && !__any_sync(0xffffffffu, (R.racc & mag) != 0u);
     }
-    if (++flush == flush_batches(NIN)) {
-      sse_flush(R.sse);
-      flush = 0;
-    }
+    // the SSE of a chunk (kChunk batches, or the piece's rest) is stored at
+    // its first batch
+    if ((b + 1) % kChunk == 0 || b + 1 == nb) batch_sse_store(R.sse, bsse + pc.batch_base + (b - b % kChunk));
   }
-  sse_flush(R.sse);
 }
 
 // ------------------------------------------------------------ the kernel
@@ -1246,7 +1271,8 @@ template <int DT, int NIN>
 __global__ void __launch_bounds__(kThreads, 2)
     scan_kernel(const CaseDesc *__restrict__ cases, const Piece *__restrict__ pieces,
                 unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base, Partial *partials,
-                int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
+                int32_t *batch_count, BatchSse *bsse, uint8_t *out, uint32_t *g_thr, unsigned long long *stats,
+                uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
   constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
@@ -1342,7 +1368,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
-    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
+    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, bsse, ring, bars, rpos, err);
     __syncwarp();
     if (stats && lane == 0)
       for (int k = 0; k < 9; ++k)
@@ -1350,7 +1376,6 @@ __global__ void __launch_bounds__(kThreads, 2)
 
     // ---- lanes -> warps -> the piece's partial
     const Best a = best_warp(abs_best64(L)), r = best_warp(rel_best64(L));
-    const double sse = warp_reduce(R.sse.acc, [](double x, double y) { return __dadd_rn(x, y); });
     const uint32_t cacc = warp_reduce(R.cacc | L->cacc, [](uint32_t x, uint32_t y) { return x | y; });
     const uint32_t racc = warp_reduce(R.racc | L->racc, [](uint32_t x, uint32_t y) { return x | y; });
     int eqs[NMV_MAX_INPUTS];
@@ -1372,7 +1397,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       w.arg_abs = a.i;
       w.best_rel = r.v;
       w.arg_rel = r.i;
-      w.sse = sse;
+      w.sse = 0.0;
       w.cacc = cacc;
       w.racc = racc;
 #pragma unroll
@@ -1394,6 +1419,19 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int64_t t = threadIdx.x; t < P.cd.tw; t += kThreads)
         if (P.sh_col[t]) atomicAdd(&P.g_col[t], (unsigned long long)P.sh_col[t]);
     }
+    {
+      // the piece's SSE: its chunks in order, thread t taking chunks t,
+      // t + kThreads, ..., then a fixed butterfly per warp and the warps in
+      // order
+      const int64_t nbp = piece_batches(pc.begin, pc.end, DT, NIN);
+      const BatchSse *bs = bsse + pc.batch_base;
+      double v = 0.0;
+      for (int64_t b = (int64_t)threadIdx.x * kChunk; b < nbp; b += (int64_t)kThreads * kChunk)
+        v = __dadd_rn(v, __dadd_rn(__dadd_rn((double)bs[b].hi, (double)bs[b].lo), bs[b].acc));
+      v = warp_reduce(v, [](double x, double y) { return __dadd_rn(x, y); });
+      if (lane == 0) red[warp].sse = v;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
       Partial Q;
       Q.cnt[0] = 0;
@@ -1431,8 +1469,8 @@ struct ScanOps {
   static int occupancy(int nin, size_t smem);
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
-                            Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
-                            unsigned long long *stats, uint32_t *err);
+                            Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out,
+                            uint32_t *g_thr, unsigned long long *stats, uint32_t *err);
 };
 
 #define NMV_SCAN_FN(DT, NIN) scan_kernel<DT, NIN>
@@ -1461,17 +1499,18 @@ struct ScanOps {
   cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases, \
                                   const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,  \
                                   int64_t piece_base,                                                     \
-                                  Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr, \
+                                  Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out,  \
+                                  uint32_t *g_thr,                                                        \
                                   unsigned long long *stats, uint32_t *err) {                            \
     if (nin == 0)                                                                                        \
       NMV_SCAN_FN(DT, 0)<<<grid, kThreads, NMV_SCAN_SMEM(0, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
     else if (nin == 1)                                                                                   \
       NMV_SCAN_FN(DT, 1)<<<grid, kThreads, NMV_SCAN_SMEM(1, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
     else                                                                                                 \
       NMV_SCAN_FN(DT, -1)<<<grid, kThreads, NMV_SCAN_SMEM(-1, smem), st>>>(                              \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
     return cudaGetLastError();                                                                           \
   }
 

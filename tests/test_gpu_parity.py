@@ -105,6 +105,22 @@ def test_deterministic_bits():
             assert a[k] == b[k], k
 
 
+def test_deterministic_sse_under_dynamic_scheduling():
+    # Blocks take pieces and warps take batches in whatever order they get
+    # to them; the sum of squared errors must still come out bit-identical.
+    g = torch.Generator(device="cuda").manual_seed(17)
+    ref = torch.randn(3000, 4099, generator=g, device="cuda")
+    cand = ref * (1 + torch.randn(ref.shape, generator=g, device="cuda") * 1e-3)
+    cand[::7, ::5] += 3.0
+    bits = set()
+    for _ in range(4):
+        r = validate(cand, ref, rtol=1e-3, atol=1e-5, tile=(64, 64), first_k=64)
+        bits.add(np.float64(r["sse"]).tobytes())
+    assert len(bits) == 1
+    want = oracle.validate(cand.cpu(), ref.cpu(), rtol=1e-3, atol=1e-5, tile=(64, 64), first_k=64)
+    assert_same(r, want, "dense noisy fp32")
+
+
 def test_first_k_overflowing_segment_lists():
     """Dense mismatches: every segment list overflows, first-K needs re-reads."""
     g = torch.Generator(device="cuda").manual_seed(5)
