@@ -1218,7 +1218,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       rp.phase ^= 1u;
     }
     if ((int64_t)off <= full_max) {
-#pragma unroll 1
+#pragma unroll 2
       for (int u = 0; u < KS; ++u) {
         const uint4 cv = lds_v4(stage + u * 512);
         const uint4 rv = lds_v4(stage + BB + u * 512);
