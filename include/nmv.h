@@ -180,7 +180,7 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
  *    array whose size is 0 may be NULL).  The call fills them and every
  *    scalar field of *out, and leaves the pointers as they were.
  *
- * A case needs about: 20 bytes per batch of 1024 (16-bit types) or 512
+ * A case needs about: 4 bytes per batch of 1024 (16-bit types) or 512
  * (32-bit types) elements (half that with one input of the candidate's type
  * and size), 8 bytes per histogram bin, 8 * (tile_rows + tile_cols) + 24 *
  * first_k bytes, and under 1 MiB of descriptors and partials.  A case that does not fit fails with NMV_EINVAL and a message

@@ -24,8 +24,8 @@ struct ScanOps {
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,
                             int64_t piece_base,
-                            Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out,
-                            uint32_t *g_thr, unsigned long long *stats, uint32_t *err);
+                            Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
+                            unsigned long long *stats, uint32_t *err);
 };
 cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
                             int, cudaStream_t);
@@ -52,21 +52,21 @@ int scan_occupancy(int dt, int nin, size_t smem) {
 
 cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                         const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
-                        Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out, uint32_t *g_thr,
+                        Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                         unsigned long long *stats, uint32_t *err) {
   switch (dt) {
     case NMV_F32:
       return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
-                                      partials, batch_count, bsse, out, g_thr, stats, err);
+                                      partials, batch_count, out, g_thr, stats, err);
     case NMV_F16:
       return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
-                                      partials, batch_count, bsse, out, g_thr, stats, err);
+                                      partials, batch_count, out, g_thr, stats, err);
     case NMV_BF16:
       return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
-                                       partials, batch_count, bsse, out, g_thr, stats, err);
+                                       partials, batch_count, out, g_thr, stats, err);
     default:
       return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
-                                      partials, batch_count, bsse, out, g_thr, stats, err);
+                                      partials, batch_count, out, g_thr, stats, err);
   }
 }
 }  // namespace nmv
@@ -698,12 +698,11 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   const size_t table = sz_cases + sz_pieces;
   const size_t sz_part = align_up(sizeof(Partial) * std::max<int64_t>(np, 1), 256);
   const size_t sz_segc = align_up(sizeof(int32_t) * std::max<int64_t>(C.n_batches, 1), 256);
-  const size_t sz_bsse = align_up(sizeof(BatchSse) * std::max<int64_t>(C.n_batches, 1), 256);
   // published thresholds (2 x u32 per case), then one piece counter per group
   const size_t sz_thr = align_up(sizeof(uint32_t) * 2 * n + sizeof(unsigned long long) * groups.size(), 256);
   const size_t sz_sse = align_up(sizeof(double) * kSseBlocksHost, 256);
-  const size_t o_part = table, o_segc = o_part + sz_part, o_bsse = o_segc + sz_segc;
-  const size_t o_sse = o_bsse + sz_bsse, o_thr = o_sse + sz_sse, o_out = o_thr + sz_thr;
+  const size_t o_part = table, o_segc = o_part + sz_part;
+  const size_t o_sse = o_segc + sz_segc, o_thr = o_sse + sz_sse, o_out = o_thr + sz_thr;
   const size_t ws = o_out + out_size;
   rc = ensure_workspace(*S, ws, table);
   if (rc) return rc;
@@ -763,7 +762,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     const Group &G = groups[gi];
     e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_ctr + gi,
                     (int64_t)G.plan.pieces.size(), G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc),
-                    (BatchSse *)(W + o_bsse), W + o_out, (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
+                    W + o_out, (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   if (prof) cudaEventRecord(g_prof.ev[1], st);
@@ -998,8 +997,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   const size_t sz_part = align_up(sizeof(Partial) * (size_t)std::max<int64_t>(n_pieces, 1), 256);
   const size_t o_segc = o_part + sz_part;
   const size_t sz_segc = align_up(sizeof(int32_t) * (size_t)std::max<int64_t>(n_batches, 1), 256);
-  const size_t o_bsse = o_segc + sz_segc;
-  const size_t o_sse = o_bsse + align_up(sizeof(BatchSse) * (size_t)std::max<int64_t>(n_batches, 1), 256);
+  const size_t o_sse = o_segc + sz_segc;
   const size_t o_thr = o_sse + align_up(sizeof(double) * kSseBlocksHost, 256);
   const size_t o_out = o_thr + 256;
   const size_t need = o_out + kCallHeader + g.out_size;
@@ -1026,8 +1024,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   if (grid > 0) {
     e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (unsigned long long *)(W + o_thr + 8), n_pieces, 0,
-                    (Partial *)(W + o_part), (int32_t *)(W + o_segc), (BatchSse *)(W + o_bsse), W + o_out,
-                    (uint32_t *)(W + o_thr), nullptr,
+                    (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr,
                     (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }

@@ -95,13 +95,6 @@ struct Partial {
   int64_t eq[NMV_MAX_INPUTS];
 };
 
-// One batch's sum of squared errors, as the scan pass leaves it: a
-// float-float pair plus the fp64 sum of the (rare) terms squared in fp64.
-struct BatchSse {
-  float hi, lo;
-  double acc;
-};
-
 // Header of one case's packed result (followed by the arrays).
 struct OutHeader {
   int64_t cnt[8];       // as Partial::cnt, but [7] = n_finite_pairs

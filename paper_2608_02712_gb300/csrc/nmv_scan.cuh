@@ -41,9 +41,10 @@
 // elements of each vector) with Knuth's TwoSum; the exact step feeds the same
 // pairs with the same arithmetic (plus 2 s e for an inexact c - r, e from
 // TwoSum), so the result does not depend on which path an element takes.
-// Each batch's lane sums are combined by a fixed butterfly and stored per
-// batch, and a piece adds its batches in order: the SSE does not depend on
-// which warp took which batch either, so it is bit-identical run to run.  Terms with |s| > 2^56 are
+// A warp's batches within a piece follow a fixed schedule and the lane,
+// warp and piece sums are combined in a fixed order, so the SSE does not
+// depend on which block took which piece either: it is bit-identical run to
+// run.  Terms with |s| > 2^56 are
 // squared in fp64.  When max |d| < 2^-38 the fp32 squares may lose tiny
 // terms; the host then recomputes that case's SSE in fp64 (sse64 kernels).
 #pragma once
@@ -244,30 +245,11 @@ __device__ __forceinline__ void ff_add(float &h, float &l, float h2, float l2) {
   l = __fadd_rn(__fadd_rn(l, l2), err);
 }
 
-// Store the warp's SSE of one batch (lane 0 writes) and restart the lane
-// accumulators: the lane's two slots, then a butterfly over the warp, after
-// which every lane holds the same bits.
-__device__ __forceinline__ void batch_sse_store(SseAcc &a, BatchSse *dst) {
-  float h = a.hi.x, l = a.lo.x;
-  ff_add(h, l, a.hi.y, a.lo.y);
-#pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    const float h2 = __shfl_xor_sync(0xffffffffu, h, o), l2 = __shfl_xor_sync(0xffffffffu, l, o);
-    ff_add(h, l, h2, l2);
-  }
-  double acc = a.acc;
-  if (__any_sync(0xffffffffu, acc != 0.0)) acc = warp_reduce(acc, [](double x, double y) { return __dadd_rn(x, y); });
-  if ((threadIdx.x & 31) == 0) *dst = BatchSse{h, l, acc};
-  a.hi = a.lo = make_float2(0.f, 0.f);
-  a.acc = 0.0;
-}
-
 // ----------------------------------------------------------------- state
 // Piece-constant data, in shared memory.
 struct PieceSh {
   CaseDesc cd;
   int64_t pbegin;  // the piece's first element
-  uint32_t next_batch;  // the piece's next unclaimed batch
   int64_t tr0, tc0;
   int32_t wr, wc, prof_smem, pad;
   int32_t *sh_cls, *sh_row, *sh_col, *sh_hist;
@@ -1090,19 +1072,34 @@ struct RingPos {
 };
 
 constexpr uint32_t kNoBatch = 0xffffffffu;
-constexpr uint32_t kChunk = 4;  // batches a warp claims at once (one SSE sum each)
+// The SSE's float-float pairs go to fp64 every kFlushBatches batches of a
+// lane (at most 128 terms per pair in between).
+constexpr int kFlushBatches = 4;
 
-// Sweep batches of a piece (each batch_elems elements; only a case's last
-// batch may be shorter) through this warp's ring, writing each batch's
-// mismatch count.  Warps claim batches from the block's counter as they
-// issue their copies (NST - 1 batches ahead of the check), so each warp's
-// batches are in ascending order and a warp slowed by exact steps takes
-// fewer.  Offsets within the piece are 32-bit (a piece holds at most
-// kMaxPiece elements).
+// Number of batches warp w takes in a piece of nb batches (the j with
+// j * kWarps + ((w - j) mod kWarps) < nb).
+__device__ __forceinline__ uint32_t warp_batches(uint32_t nb, int warp) {
+  const uint32_t J = nb / kWarps;
+  const uint32_t last = (uint32_t)(((warp - (int)(J % kWarps)) % kWarps + kWarps) % kWarps);
+  return J + (last < nb % kWarps ? 1u : 0u);
+}
+
+__device__ __forceinline__ void sse_flush(SseAcc &a) {
+  // TwoSum of the two slots' high parts, then two fp64 additions.
+  float h = a.hi.x, l = a.lo.x;
+  ff_add(h, l, a.hi.y, a.lo.y);
+  a.acc = __dadd_rn(a.acc, __dadd_rn((double)h, (double)l));
+  a.hi = a.lo = make_float2(0.f, 0.f);
+}
+
+// Sweep this warp's batches of a piece (each batch_elems elements; only a
+// case's last batch may be shorter) through its ring, NST - 1 batches of
+// copies ahead of the check, writing each batch's mismatch count.  Offsets
+// within the piece are 32-bit (a piece holds at most kMaxPiece elements).
 template <int DT, int NIN>
 __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
-                                      int32_t *batch_count, BatchSse *bsse, uint8_t *ring, uint64_t *bars,
-                                      RingPos &rp, uint32_t *err) {
+                                      int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
+                                      uint32_t *err) {
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
@@ -1124,27 +1121,24 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   const char *src_r = (const char *)P->cd.ref + pc.begin * EB;
   const char *src_x = NIN == 1 ? (const char *)P->cd.in_ptr[0] + pc.begin * EB : nullptr;
   int32_t *bcount = batch_count + pc.batch_base;
-  // lane 0: claim the next batch into stage st_i and issue its copies
-  uint32_t st_i = rp.stage;
-  bool claiming = true;  // chunks may remain
-  bool live = true;      // the end of the piece has not been marked yet
-  // Batches are claimed kChunk at a time (next_batch counts chunks); a
-  // warp issues a chunk's batches in order before it claims the next.
-  uint32_t i_next = 0, i_left = 0;
+  // lane 0: issue the copies of the warp's next batch into stage st_i.  The
+  // j-th batch of warp w is j * kWarps + ((w - j) mod kWarps): in round j
+  // the block's warps take batches j * kWarps .. j * kWarps + kWarps - 1, a
+  // warp's batches stay in ascending order, and a pattern that repeats every
+  // few batches (a faulty column band) spreads over all warps.  The schedule
+  // is fixed, so each lane's sums do not depend on timing.
+  const uint32_t nj = warp_batches(nb, warp);
+  uint32_t st_i = rp.stage, j_i = 0, rot_i = (uint32_t)warp;
+  bool live = true;  // the end of the piece has not been marked yet
   auto issue_next = [&]() {
-    if (i_left == 0 && claiming) {
-      const uint32_t c = atomicAdd(&P->next_batch, 1u);
-      i_next = c * kChunk;
-      i_left = i_next < nb ? (nb - i_next < kChunk ? nb - i_next : kChunk) : 0u;
-      if (i_left == 0) claiming = false;
-    }
-    if (i_left == 0) {
+    if (j_i >= nj) {
       W->stage_b[st_i] = kNoBatch;
       live = false;
       return;
     }
-    const uint32_t b = i_next++;
-    --i_left;
+    const uint32_t b = j_i * kWarps + rot_i;
+    rot_i = (rot_i + kWarps - 1) & (kWarps - 1);
+    ++j_i;
     W->stage_b[st_i] = b;
     const uint32_t off = b * BB;
     uint32_t bytes = 0;
@@ -1169,6 +1163,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   // latency hides and the hot word sees few readers).
   uint64_t gAR = ld_relaxed64(g_thr);
   const uint32_t lane_off = (uint32_t)lane * V;
+  int flush = 0;
   for (uint32_t j = 0;; ++j) {
     const uint32_t b = W->stage_b[rp.stage];
     if (b == kNoBatch) break;
@@ -1254,10 +1249,12 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
       R.track_r = R.track_r && !__any_sync(0xffffffffu, (R.racc & mag) != 0u);
     }
-    // the SSE of a chunk (kChunk batches, or the piece's rest) is stored at
-    // its first batch
-    if ((b + 1) % kChunk == 0 || b + 1 == nb) batch_sse_store(R.sse, bsse + pc.batch_base + (b - b % kChunk));
+    if (++flush == kFlushBatches) {
+      sse_flush(R.sse);
+      flush = 0;
+    }
   }
+  sse_flush(R.sse);
 }
 
 // ------------------------------------------------------------ the kernel
@@ -1271,8 +1268,7 @@ template <int DT, int NIN>
 __global__ void __launch_bounds__(kThreads, 2)
     scan_kernel(const CaseDesc *__restrict__ cases, const Piece *__restrict__ pieces,
                 unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base, Partial *partials,
-                int32_t *batch_count, BatchSse *bsse, uint8_t *out, uint32_t *g_thr, unsigned long long *stats,
-                uint32_t *err) {
+                int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
   constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
@@ -1308,7 +1304,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (threadIdx.x == 0) {
       P.cd = cases[pc.case_id];
       P.pbegin = pc.begin;
-      P.next_batch = 0;
       P.tr0 = pc.tr0;
       P.tc0 = pc.tc0;
       P.wr = pc.wr;
@@ -1368,7 +1363,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
-    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, bsse, ring, bars, rpos, err);
+    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
     __syncwarp();
     if (stats && lane == 0)
       for (int k = 0; k < 9; ++k)
@@ -1376,6 +1371,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 
     // ---- lanes -> warps -> the piece's partial
     const Best a = best_warp(abs_best64(L)), r = best_warp(rel_best64(L));
+    const double sse = warp_reduce(R.sse.acc, [](double x, double y) { return __dadd_rn(x, y); });
     const uint32_t cacc = warp_reduce(R.cacc | L->cacc, [](uint32_t x, uint32_t y) { return x | y; });
     const uint32_t racc = warp_reduce(R.racc | L->racc, [](uint32_t x, uint32_t y) { return x | y; });
     int eqs[NMV_MAX_INPUTS];
@@ -1397,7 +1393,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       w.arg_abs = a.i;
       w.best_rel = r.v;
       w.arg_rel = r.i;
-      w.sse = 0.0;
+      w.sse = sse;
       w.cacc = cacc;
       w.racc = racc;
 #pragma unroll
@@ -1419,19 +1415,6 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int64_t t = threadIdx.x; t < P.cd.tw; t += kThreads)
         if (P.sh_col[t]) atomicAdd(&P.g_col[t], (unsigned long long)P.sh_col[t]);
     }
-    {
-      // the piece's SSE: its chunks in order, thread t taking chunks t,
-      // t + kThreads, ..., then a fixed butterfly per warp and the warps in
-      // order
-      const int64_t nbp = piece_batches(pc.begin, pc.end, DT, NIN);
-      const BatchSse *bs = bsse + pc.batch_base;
-      double v = 0.0;
-      for (int64_t b = (int64_t)threadIdx.x * kChunk; b < nbp; b += (int64_t)kThreads * kChunk)
-        v = __dadd_rn(v, __dadd_rn(__dadd_rn((double)bs[b].hi, (double)bs[b].lo), bs[b].acc));
-      v = warp_reduce(v, [](double x, double y) { return __dadd_rn(x, y); });
-      if (lane == 0) red[warp].sse = v;
-    }
-    __syncthreads();
     if (threadIdx.x == 0) {
       Partial Q;
       Q.cnt[0] = 0;
@@ -1469,8 +1452,8 @@ struct ScanOps {
   static int occupancy(int nin, size_t smem);
   static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
                             const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
-                            Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out,
-                            uint32_t *g_thr, unsigned long long *stats, uint32_t *err);
+                            Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
+                            unsigned long long *stats, uint32_t *err);
 };
 
 #define NMV_SCAN_FN(DT, NIN) scan_kernel<DT, NIN>
@@ -1499,18 +1482,17 @@ struct ScanOps {
   cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases, \
                                   const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,  \
                                   int64_t piece_base,                                                     \
-                                  Partial *partials, int32_t *batch_count, BatchSse *bsse, uint8_t *out,  \
-                                  uint32_t *g_thr,                                                        \
+                                  Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr, \
                                   unsigned long long *stats, uint32_t *err) {                            \
     if (nin == 0)                                                                                        \
       NMV_SCAN_FN(DT, 0)<<<grid, kThreads, NMV_SCAN_SMEM(0, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     else if (nin == 1)                                                                                   \
       NMV_SCAN_FN(DT, 1)<<<grid, kThreads, NMV_SCAN_SMEM(1, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     else                                                                                                 \
       NMV_SCAN_FN(DT, -1)<<<grid, kThreads, NMV_SCAN_SMEM(-1, smem), st>>>(                              \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, bsse, out, g_thr, stats, err);        \
+          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
     return cudaGetLastError();                                                                           \
   }
 
