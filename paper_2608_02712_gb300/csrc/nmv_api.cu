@@ -30,6 +30,7 @@ struct ScanOps {
 cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
                             int, cudaStream_t);
 cudaError_t launch_sse64(const CaseDesc *cd, double *part, double *dst, cudaStream_t st);
+
 constexpr int kSseBlocksHost = 1024;  // scratch doubles of launch_sse64
 
 cudaError_t scan_prepare(int dt, int nin, size_t smem) {

@@ -310,7 +310,12 @@ __device__ __forceinline__ float rel32(float as, float ar) {
 }
 
 // A strict fp32 lower bound of n / d (n >= 0, d > 0): rel32 is within 2^-22.
-__device__ __forceinline__ float quot_lb(float n, float d) { return __fmul_rz(rel32(n, d), 1.0f - 0x1p-21f); }
+// A quotient beyond the fp32 range (d subnormal, say) gives the largest
+// finite float, still a lower bound; an infinite bound would make every
+// warp skip the larger quotients it cannot tell apart.
+__device__ __forceinline__ float quot_lb(float n, float d) {
+  return __fmul_rz(fminf(rel32(n, d), 0x1.fffffep127f), 1.0f - 0x1p-21f);
+}
 
 // fp32 lower bounds of a lane's maxima (-1 when none held).
 __device__ __forceinline__ float abs_lb(const LaneSh *L) {
@@ -1257,6 +1262,29 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   sse_flush(R.sse);
 }
 
+// ------------------------------------------------------------ seeding
+// Lower bounds of |d| and |d|/|r| of element i (fp32 values rounded down
+// from its fp64 error; nothing for a non-finite pair), folded into ma, mr.
+template <int DT>
+__device__ __forceinline__ void seed_elem(const CaseDesc &cd, int64_t i, float &ma, float &mr) {
+  constexpr int EB = Tr<DT>::EB;
+  const uint32_t cb = ld_one<EB>(cd.cand, i), rb = ld_one<EB>(cd.ref, i);
+  float as, ar;
+  if constexpr (Tr<DT>::kInt) {
+    const long long d = (long long)(int32_t)cb - (long long)(int32_t)rb;
+    as = __ll2float_rd(d < 0 ? -d : d);
+    const long long r = (long long)(int32_t)rb;
+    ar = __ll2float_ru(r < 0 ? -r : r);
+  } else {
+    const float c = to_f32<DT>(cb), r = to_f32<DT>(rb);
+    if (!(isfinite(c) && isfinite(r))) return;
+    as = __fsub_rd(fmaxf(c, r), fminf(c, r));  // <= |c - r|
+    ar = fabsf(r);
+  }
+  ma = fmaxf(ma, as);
+  if (ar > 0.f) mr = fmaxf(mr, quot_lb(as, ar));
+}
+
 // ------------------------------------------------------------ the kernel
 // Dynamic shared memory: the warps' rings (ring_bytes(NIN): stage data, then
 // one mbarrier per stage), then int32 words: [0, 8) class counters
@@ -1291,6 +1319,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   }
   __syncwarp();
   RingPos rpos = {0u, 0u};
+  bool tr_first = true;  // the block's first piece seeds the published maxima
   // Blocks take pieces from the launch's counter as they finish the last
   // one, so pieces of uneven cost (a region wrong everywhere next to a clean
   // one) balance over the blocks.
@@ -1327,6 +1356,35 @@ __global__ void __launch_bounds__(kThreads, 2)
       P.stats = stats;
     }
     __syncthreads();
+    if (tr_first) {
+      // A sample of the case (two elements per thread of every block,
+      // spread over the whole case) seeds the published maxima, so warps
+      // start near the final thresholds instead of establishing them one
+      // light step at a time.  Every value is a lower bound of an actual
+      // element's error, published like the scan's own.
+      constexpr int kSamples = 2;
+      const int64_t total = (int64_t)gridDim.x * kThreads * kSamples;
+      const int64_t stride = P.cd.numel > total ? P.cd.numel / total : 1;
+      float ma = -1.f, mr = -1.f;
+#pragma unroll
+      for (int s2 = 0; s2 < kSamples; ++s2) {
+        const int64_t i = (((int64_t)blockIdx.x * kThreads + threadIdx.x) * kSamples + s2) * stride;
+        if (i < P.cd.numel) seed_elem<DT>(P.cd, i, ma, mr);
+      }
+      ma = warp_reduce(ma, [](float x, float y) { return fmaxf(x, y); });
+      mr = warp_reduce(mr, [](float x, float y) { return fmaxf(x, y); });
+      if (lane == 0) {
+        if (ma > 0.f) {
+          atomicMax(&cta_thr[0], __float_as_uint(ma));
+          atomicMax(&P.g_thr[0], __float_as_uint(ma));
+        }
+        if (mr > 0.f) {
+          atomicMax(&cta_thr[1], __float_as_uint(mr));
+          atomicMax(&P.g_thr[1], __float_as_uint(mr));
+        }
+      }
+      tr_first = false;
+    }
     const int64_t used = (int64_t)(P.sh_hist - smem) + (int64_t)pc.wr * pc.wc;
     for (int64_t t = threadIdx.x; t < used; t += kThreads) smem[t] = 0;
     L->a_i = L->r_i = INT64_MAX;
