@@ -215,3 +215,19 @@ def test_results_stay_valid_until_freed():
     assert_same(m.result_to_dict(outs[0][0]), d[0], "live result after reuse")
     for o in (outs[0], outs[2], out):
         lib.nmv_result_free(o)
+
+
+def test_relative_errors_beyond_fp32_range():
+    # |d| / |r| above the fp32 range (a subnormal reference): the thresholds
+    # the warps share must stay finite lower bounds, or the larger of two such
+    # quotients in different pieces would be skipped.
+    g = torch.Generator().manual_seed(9)
+    ref = torch.randn(4, 1 << 20, generator=g)
+    cand = ref.clone()
+    flat_r, flat_c = ref.view(-1), cand.view(-1)
+    flat_r[1000], flat_c[1000] = 1e-42, 1.0
+    flat_r[3_000_000], flat_c[3_000_000] = 1e-43, 4.0
+    want = oracle.validate(cand, ref, rtol=1e-5, atol=1e-6, tile=(1, 4096), first_k=8)
+    got = validate(cand.cuda(), ref.cuda(), rtol=1e-5, atol=1e-6, tile=(1, 4096), first_k=8)
+    assert_same(got, want, "rel beyond fp32")
+    assert got["argmax_rel"] == 3_000_000 and got["max_rel"] > 3.4e38
