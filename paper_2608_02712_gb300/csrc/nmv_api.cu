@@ -28,7 +28,7 @@ struct ScanOps {
                             unsigned long long *stats, uint32_t *err);
 };
 cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
-                            int, cudaStream_t);
+                            int, int, cudaStream_t);
 cudaError_t launch_sse64(const CaseDesc *cd, double *part, double *dst, cudaStream_t st);
 
 constexpr int kSseBlocksHost = 1024;  // scratch doubles of launch_sse64
@@ -459,6 +459,7 @@ struct PlanCache {
   std::vector<CaseDesc> desc;
   std::vector<Piece> pieces;
   int64_t np = 0, n_batches = 0;
+  int fin_helpers = 0;          // most finalize helper blocks of any case
   size_t out_size = 0;
   void *uploaded_ws = nullptr;  // workspace holding this plan's descriptors
 };
@@ -587,6 +588,12 @@ int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo
   }
   C.np = np;
   C.n_batches = n_batches;
+  C.fin_helpers = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    const CaseDesc &d = C.desc[i];
+    const int h = fin_helpers(d.first_k, d.batch_end - d.batch_begin);
+    if (h > C.fin_helpers) C.fin_helpers = h;
+  }
   C.out_size = out_size;
   C.uploaded_ws = nullptr;
   C.valid = true;
@@ -768,7 +775,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   }
   if (prof) cudaEventRecord(g_prof.ev[1], st);
   e = launch_finalize(d_cases, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc),
-                      W + o_out, (int)n, st);
+                      W + o_out, (int)n, C.fin_helpers, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   if (prof) cudaEventRecord(g_prof.ev[2], st);
   e = cudaMemcpyAsync(HO, W + o_out, out_size, cudaMemcpyDeviceToHost, st);
@@ -1030,7 +1037,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   e = launch_finalize(d_case, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc), W + o_out,
-                      1, st);
+                      1, fin_helpers(g_na_desc.first_k, g_na_desc.batch_end - g_na_desc.batch_begin), st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   const uint8_t *ob = W + o_out + kCallHeader;
   uint32_t kerr = 0;

@@ -116,16 +116,29 @@ struct OutHeader {
 // Warp steps (32 lanes x 16 bytes of each tensor) per batch, by input class
 // (0, 1 or -1 = several inputs read from global memory; one staged input
 // leaves shared memory for shorter batches only), and elements per batch.  A
-// batch is the unit of the first-K counts and of the warps' shared-memory
-// rings.
-constexpr int kMaxSteps = 4;
-NMV_CHD int batch_steps(int nin) { return nin == 1 ? 2 : 4; }
-NMV_CHD int batch_bytes(int nin) { return 32 * 16 * batch_steps(nin); }  // one tensor's bytes
+// batch is the unit of the first-K counts and of the scan's bookkeeping; it
+// streams through a warp's shared-memory ring as two stages of half a batch.
+constexpr int kMaxSteps = 8;
+NMV_CHD int batch_steps(int nin) { return nin == 1 ? 4 : 8; }
+NMV_CHD int stage_steps(int nin) { return batch_steps(nin) / 2; }
+NMV_CHD int stage_bytes(int nin) { return 32 * 16 * stage_steps(nin); }  // one tensor's bytes per stage
 NMV_CHD int nin_class_of(int n_elig) { return n_elig == 0 ? 0 : (n_elig == 1 ? 1 : -1); }
 NMV_HD int64_t batch_elems(int dt, int nin) { return (int64_t)32 * vec_elems(dt) * batch_steps(nin); }
 NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt, int nin) {
   const int64_t be = batch_elems(dt, nin);
   return (end - begin + be - 1) / be;
+}
+
+// Finalize blocks of one case beyond the first: a case with records to write
+// and at least kFinHelperBatches batches gets one helper block per that many
+// batches (at most kFinMaxHelpers); the helpers then write the records while
+// the first block reduces the partials.
+constexpr int kFinMaxHelpers = 16;
+constexpr int64_t kFinHelperBatches = 4096;
+NMV_HD int fin_helpers(int64_t first_k, int64_t n_batches) {
+  if (first_k <= 0 || n_batches < kFinHelperBatches) return 0;
+  const int64_t h = n_batches / kFinHelperBatches;
+  return h < kFinMaxHelpers ? (int)h : kFinMaxHelpers;
 }
 
 // Ring of each scan warp, by input class: stages, tensors staged per batch,
@@ -134,7 +147,7 @@ NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt, int nin) {
 NMV_CHD int ring_stages(int) { return 2; }
 NMV_CHD int ring_streams(int nin) { return nin == 1 ? 3 : 2; }
 NMV_CHD size_t ring_bytes(int nin) {
-  return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * batch_bytes(nin) + 8);
+  return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * stage_bytes(nin) + 8);
 }
 
 }  // namespace nmv

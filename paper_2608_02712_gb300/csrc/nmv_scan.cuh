@@ -1054,8 +1054,8 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   reload_thr(R, W);
 }
 
-// Issue the copies of one batch, at byte offset `off` of the piece and with
-// `bytes` (whole steps only) per tensor, into a ring stage (lane 0 only).  A
+// Issue the copies of one stage (half a batch), at byte offset `off` of the
+// piece and with `bytes` (whole steps only) per tensor (lane 0 only).  A
 // ragged rest and the buffers of a case that is not 16-byte aligned
 // (bytes = 0) are read from global memory by tail_step.
 template <int NIN>
@@ -1065,8 +1065,8 @@ __device__ __forceinline__ void ring_issue(const char *c, const char *r, const c
   if (bytes) {
     const uint64_t pol = evict_first_policy();
     bulk_load(stage, c + off, bytes, bar, pol);
-    bulk_load(stage + batch_bytes(NIN), r + off, bytes, bar, pol);
-    if constexpr (NIN == 1) bulk_load(stage + 2 * batch_bytes(NIN), x + off, bytes, bar, pol);
+    bulk_load(stage + stage_bytes(NIN), r + off, bytes, bar, pol);
+    if constexpr (NIN == 1) bulk_load(stage + 2 * stage_bytes(NIN), x + off, bytes, bar, pol);
   }
 }
 
@@ -1079,7 +1079,7 @@ struct RingPos {
 constexpr uint32_t kNoBatch = 0xffffffffu;
 // The SSE's float-float pairs go to fp64 every kFlushBatches batches of a
 // lane (at most 128 terms per pair in between).
-constexpr int kFlushBatches = 4;
+constexpr int kFlushBatches = 2;
 
 // Number of batches warp w takes in a piece of nb batches (the j with
 // j * kWarps + ((w - j) mod kWarps) < nb).
@@ -1098,9 +1098,10 @@ __device__ __forceinline__ void sse_flush(SseAcc &a) {
 }
 
 // Sweep this warp's batches of a piece (each batch_elems elements; only a
-// case's last batch may be shorter) through its ring, NST - 1 batches of
-// copies ahead of the check, writing each batch's mismatch count.  Offsets
-// within the piece are 32-bit (a piece holds at most kMaxPiece elements).
+// case's last batch may be shorter) through its ring, one stage (half a
+// batch) of copies ahead of the check, writing each batch's mismatch count.
+// Offsets within the piece are 32-bit (a piece holds at most kMaxPiece
+// elements).
 template <int DT, int NIN>
 __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
                                       int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
@@ -1109,31 +1110,31 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
   constexpr int KS = batch_steps(NIN);
+  constexpr int HS = stage_steps(NIN);
   constexpr int BATCH = STEP * KS;
-  constexpr uint32_t BB = BATCH * EB;  // bytes of one tensor's batch (batch_bytes)
+  constexpr uint32_t BB = BATCH * EB;          // bytes of one tensor's batch
+  constexpr uint32_t HB = stage_bytes(NIN);    // bytes of one tensor's stage (half a batch)
   constexpr uint32_t NST = ring_stages(NIN);
-  constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
+  constexpr int STAGE = ring_streams(NIN) * stage_bytes(NIN);
   constexpr int kPoll = kWarps;  // batches between a warp's readings of the case-wide maxima
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t *g_thr = P->g_thr;
   const uint32_t nb = (uint32_t)((pc.end - pc.begin + BATCH - 1) / BATCH);
   const uint32_t mag = Tr<DT>::kInt ? 0xffffffffu : (Tr<DT>::EB == 2 ? 0x7fff7fffu : 0x7fffffffu);
   const uint32_t pbytes = (uint32_t)((pc.end - pc.begin) * EB);
-  // batches at byte offsets <= full_max are whole and staged (all batches
-  // but a case's last; none when the case is not 16-byte aligned)
-  const int64_t full_max = P->cd.vec_ok ? (int64_t)pbytes - BB : -1;
+  const bool vec_ok = P->cd.vec_ok != 0;
   const char *src_c = (const char *)P->cd.cand + pc.begin * EB;
   const char *src_r = (const char *)P->cd.ref + pc.begin * EB;
   const char *src_x = NIN == 1 ? (const char *)P->cd.in_ptr[0] + pc.begin * EB : nullptr;
   int32_t *bcount = batch_count + pc.batch_base;
-  // lane 0: issue the copies of the warp's next batch into stage st_i.  The
-  // j-th batch of warp w is j * kWarps + ((w - j) mod kWarps): in round j
+  // lane 0: issue the copies of the warp's next stage into ring stage st_i.
+  // The j-th batch of warp w is j * kWarps + ((w - j) mod kWarps): in round j
   // the block's warps take batches j * kWarps .. j * kWarps + kWarps - 1, a
   // warp's batches stay in ascending order, and a pattern that repeats every
   // few batches (a faulty column band) spreads over all warps.  The schedule
   // is fixed, so each lane's sums do not depend on timing.
   const uint32_t nj = warp_batches(nb, warp);
-  uint32_t st_i = rp.stage, j_i = 0, rot_i = (uint32_t)warp;
+  uint32_t st_i = rp.stage, j_i = 0, h_i = 0, rot_i = (uint32_t)warp;
   bool live = true;  // the end of the piece has not been marked yet
   auto issue_next = [&]() {
     if (j_i >= nj) {
@@ -1142,19 +1143,20 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       return;
     }
     const uint32_t b = j_i * kWarps + rot_i;
-    rot_i = (rot_i + kWarps - 1) & (kWarps - 1);
-    ++j_i;
     W->stage_b[st_i] = b;
-    const uint32_t off = b * BB;
+    const uint32_t off = b * BB + h_i * HB;
     uint32_t bytes = 0;
-    if ((int64_t)off <= full_max) {
-      bytes = BB;
-    } else if (P->cd.vec_ok && off < pbytes) {
-      bytes = (pbytes - off) / (STEP * EB) * (STEP * EB);
-    }
+    if (vec_ok && off < pbytes) bytes = pbytes - off >= HB ? HB : (pbytes - off) / (STEP * EB) * (STEP * EB);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i);
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
+    if (h_i == 0) {
+      h_i = 1;
+    } else {
+      h_i = 0;
+      ++j_i;
+      rot_i = (rot_i + kWarps - 1) & (kWarps - 1);
+    }
   };
   if (lane == 0) {
     for (uint32_t i = 0; i < NST - 1 && live; ++i) issue_next();
@@ -1173,12 +1175,8 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     const uint32_t b = W->stage_b[rp.stage];
     if (b == kNoBatch) break;
     const uint32_t erel = b * BATCH;  // element offset of the batch in the piece
-    const uint32_t off = b * BB;
     __syncwarp();
-    if (lane == 0) {
-      if (live) issue_next();  // refills the stage released last batch
-      W->mism = 0;
-    }
+    if (lane == 0) W->mism = 0;
     if ((j + warp) % kPoll == 0) {
       if (lane == 0) {
         atomicMax(&P->cta_thr[0], (uint32_t)gAR);
@@ -1205,47 +1203,53 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
         reload_thr(R, W);
       }
     }
-    __syncwarp();
-    const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
-    if (!dead && !mbar_try_wait(bars + rp.stage, rp.phase)) {
-      if (!mbar_wait_slow(bars + rp.stage, rp.phase)) {
-        dead = true;  // report, and stop waiting (the data of this call is void)
-        if (lane == 0) atomicOr(err, 1u);
-      }
-    }
-    if (++rp.stage == NST) {
-      rp.stage = 0;
-      rp.phase ^= 1u;
-    }
-    if ((int64_t)off <= full_max) {
-#pragma unroll 2
-      for (int u = 0; u < KS; ++u) {
-        const uint4 cv = lds_v4(stage + u * 512);
-        const uint4 rv = lds_v4(stage + BB + u * 512);
-        uint4 xv = make_uint4(0, 0, 0, 0);
-        if constexpr (NIN == 1) xv = lds_v4(stage + 2 * BB + u * 512);
-        step<DT, NIN>(P, L, W, R, cv, rv, xv, erel + u * STEP + lane_off);
-      }
-    } else {
-      // the case's last batch, or a case that is not 16-byte aligned
-      const uint32_t pel = pbytes / EB;  // elements in the piece
-      const uint32_t nfull = P->cd.vec_ok ? (pel - erel) / STEP : 0u;
-      for (int u = 0; u < KS; ++u) {
-        const uint32_t e = erel + u * STEP + lane_off;
-        if ((uint32_t)u < nfull) {
-          const uint4 cv = lds_v4(stage + u * 512);
-          const uint4 rv = lds_v4(stage + BB + u * 512);
-          uint4 xv = make_uint4(0, 0, 0, 0);
-          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * BB + u * 512);
-          step<DT, NIN>(P, L, W, R, cv, rv, xv, e);
-        } else if (erel + u * STEP < pel) {
-          const int n = e >= pel ? 0 : (pel - e > (uint32_t)V ? V : (int)(pel - e));
-          R.sse = tail_step<DT, NIN>(P, L, W, P->pbegin + e, n, R.sse);
-          reload_thr(R, W);
+#pragma unroll 1
+    for (int h = 0; h < 2; ++h) {
+      if (lane == 0 && live) issue_next();  // refills the stage released before this one
+      __syncwarp();
+      const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
+      if (!dead && !mbar_try_wait(bars + rp.stage, rp.phase)) {
+        if (!mbar_wait_slow(bars + rp.stage, rp.phase)) {
+          dead = true;  // report, and stop waiting (the data of this call is void)
+          if (lane == 0) atomicOr(err, 1u);
         }
       }
+      if (++rp.stage == NST) {
+        rp.stage = 0;
+        rp.phase ^= 1u;
+      }
+      const uint32_t hoff = b * BB + h * HB;
+      const uint32_t hrel = erel + h * (HS * STEP);
+      if (vec_ok && hoff < pbytes && pbytes - hoff >= HB) {
+#pragma unroll 2
+        for (int u = 0; u < HS; ++u) {
+          const uint4 cv = lds_v4(stage + u * 512);
+          const uint4 rv = lds_v4(stage + HB + u * 512);
+          uint4 xv = make_uint4(0, 0, 0, 0);
+          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+          step<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+        }
+      } else {
+        // part of the case's last batch, or a case that is not 16-byte aligned
+        const uint32_t pel = pbytes / EB;  // elements in the piece
+        const uint32_t nfull = vec_ok && hrel < pel ? (pel - hrel) / STEP : 0u;
+        for (int u = 0; u < HS; ++u) {
+          const uint32_t e = hrel + u * STEP + lane_off;
+          if ((uint32_t)u < nfull) {
+            const uint4 cv = lds_v4(stage + u * 512);
+            const uint4 rv = lds_v4(stage + HB + u * 512);
+            uint4 xv = make_uint4(0, 0, 0, 0);
+            if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+            step<DT, NIN>(P, L, W, R, cv, rv, xv, e);
+          } else if (hrel + u * STEP < pel) {
+            const int n = e >= pel ? 0 : (pel - e > (uint32_t)V ? V : (int)(pel - e));
+            R.sse = tail_step<DT, NIN>(P, L, W, P->pbegin + e, n, R.sse);
+            reload_thr(R, W);
+          }
+        }
+      }
+      __syncwarp();  // every lane is done with the stage before it is refilled
     }
-    __syncwarp();  // every lane is done with the stage before it is refilled
     if (lane == 0) {
       bcount[b] = (int32_t)W->mism;
       W->mism_tot += W->mism;
@@ -1299,7 +1303,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 int32_t *batch_count, uint8_t *out, uint32_t *g_thr, unsigned long long *stats, uint32_t *err) {
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
-  constexpr int STAGE = ring_streams(NIN) * batch_bytes(NIN);
+  constexpr int STAGE = ring_streams(NIN) * stage_bytes(NIN);
   extern __shared__ __align__(128) uint8_t dsm[];
   __shared__ PieceSh P;
   __shared__ LaneSh lanes[kThreads];
