@@ -811,28 +811,60 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
   return sse;
 }
 
-// A step of finite elements whose predicate the fp32 bounds decide and none
-// of which can be a new maximum (|s| <= tA and |s| <= tR |r|, tR uncapped):
-// the dense-mismatch case (an output that is wrong almost everywhere).
-// Only the mismatch count, the localisation maps and the SSE remain; the
-// SSE terms take the exact path's arithmetic (c - r as s + e by TwoSum), so
-// the result does not depend on which path an element took.  Float types.
+// A float step that needs more than a maximum update: one classification
+// pass over the lane's elements decides for the warp between
+//  * dense: every element finite, its predicate decided by the fp32 bounds
+//    and no candidate for a maximum (|s| <= tA and |s| <= tR |r|, tR
+//    uncapped): only the mismatch count, the maps and the SSE remain, done
+//    here; the SSE terms take the exact path's arithmetic (c - r as s + e by
+//    TwoSum, d^2 = p + pe + 2se), so the result does not depend on which path
+//    an element took;
+//  * otherwise the exact step.
 template <int DT>
-__device__ __noinline__ SseAcc dense_step(const PieceSh *P, WarpSh *W, uint4 cv, uint4 rv, int64_t idx0,
-                                          SseAcc sse) {
+__device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W, uint4 cv, uint4 rv,
+                                         int64_t idx0, SseAcc sse) {
   constexpr int V = Tr<DT>::V;
   const long long t_start = P->stats ? clock64() : 0;
-  const float lo_r = P->cd.lo_r, lo_a = P->cd.lo_a;
+  const float2 m1 = make_float2(-1.f, -1.f);
+  const float2 lo_r2 = make_float2(P->cd.lo_r, P->cd.lo_r), lo_a2 = make_float2(P->cd.lo_a, P->cd.lo_a);
+  const float2 hi_r2 = make_float2(P->cd.hi_r, P->cd.hi_r), hi_a2 = make_float2(P->cd.hi_a, P->cd.hi_a);
+  const float tA = W->tA, tR = W->tR;
+  const float2 tR2 = make_float2(tR, tR);
+  float2 s[V / 2], e[V / 2];
+  bool dense = true;
   uint32_t mask = 0;
 #pragma unroll
-  for (int k = 0; k < V; ++k) {
-    const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
-    const float sk = __fsub_rn(cf, rf);
-    const float bb = __fsub_rn(sk, cf);
-    const float ek = __fsub_rn(__fsub_rn(cf, __fsub_rn(sk, bb)), __fadd_rn(rf, bb));  // TwoSum(c, -r)
-    if (!(fabsf(sk) <= __fmaf_rz(lo_r, fabsf(rf), lo_a))) mask |= 1u << k;
-    if (k & 1) ff_term(sse.hi.y, sse.lo.y, sk, ek);
-    else ff_term(sse.hi.x, sse.lo.x, sk, ek);
+  for (int j = 0; j < V / 2; ++j) {
+    const float2 c2 = make_float2(vdec<DT>(cv, 2 * j), vdec<DT>(cv, 2 * j + 1));
+    const float2 r2 = make_float2(vdec<DT>(rv, 2 * j), vdec<DT>(rv, 2 * j + 1));
+    // TwoSum(c, -r): s + e = c - r exactly when both are finite
+    const float2 s2 = __ffma2_rn(r2, m1, c2);
+    const float2 bb = __ffma2_rn(c2, m1, s2);
+    const float2 y = __ffma2_rn(__ffma2_rn(bb, m1, s2), m1, c2);
+    s[j] = s2;
+    e[j] = __ffma2_rn(__fadd2_rn(r2, bb), m1, y);
+    const float2 ar2 = make_float2(fabsf(r2.x), fabsf(r2.y));
+    const float2 a2 = __ffma2_rz(ar2, lo_r2, lo_a2);
+    const float2 h2 = __ffma2_ru(ar2, hi_r2, hi_a2);
+    const float2 t2 = __fmul2_rz(ar2, tR2);
+    const float as0 = fabsf(s2.x), as1 = fabsf(s2.y);
+    dense &= (as0 <= a2.x || as0 > h2.x) && as0 <= tA && as0 <= t2.x;
+    dense &= (as1 <= a2.y || as1 > h2.y) && as1 <= tA && as1 <= t2.y;
+    if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
+    if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
+  }
+  if (!__all_sync(0xffffffffu, dense)) return slow_step<DT>(P, L, W, cv, rv, idx0, V, sse);
+#pragma unroll
+  for (int j = 0; j < V / 2; ++j) {
+    const float2 p = __fmul2_rn(s[j], s[j]);
+    const float2 pe = __ffma2_rn(s[j], s[j], __fmul2_rn(p, m1));
+    const float2 q = __ffma2_rn(__fadd2_rn(s[j], s[j]), e[j], pe);
+    const float2 t = __fadd2_rn(sse.hi, p);
+    const float2 bp = __ffma2_rn(sse.hi, m1, t);
+    const float2 x2 = __ffma2_rn(__ffma2_rn(bp, m1, t), m1, sse.hi);
+    const float2 err = __fadd2_rn(x2, __ffma2_rn(bp, m1, p));
+    sse.lo = __fadd2_rn(sse.lo, __fadd2_rn(err, q));
+    sse.hi = t;
   }
   if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0, V);
   if (P->stats) count_stats(W, 2, t_start, 0, 0, 0);
@@ -1011,19 +1043,27 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
       const float2 s2 = __ffma2_rn(r2, m1, c2);  // fl(c - r), one rounding
       s[k] = s2.x;
       s[k + 1] = s2.y;
-      const float a0 = __fmaf_rz(R.lo_r, fabsf(r2.x), R.lo_a), a1 = __fmaf_rz(R.lo_r, fabsf(r2.y), R.lo_a);
-      const float b0 = __fmul_rz(R.tRq, fabsf(r2.x)), b1 = __fmul_rz(R.tRq, fabsf(r2.y));
-      hard |= !(fabsf(s2.x) <= min3f(a0, b0, R.tA));
-      hard |= !(fabsf(s2.y) <= min3f(a1, b1, R.tA));
+      const float2 ar2 = make_float2(fabsf(r2.x), fabsf(r2.y));
+      float2 a2, b2;
+      if constexpr (Tr<DT>::EB == 2) {
+        // the bounds in packed form (the same roundings as the scalar ones)
+        a2 = __ffma2_rz(ar2, make_float2(R.lo_r, R.lo_r), make_float2(R.lo_a, R.lo_a));
+        b2 = __fmul2_rz(ar2, make_float2(R.tRq, R.tRq));
+      } else {
+        a2 = make_float2(__fmaf_rz(R.lo_r, ar2.x, R.lo_a), __fmaf_rz(R.lo_r, ar2.y, R.lo_a));
+        b2 = make_float2(__fmul_rz(R.tRq, ar2.x), __fmul_rz(R.tRq, ar2.y));
+      }
+      hard |= !(fabsf(s2.x) <= min3f(a2.x, b2.x, R.tA));
+      hard |= !(fabsf(s2.y) <= min3f(a2.y, b2.y, R.tA));
     }
     if (!__any_sync(0xffffffffu, hard)) {
 #pragma unroll
       for (int k = 0; k < V; k += 2) ff_pair<Tr<DT>::EB == 4>(R.sse, make_float2(s[k], s[k + 1]));
       return;
     }
-    // Which steps need the exact path (a mismatch, a non-finite value, an
-    // inexact c - r, an undecided predicate) and which only a maximum update
-    // (the finite cap keeps infinities out of the light path).
+    // Which steps need more than a maximum update (a mismatch, a non-finite
+    // value, an inexact c - r, an undecided predicate; the finite cap keeps
+    // infinities out of the light path).
     other = false;
 #pragma unroll
     for (int k = 0; k < V; ++k) {
@@ -1033,21 +1073,8 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
     }
   }
   if (__any_sync(0xffffffffu, other)) {
-    bool dense = false;
-    if constexpr (!Tr<DT>::kInt) {
-      // every element finite, decided by the fp32 bounds, and no candidate
-      // for a maximum (|s| <= tA also rules out NaN and infinities)
-      dense = true;
-#pragma unroll
-      for (int k = 0; k < V; ++k) {
-        const float cf = vdec<DT>(cv, k), rf = vdec<DT>(rv, k);
-        const float as = fabsf(__fsub_rn(cf, rf)), ar = fabsf(rf);
-        const bool decided = as <= __fmaf_rz(R.lo_r, ar, R.lo_a) || as > __fmaf_ru(P->cd.hi_r, ar, P->cd.hi_a);
-        dense &= decided && as <= R.tA && as <= __fmul_rz(R.tR, ar);
-      }
-    }
-    if (__all_sync(0xffffffffu, dense)) R.sse = dense_step<DT>(P, W, cv, rv, P->pbegin + erel, R.sse);
-    else R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
+    if constexpr (Tr<DT>::kInt) R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
+    else R.sse = hard_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
   } else {
     R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
   }
