@@ -101,6 +101,31 @@ __device__ __forceinline__ float min3f(float a, float b, float c) {
   return r;
 }
 
+// Atomic updates whose result is not used, with the state space explicit:
+// the localisation maps and class counters sit in shared memory behind
+// pointers kept in PieceSh, which a plain atomicAdd would reach through a
+// generic (slow) atomic.  No memory clobber: these words are read only
+// after a block barrier, and the reductions may be reordered among
+// themselves.
+__device__ __forceinline__ void sh_add_at(uint32_t addr, int v) {
+  asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(addr), "r"(v));
+}
+__device__ __forceinline__ void sh_add(int32_t *p, int v) { sh_add_at((uint32_t)__cvta_generic_to_shared(p), v); }
+__device__ __forceinline__ void gl_add(unsigned long long *p, unsigned long long v) {
+  asm volatile("red.global.add.u64 [%0], %1;" ::"l"(p), "l"(v));
+}
+__device__ __forceinline__ void sh_max(uint32_t *p, uint32_t v) {
+  asm volatile("red.shared.max.u32 [%0], %1;" ::"r"((uint32_t)__cvta_generic_to_shared(p)), "r"(v));
+}
+__device__ __forceinline__ uint32_t sh_max_old(uint32_t *p, uint32_t v) {
+  uint32_t old;
+  asm volatile("atom.shared.max.u32 %0, [%1], %2;"
+               : "=r"(old)
+               : "r"((uint32_t)__cvta_generic_to_shared(p)), "r"(v)
+               : "memory");
+  return old;
+}
+
 // ---------------------------------------------------------- dtype traits
 template <int DT>
 struct Tr {
@@ -470,15 +495,18 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
   const uint64_t rp_l = __shfl_sync(0xffffffffu, rp, lead);
   if (__all_sync(0xffffffffu, mask == 0 || (single && hbin == hb_l && rp == rp_l))) {
     if (lane == lead) {
-      if (P->wr > 0) atomicAdd(&P->sh_hist[hbin], total);
-      else atomicAdd(&P->g_hist[hbin], (unsigned long long)total);
-      if (P->prof_smem) atomicAdd(&P->sh_row[rp], total);
-      else atomicAdd(&P->g_row[rp], (unsigned long long)total);
+      if (P->wr > 0) sh_add(&P->sh_hist[hbin], total);
+      else gl_add(&P->g_hist[hbin], (unsigned long long)total);
+      if (P->prof_smem) sh_add(&P->sh_row[rp], total);
+      else gl_add(&P->g_row[rp], (unsigned long long)total);
     }
-    for (uint32_t m = mask; m; m &= m - 1) {
-      const int k = __ffs(m) - 1;
-      if (P->prof_smem) atomicAdd(&P->sh_col[cp + k], 1);
-      else atomicAdd(&P->g_col[cp + k], 1ull);
+    if (P->prof_smem) {
+      const uint32_t base = (uint32_t)__cvta_generic_to_shared(P->sh_col + cp);
+#pragma unroll
+      for (int k = 0; k < 8; ++k)
+        if (k < V && ((mask >> k) & 1u)) sh_add_at(base + 4 * k, 1);
+    } else {
+      for (uint32_t m = mask; m; m &= m - 1) gl_add(&P->g_col[cp + __ffs(m) - 1], 1ull);
     }
     return;
   }
@@ -519,8 +547,8 @@ static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask,
                                  : (int64_t)(tr * (uint64_t)cd.GC + tc);
     if (hb != hb_cur) {
       if (hcnt) {
-        if (P->wr > 0) atomicAdd(&P->sh_hist[hb_cur], hcnt);
-        else atomicAdd(&P->g_hist[hb_cur], (unsigned long long)hcnt);
+        if (P->wr > 0) sh_add(&P->sh_hist[hb_cur], hcnt);
+        else gl_add(&P->g_hist[hb_cur], (unsigned long long)hcnt);
       }
       hb_cur = hb;
       hcnt = 0;
@@ -528,20 +556,20 @@ static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask,
     ++hcnt;
     if ((int64_t)rp != rbin) {
       if (rcnt) {
-        if (P->prof_smem) atomicAdd(&P->sh_row[rbin], rcnt);
-        else atomicAdd(&P->g_row[rbin], (unsigned long long)rcnt);
+        if (P->prof_smem) sh_add(&P->sh_row[rbin], rcnt);
+        else gl_add(&P->g_row[rbin], (unsigned long long)rcnt);
       }
       rbin = (int64_t)rp;
       rcnt = 0;
     }
     ++rcnt;
-    if (P->prof_smem) atomicAdd(&P->sh_col[cp], 1);
-    else atomicAdd(&P->g_col[cp], 1ull);
+    if (P->prof_smem) sh_add(&P->sh_col[cp], 1);
+    else gl_add(&P->g_col[cp], 1ull);
   }
-  if (P->wr > 0) atomicAdd(&P->sh_hist[hb_cur], hcnt);
-  else atomicAdd(&P->g_hist[hb_cur], (unsigned long long)hcnt);
-  if (P->prof_smem) atomicAdd(&P->sh_row[rbin], rcnt);
-  else atomicAdd(&P->g_row[rbin], (unsigned long long)rcnt);
+  if (P->wr > 0) sh_add(&P->sh_hist[hb_cur], hcnt);
+  else gl_add(&P->g_hist[hb_cur], (unsigned long long)hcnt);
+  if (P->prof_smem) sh_add(&P->sh_row[rbin], rcnt);
+  else gl_add(&P->g_row[rbin], (unsigned long long)rcnt);
 }
 
 // After a step in which some lane's maximum changed: the warp's own
@@ -563,12 +591,12 @@ static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, W
     // the block's value (the block's value came from the case or from a
     // warp that published it there).
     if (fa > 0.f && __float_as_uint(fa) > W->pubA) {
-      if (atomicMax(&P->cta_thr[0], __float_as_uint(fa)) < __float_as_uint(fa))
+      if (sh_max_old(&P->cta_thr[0], __float_as_uint(fa)) < __float_as_uint(fa))
         atomicMax(&P->g_thr[0], __float_as_uint(fa));
       W->pubA = __float_as_uint(fa);
     }
     if (fr > 0.f && __float_as_uint(fr) > W->pubR) {
-      if (atomicMax(&P->cta_thr[1], __float_as_uint(fr)) < __float_as_uint(fr))
+      if (sh_max_old(&P->cta_thr[1], __float_as_uint(fr)) < __float_as_uint(fr))
         atomicMax(&P->g_thr[1], __float_as_uint(fr));
       W->pubR = __float_as_uint(fr);
     }
@@ -629,8 +657,8 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
       cfin = isfinite(cf);
       rfin = isfinite(rf);
       equal = cf == rf;
-      if (!cfin) atomicAdd(&P->sh_cls[isnan(cf) ? 0 : (cf > 0.f ? 1 : 2)], 1);
-      if (!rfin) atomicAdd(&P->sh_cls[isnan(rf) ? 3 : (rf > 0.f ? 4 : 5)], 1);
+      if (!cfin) sh_add(&P->sh_cls[isnan(cf) ? 0 : (cf > 0.f ? 1 : 2)], 1);
+      if (!rfin) sh_add(&P->sh_cls[isnan(rf) ? 3 : (rf > 0.f ? 4 : 5)], 1);
     }
     const float as = fabsf(s[k]), ar = fabsf(rf);
     const bool fin = cfin && rfin;
@@ -666,7 +694,7 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
         sse.acc = __dadd_rn(sse.acc, __dmul_rn(d, d));
       }
     } else {
-      atomicAdd(&P->sh_cls[6], 1);
+      sh_add(&P->sh_cls[6], 1);
     }
   }
   // Exact evaluation of the screened candidates.  abs: values below the
@@ -1206,8 +1234,8 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     if (lane == 0) W->mism = 0;
     if ((j + warp) % kPoll == 0) {
       if (lane == 0) {
-        atomicMax(&P->cta_thr[0], (uint32_t)gAR);
-        atomicMax(&P->cta_thr[1], (uint32_t)(gAR >> 32));
+        sh_max(&P->cta_thr[0], (uint32_t)gAR);
+        sh_max(&P->cta_thr[1], (uint32_t)(gAR >> 32));
       }
       gAR = ld_relaxed64(g_thr);
     }
@@ -1494,15 +1522,15 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int v = P.sh_hist[t];
         if (v) {
           const int64_t tr = pc.tr0 + t / pc.wc, tc = pc.tc0 + t % pc.wc;
-          atomicAdd(&P.g_hist[tr * P.cd.GC + tc], (unsigned long long)v);
+          gl_add(&P.g_hist[tr * P.cd.GC + tc], (unsigned long long)v);
         }
       }
     }
     if (pc.prof_smem) {
       for (int64_t t = threadIdx.x; t < P.cd.th; t += kThreads)
-        if (P.sh_row[t]) atomicAdd(&P.g_row[t], (unsigned long long)P.sh_row[t]);
+        if (P.sh_row[t]) gl_add(&P.g_row[t], (unsigned long long)P.sh_row[t]);
       for (int64_t t = threadIdx.x; t < P.cd.tw; t += kThreads)
-        if (P.sh_col[t]) atomicAdd(&P.g_col[t], (unsigned long long)P.sh_col[t]);
+        if (P.sh_col[t]) gl_add(&P.g_col[t], (unsigned long long)P.sh_col[t]);
     }
     if (threadIdx.x == 0) {
       Partial Q;
