@@ -575,9 +575,12 @@ static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask,
 // After a step in which some lane's maximum changed: the warp's own
 // thresholds from the lanes' maxima (fp32 lower bounds, so no fp64 is
 // needed), publication of improvements to the case, the merged thresholds.
-//   abs: the largest fp32 strictly below fl_rd(max), or 0 when max == 0
-//        (elements not above it are not larger than a maximum at a lower
-//        index of this warp);
+//   abs: fl_rd(max), which is max itself when max is exact in fp32: an
+//        element whose exact |d| is not above it is not larger than a
+//        maximum held at a lower index of this warp (the warp sweeps its
+//        batches of a piece in ascending order), so ties with the warp's
+//        own maximum leave the fast path alone.  An inexact difference whose
+//        rounded |s| equals it may exceed it and stays a candidate;
 //   rel: fl_rd(max) (1 - 2^-20) rounded toward zero.
 static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpSh *W) {
   const int lane = threadIdx.x & 31;
@@ -585,7 +588,7 @@ static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, W
   const float fr = warp_reduce(rel_lb(L), [](float x, float y) { return fmaxf(x, y); });
   __syncwarp();
   if (lane == 0) {
-    W->wA = fa < 0.f ? -1.f : (fa > 0.f ? __uint_as_float(__float_as_uint(fa) - 1u) : 0.f);
+    W->wA = fa < 0.f ? -1.f : fa;
     W->wR = fr < 0.f ? -1.f : __fmul_rz(fr, kMarginLo);
     // Publish improvements to the block, and to the case when they raise
     // the block's value (the block's value came from the case or from a
@@ -677,7 +680,8 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     }
     if (!pass) mask |= 1u << k;
     if (fin) {
-      if (!(as <= tA)) {
+      // an inexact difference rounded onto the threshold may lie above it
+      if (!(as <= tA) || (as == tA && e[k] != 0.f)) {
         candA |= 1u << k;
         mA = fmaxf(mA, as);
       }
@@ -876,8 +880,9 @@ __device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     const float2 h2 = __ffma2_ru(ar2, hi_r2, hi_a2);
     const float2 t2 = __fmul2_rz(ar2, tR2);
     const float as0 = fabsf(s2.x), as1 = fabsf(s2.y);
-    dense &= (as0 <= a2.x || as0 > h2.x) && as0 <= tA && as0 <= t2.x;
-    dense &= (as1 <= a2.y || as1 > h2.y) && as1 <= tA && as1 <= t2.y;
+    // (an inexact difference rounded onto tA may lie above it)
+    dense &= (as0 <= a2.x || as0 > h2.x) && (as0 < tA || (as0 == tA && e[j].x == 0.f)) && as0 <= t2.x;
+    dense &= (as1 <= a2.y || as1 > h2.y) && (as1 < tA || (as1 == tA && e[j].y == 0.f)) && as1 <= t2.y;
     if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
     if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
   }

@@ -231,3 +231,30 @@ def test_relative_errors_beyond_fp32_range():
     got = validate(cand.cuda(), ref.cuda(), rtol=1e-5, atol=1e-6, tile=(1, 4096), first_k=8)
     assert_same(got, want, "rel beyond fp32")
     assert got["argmax_rel"] == 3_000_000 and got["max_rel"] > 3.4e38
+
+
+@pytest.mark.parametrize("where", [5_000, 3_000_001, (1 << 22) - 3])
+def test_max_abs_tie_with_an_inexact_difference(where):
+    # Every |c - r| is exactly 1 (all tie for the maximum; the lowest index
+    # wins) except one whose exact difference 1 + 2^-25 rounds to 1 in fp32.
+    # A warp that already holds the maximum 1 must still take that element
+    # as a candidate: its fp64 |d| is the true maximum.
+    g = torch.Generator().manual_seed(17)
+    ref = torch.randint(-1000, 1000, (1 << 22,), generator=g).float()
+    cand = ref + 1.0
+    ref[where], cand[where] = -(2.0 ** -25), 1.0
+    want = oracle.validate(cand, ref, rtol=0.0, atol=0.5, tile=(64, 64), first_k=16)
+    got = validate(cand.cuda(), ref.cuda(), rtol=0.0, atol=0.5, tile=(64, 64), first_k=16)
+    assert_same(got, want, "inexact tie")
+    assert got["argmax_abs"] == where and got["max_abs"] == 1.0 + 2.0 ** -25
+
+
+def test_max_abs_ties_everywhere_bf16():
+    # |c - r| takes a few quantised values, the largest at many indices in
+    # every piece: the argmax is the lowest of them.
+    g = torch.Generator().manual_seed(23)
+    ref = (torch.rand(6, 1024, 1024, generator=g) * 8 - 4).to(torch.bfloat16)
+    cand = (ref.float() + 0.5).to(torch.bfloat16)
+    want = oracle.validate(cand, ref, rtol=1.6e-2, atol=1e-3, tile=(128, 128), first_k=64)
+    got = validate(cand.cuda(), ref.cuda(), rtol=1.6e-2, atol=1e-3, tile=(128, 128), first_k=64)
+    assert_same(got, want, "bf16 ties")
