@@ -274,6 +274,7 @@ __device__ __forceinline__ void ff_add(float &h, float &l, float h2, float l2) {
 // Piece-constant data, in shared memory.
 struct PieceSh {
   CaseDesc cd;
+  int64_t piece;   // the piece's index in the launch
   int64_t pbegin;  // the piece's first element
   int64_t tr0, tc0;
   int32_t wr, wc, prof_smem, pad;
@@ -1327,12 +1328,11 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
 }
 
 // ------------------------------------------------------------ seeding
-// Lower bounds of |d| and |d|/|r| of element i (fp32 values rounded down
-// from its fp64 error; nothing for a non-finite pair), folded into ma, mr.
+// Lower bounds of |d| and |d|/|r| of one element from its stored bits (fp32
+// values rounded down from its fp64 error; nothing for a non-finite pair),
+// folded into ma, mr.
 template <int DT>
-__device__ __forceinline__ void seed_elem(const CaseDesc &cd, int64_t i, float &ma, float &mr) {
-  constexpr int EB = Tr<DT>::EB;
-  const uint32_t cb = ld_one<EB>(cd.cand, i), rb = ld_one<EB>(cd.ref, i);
+__device__ __forceinline__ void seed_bits(uint32_t cb, uint32_t rb, float &ma, float &mr) {
   float as, ar;
   if constexpr (Tr<DT>::kInt) {
     const long long d = (long long)(int32_t)cb - (long long)(int32_t)rb;
@@ -1347,6 +1347,27 @@ __device__ __forceinline__ void seed_elem(const CaseDesc &cd, int64_t i, float &
   }
   ma = fmaxf(ma, as);
   if (ar > 0.f) mr = fmaxf(mr, quot_lb(as, ar));
+}
+
+template <int DT>
+__device__ __forceinline__ void seed_elem(const CaseDesc &cd, int64_t i, float &ma, float &mr) {
+  constexpr int EB = Tr<DT>::EB;
+  seed_bits<DT>(ld_one<EB>(cd.cand, i), ld_one<EB>(cd.ref, i), ma, mr);
+}
+
+// The same for the V elements e .. e + V - 1 of one lane (e a multiple of
+// V): one vector load per tensor when the case is 16-byte aligned.
+template <int DT>
+__device__ __forceinline__ void seed_step(const CaseDesc &cd, int64_t e, float &ma, float &mr) {
+  constexpr int V = Tr<DT>::V;
+  if (!cd.vec_ok) {
+    for (int k = 0; k < V; ++k) seed_elem<DT>(cd, e + k, ma, mr);
+    return;
+  }
+  const uint4 cv = ld_v4((const char *)cd.cand + e * Tr<DT>::EB);
+  const uint4 rv = ld_v4((const char *)cd.ref + e * Tr<DT>::EB);
+#pragma unroll
+  for (int k = 0; k < V; ++k) seed_bits<DT>(vbits<DT>(cv, k), vbits<DT>(rv, k), ma, mr);
 }
 
 // ------------------------------------------------------------ the kernel
@@ -1386,68 +1407,87 @@ __global__ void __launch_bounds__(kThreads, 2)
   bool tr_first = true;  // the block's first piece seeds the published maxima
   // Blocks take pieces from the launch's counter as they finish the last
   // one, so pieces of uneven cost (a region wrong everywhere next to a clean
-  // one) balance over the blocks.
+  // one) balance over the blocks.  The next piece is claimed, and its
+  // descriptor fetched, by the first warp of the block to finish its sweep
+  // of the current one, behind the other warps' work.
   __shared__ int64_t sh_piece;
+  __shared__ Piece sh_pc;
+  __shared__ int32_t sh_case;    // case whose descriptor P holds (-1: none)
+  __shared__ int32_t sh_done;    // warps done with the current sweep
+  __shared__ uint32_t sh_pat[2];  // the case's first stored words (replicated for 16-bit types)
+  if (threadIdx.x == 0) {
+    const int64_t p0 = (int64_t)atomicAdd(piece_ctr, 1ull);
+    sh_piece = p0;
+    if (p0 < n_pieces) sh_pc = pieces[p0];
+    sh_case = -1;
+  }
   for (;;) {
-    if (threadIdx.x == 0) sh_piece = (int64_t)atomicAdd(piece_ctr, 1ull);
     __syncthreads();
     const int64_t p = sh_piece;
     if (p >= n_pieces) break;
-    const Piece pc = pieces[p];
+    const Piece pc = sh_pc;
+    if (sh_case != pc.case_id) {
+      // a new case: its descriptor, copied by the block in 8-byte words
+      static_assert(sizeof(CaseDesc) % 8 == 0, "CaseDesc copy");
+      const uint64_t *src = (const uint64_t *)&cases[pc.case_id];
+      for (int w = threadIdx.x; w < (int)(sizeof(CaseDesc) / 8); w += kThreads) ((uint64_t *)&P.cd)[w] = src[w];
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        uint8_t *o = out + P.cd.out_off;
+        P.g_hist = (unsigned long long *)(o + P.cd.hist_off);
+        P.g_row = (unsigned long long *)(o + P.cd.rowp_off);
+        P.g_col = (unsigned long long *)(o + P.cd.colp_off);
+        P.g_thr = g_thr + 2 * pc.case_id;
+        P.sh_cls = smem;
+        P.sh_eq = sh_eq;
+        P.cta_thr = cta_thr;
+        P.stats = stats;
+        // the block's view starts from what the case has published so far
+        const uint64_t g = ld_relaxed64(P.g_thr);
+        cta_thr[0] = (uint32_t)g;
+        cta_thr[1] = (uint32_t)(g >> 32);
+        const uint32_t c0 = ld_one<EB>(P.cd.cand, 0), r0 = ld_one<EB>(P.cd.ref, 0);
+        sh_pat[0] = EB == 2 ? (c0 | (c0 << 16)) : c0;
+        sh_pat[1] = EB == 2 ? (r0 | (r0 << 16)) : r0;
+        sh_case = pc.case_id;
+      }
+    }
     if (threadIdx.x == 0) {
-      P.cd = cases[pc.case_id];
+      P.piece = p;
       P.pbegin = pc.begin;
       P.tr0 = pc.tr0;
       P.tc0 = pc.tc0;
       P.wr = pc.wr;
       P.wc = pc.wc;
       P.prof_smem = pc.prof_smem;
-      P.sh_cls = smem;
       P.sh_row = smem + kShHead;
       P.sh_col = P.sh_row + (pc.prof_smem ? P.cd.th : 0);
       P.sh_hist = P.sh_col + (pc.prof_smem ? P.cd.tw : 0);
-      uint8_t *o = out + P.cd.out_off;
-      P.g_hist = (unsigned long long *)(o + P.cd.hist_off);
-      P.g_row = (unsigned long long *)(o + P.cd.rowp_off);
-      P.g_col = (unsigned long long *)(o + P.cd.colp_off);
-      P.g_thr = g_thr + 2 * pc.case_id;
-      P.sh_eq = sh_eq;
-      P.cta_thr = cta_thr;
-      // the block's view starts from what the case has published so far
-      const uint64_t g = ld_relaxed64(P.g_thr);
-      cta_thr[0] = (uint32_t)g;
-      cta_thr[1] = (uint32_t)(g >> 32);
-      P.stats = stats;
+      sh_done = 0;
     }
     __syncthreads();
     if (tr_first) {
-      // A sample of the case (two elements per thread of every block,
-      // spread over the whole case) seeds the published maxima, so warps
-      // start near the final thresholds instead of establishing them one
-      // light step at a time.  Every value is a lower bound of an actual
-      // element's error, published like the scan's own.
-      constexpr int kSamples = 2;
-      const int64_t total = (int64_t)gridDim.x * kThreads * kSamples;
-      const int64_t stride = P.cd.numel > total ? P.cd.numel / total : 1;
-      float ma = -1.f, mr = -1.f;
-#pragma unroll
-      for (int s2 = 0; s2 < kSamples; ++s2) {
-        const int64_t i = (((int64_t)blockIdx.x * kThreads + threadIdx.x) * kSamples + s2) * stride;
-        if (i < P.cd.numel) seed_elem<DT>(P.cd, i, ma, mr);
-      }
-      ma = warp_reduce(ma, [](float x, float y) { return fmaxf(x, y); });
-      mr = warp_reduce(mr, [](float x, float y) { return fmaxf(x, y); });
-      if (lane == 0) {
-        if (ma > 0.f) {
-          atomicMax(&cta_thr[0], __float_as_uint(ma));
-          atomicMax(&P.g_thr[0], __float_as_uint(ma));
-        }
-        if (mr > 0.f) {
-          atomicMax(&cta_thr[1], __float_as_uint(mr));
-          atomicMax(&P.g_thr[1], __float_as_uint(mr));
+      // A sample of the case seeds the published maxima, so warps start near
+      // the final thresholds instead of establishing them one light step at
+      // a time: each warp of every block reads one warp step (32 vectors,
+      // coalesced) at its own place, spread over the whole case.  Every
+      // value is a lower bound of an actual element's error, published like
+      // the scan's own (lanes -> the block's view -> once to the case).
+      constexpr int V = Tr<DT>::V;
+      const int64_t nsteps = P.cd.numel / (32 * V);
+      const int64_t slots = (int64_t)gridDim.x * kWarps;
+      if (nsteps > 0) {
+        const int64_t slot = (int64_t)blockIdx.x * kWarps + warp;
+        const int64_t st = nsteps > slots ? (nsteps / slots) * slot : slot % nsteps;
+        float ma = -1.f, mr = -1.f;
+        seed_step<DT>(P.cd, st * (32 * V) + lane * V, ma, mr);
+        ma = warp_reduce(ma, [](float x, float y) { return fmaxf(x, y); });
+        mr = warp_reduce(mr, [](float x, float y) { return fmaxf(x, y); });
+        if (lane == 0) {
+          if (ma > 0.f) atomicMax(&cta_thr[0], __float_as_uint(ma));
+          if (mr > 0.f) atomicMax(&cta_thr[1], __float_as_uint(mr));
         }
       }
-      tr_first = false;
     }
     const int64_t used = (int64_t)(P.sh_hist - smem) + (int64_t)pc.wr * pc.wc;
     for (int64_t t = threadIdx.x; t < used; t += kThreads) smem[t] = 0;
@@ -1469,6 +1509,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int k = 0; k < 9; ++k) W->st[k] = 0;
     }
     __syncthreads();
+    if (tr_first) {
+      if (threadIdx.x == 0) {
+        if (cta_thr[0] != 0u) atomicMax(&P.g_thr[0], cta_thr[0]);
+        if (cta_thr[1] != 0u) atomicMax(&P.g_thr[1], cta_thr[1]);
+      }
+      tr_first = false;
+    }
 
     Regs<NIN> R;
     R.sse.hi = R.sse.lo = make_float2(0.f, 0.f);
@@ -1476,17 +1523,20 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.cacc = R.racc = 0;
 #pragma unroll
     for (int j = 0; j < (NIN > 0 ? NIN : 1); ++j) R.eq[j] = 0;
-    {
-      const uint32_t c0 = ld_one<EB>(P.cd.cand, 0), r0 = ld_one<EB>(P.cd.ref, 0);
-      R.cpat = EB == 2 ? (c0 | (c0 << 16)) : c0;
-      R.rpat = EB == 2 ? (r0 | (r0 << 16)) : r0;
-    }
+    R.cpat = sh_pat[0];
+    R.rpat = sh_pat[1];
     R.tA = R.tR = R.tRq = R.ga = R.gr = -1.f;
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
     sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
     __syncwarp();
+    if (lane == 0 && atomicAdd(&sh_done, 1) == 0) {
+      // the first warp done claims the block's next piece
+      const int64_t nx = (int64_t)atomicAdd(piece_ctr, 1ull);
+      sh_piece = nx;
+      if (nx < n_pieces) sh_pc = pieces[nx];
+    }
     if (stats && lane == 0)
       for (int k = 0; k < 9; ++k)
         if (W->st[k]) atomicAdd(&stats[k], W->st[k]);
@@ -1522,16 +1572,16 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) w.eq[j] = eqs[j];
     }
     __syncthreads();
-    if (pc.wr > 0) {
-      for (int64_t t = threadIdx.x; t < (int64_t)pc.wr * pc.wc; t += kThreads) {
+    if (P.wr > 0) {
+      for (int64_t t = threadIdx.x; t < (int64_t)P.wr * P.wc; t += kThreads) {
         const int v = P.sh_hist[t];
         if (v) {
-          const int64_t tr = pc.tr0 + t / pc.wc, tc = pc.tc0 + t % pc.wc;
+          const int64_t tr = P.tr0 + t / P.wc, tc = P.tc0 + t % P.wc;
           gl_add(&P.g_hist[tr * P.cd.GC + tc], (unsigned long long)v);
         }
       }
     }
-    if (pc.prof_smem) {
+    if (P.prof_smem) {
       for (int64_t t = threadIdx.x; t < P.cd.th; t += kThreads)
         if (P.sh_row[t]) gl_add(&P.g_row[t], (unsigned long long)P.sh_row[t]);
       for (int64_t t = threadIdx.x; t < P.cd.tw; t += kThreads)
@@ -1559,9 +1609,8 @@ __global__ void __launch_bounds__(kThreads, 2)
       Q.arg_abs = ba.i;
       Q.best_rel = br.v;
       Q.arg_rel = br.i;
-      partials[piece_base + p] = Q;
+      partials[piece_base + P.piece] = Q;
     }
-    __syncthreads();
   }
 }
 
