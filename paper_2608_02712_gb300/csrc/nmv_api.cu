@@ -327,20 +327,38 @@ size_t piece_smem(const nmv_case &c, const Piece &p) {
   return words * 4;
 }
 
-// Split the concatenated bytes of the cases `ids` into `grid` balanced
-// ranges; cut them at case boundaries (and at kMaxPiece) into pieces whose
-// element boundaries are multiples of the case's batch (batch_elems).  The
-// scan blocks take the pieces dynamically.
+// Split the concatenated bytes of the cases `ids` into ranges for `blocks`
+// scan blocks, which take them dynamically in order: up to kGuidedLevels rounds
+// of `blocks` ranges, each round's ranges half the size of the previous
+// round's (guided self-scheduling), so the blocks start on large pieces and
+// the last ones to be taken are small and even out the blocks' finishing
+// times.  Fewer rounds are used when the smallest range would fall below a
+// minimum size (bytes of one tensor), where a piece's fixed costs would
+// outweigh the balance it buys: small for 16-bit elements, whose scan is
+// bound by instruction issue and varies more between blocks, larger for
+// 32-bit ones, which stream at close to the memory bandwidth.
+// Ranges are cut at case boundaries (and at kMaxPiece) into pieces whose
+// element boundaries are multiples of the case's batch (batch_elems).
+constexpr int kGuidedLevels = 4;
+inline int64_t min_piece_bytes(int dt) { return elem_bytes(dt) == 2 ? (96 << 10) : (512 << 10); }
+
 void make_plan(const nmv_case *cases, const std::vector<Geo> &geo, const std::vector<int64_t> &ids,
-               int grid, int nin, Plan &plan) {
+               int blocks, int nin, Plan &plan) {
   const int64_t n = (int64_t)ids.size();
   std::vector<int64_t> off(n + 1, 0);
   for (int64_t i = 0; i < n; ++i) off[i + 1] = off[i] + geo[ids[i]].numel * geo[ids[i]].eb;
   const int64_t total = off[n];
+  int levels = kGuidedLevels;
+  const int64_t min_bytes = ids.empty() ? 0 : min_piece_bytes(geo[ids[0]].dt);
+  while (levels > 1 && total / blocks / ((int64_t(1) << levels) - 1) < min_bytes) --levels;
+  // range r of round r / blocks weighs 2^(levels - 1 - round) units
+  const int grid = blocks * levels;
+  std::vector<int64_t> units(grid + 1, 0);
+  for (int r = 0; r < grid; ++r) units[r + 1] = units[r] + (int64_t(1) << (levels - 1 - r / blocks));
   std::vector<int64_t> sc(grid + 1), se(grid + 1);
   int64_t ci = 0;
   for (int b = 0; b <= grid; ++b) {
-    const int64_t x = (b == grid) ? total : (int64_t)((__int128)total * b / grid);
+    const int64_t x = (b == grid) ? total : (int64_t)((__int128)total * units[b] / units[grid]);
     while (ci < n && off[ci + 1] <= x) ++ci;
     if (ci >= n || b == grid) {
       sc[b] = n;
@@ -539,7 +557,7 @@ int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo
       int64_t g = (int64_t)S->sms * occ;
       g = std::min(g, std::max<int64_t>(1, total_bytes / 16384));
       G.grid = (int)g;
-      make_plan(cases, geo, G.ids, G.grid * kPiecesPerBlock, G.nin, G.plan);
+      make_plan(cases, geo, G.ids, G.grid, G.nin, G.plan);
       G.smem = std::max(G.plan.smem, (size_t)1024);
       if (G.plan.smem <= want) break;
       guess = G.plan.smem;

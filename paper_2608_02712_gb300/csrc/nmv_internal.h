@@ -24,7 +24,7 @@ constexpr int64_t kProfCap = 4096;        // smem row / column profile (bins eac
 // Elements per piece at most: a multiple of every batch size (so piece
 // boundaries stay on batch boundaries), small enough for int32 shared-memory
 // counters and 32-bit byte offsets within a piece.
-constexpr int kPiecesPerBlock = 2;       // pieces planned per scan block (taken dynamically)
+constexpr int kPiecesPerBlock = 2;       // pieces per scan block of the no-allocation entry point
 constexpr int64_t kMaxPiece = int64_t(3) << 27;
 
 // Element size in bytes and elements per 16-byte vector.

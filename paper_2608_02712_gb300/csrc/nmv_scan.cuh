@@ -306,6 +306,7 @@ struct LaneSh {
 struct WarpSh {
   float tA, tR;       // thresholds in force
   float wA, wR;       // the warp's own part of them (-1: no maximum held yet)
+  float cA, cR;       // the part carried from the warp's earlier pieces of the case
   float ga, gr;       // the case-wide part at the last merge (-1: none)
   uint32_t pubA, pubR;
   int64_t mism;       // mismatches so far in this batch
@@ -354,15 +355,10 @@ __device__ __forceinline__ float rel_lb(const LaneSh *L) {
   return L->r_x ? quot_lb(L->r_n, L->r_d) : __double2float_rd(L->r_v);
 }
 
-// The lane's maxima as fp64 (for the reduction at the end of a piece).
+// The lane's maximum |d| as fp64 (for the reduction at the end of a piece).
 __device__ __forceinline__ Best abs_best64(const LaneSh *L) {
   if (L->a_i == INT64_MAX) return {-1.0, INT64_MAX};
   return {L->a_x ? (double)L->a_f : L->a_v, L->a_i};
-}
-
-__device__ __forceinline__ Best rel_best64(const LaneSh *L) {
-  if (L->r_i == INT64_MAX) return {-1.0, INT64_MAX};
-  return {L->r_x ? __ddiv_rn((double)L->r_n, (double)L->r_d) : L->r_v, L->r_i};
 }
 
 // Offer |d| of element idx: as = |fl32(c - r)|, exact when e == 0; a64 is
@@ -407,6 +403,48 @@ __device__ __forceinline__ int frac_cmp(float n1, float d1, float n2, float d2) 
   const float e1 = __fmaf_rn(n1, d2, -p1), e2 = __fmaf_rn(n2, d1, -p2);
   if (e1 != e2) return e1 > e2 ? 1 : -1;
   return 0;
+}
+
+// The warp's best |d|/|r| (largest, lowest index on ties) from the lanes'
+// maxima, comparing exact fractions through frac_cmp and anything else
+// through fp64 quotients, so that an fp64 division is needed only for
+// inexact maxima and for the result; every lane returns the result.
+__device__ __forceinline__ Best rel_best_warp(const LaneSh *L) {
+  int64_t i = L->r_i;
+  int x = L->r_x;
+  float n = L->r_n, d = L->r_d;
+  double v = L->r_v;
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const int64_t i2 = __shfl_xor_sync(0xffffffffu, i, o);
+    const int x2 = __shfl_xor_sync(0xffffffffu, x, o);
+    const float n2 = __shfl_xor_sync(0xffffffffu, n, o), d2 = __shfl_xor_sync(0xffffffffu, d, o);
+    const double v2 = __shfl_xor_sync(0xffffffffu, v, o);
+    bool take;
+    if (i2 == INT64_MAX) {
+      take = false;
+    } else if (i == INT64_MAX) {
+      take = true;
+    } else {
+      const int c = (x && x2) ? frac_cmp(n2, d2, n, d) : 2;
+      if (c != 2) {
+        take = c > 0 || (c == 0 && i2 < i);
+      } else {
+        const double q = x ? __ddiv_rn((double)n, (double)d) : v;
+        const double q2 = x2 ? __ddiv_rn((double)n2, (double)d2) : v2;
+        take = beats(q2, i2, q, i);
+      }
+    }
+    if (take) {
+      i = i2;
+      x = x2;
+      n = n2;
+      d = d2;
+      v = v2;
+    }
+  }
+  if (i == INT64_MAX) return {-1.0, INT64_MAX};
+  return {x ? __ddiv_rn((double)n, (double)d) : v, i};
 }
 
 // Offer |d|/|r| of element idx (q32: its fp32 quotient for screening;
@@ -589,8 +627,8 @@ static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, W
   const float fr = warp_reduce(rel_lb(L), [](float x, float y) { return fmaxf(x, y); });
   __syncwarp();
   if (lane == 0) {
-    W->wA = fa < 0.f ? -1.f : fa;
-    W->wR = fr < 0.f ? -1.f : __fmul_rz(fr, kMarginLo);
+    W->wA = fmaxf(W->cA, fa < 0.f ? -1.f : fa);
+    W->wR = fmaxf(W->cR, fr < 0.f ? -1.f : __fmul_rz(fr, kMarginLo));
     // Publish improvements to the block, and to the case when they raise
     // the block's value (the block's value came from the case or from a
     // warp that published it there).
@@ -1414,6 +1452,7 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ Piece sh_pc;
   __shared__ int32_t sh_case;    // case whose descriptor P holds (-1: none)
   __shared__ int32_t sh_done;    // warps done with the current sweep
+  __shared__ int32_t sh_newcase;  // the current piece starts a case for this block
   __shared__ uint32_t sh_pat[2];  // the case's first stored words (replicated for 16-bit types)
   if (threadIdx.x == 0) {
     const int64_t p0 = (int64_t)atomicAdd(piece_ctr, 1ull);
@@ -1426,7 +1465,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int64_t p = sh_piece;
     if (p >= n_pieces) break;
     const Piece pc = sh_pc;
-    if (sh_case != pc.case_id) {
+    const bool newcase = sh_case != pc.case_id;
+    if (newcase) {
       // a new case: its descriptor, copied by the block in 8-byte words
       static_assert(sizeof(CaseDesc) % 8 == 0, "CaseDesc copy");
       const uint64_t *src = (const uint64_t *)&cases[pc.case_id];
@@ -1454,6 +1494,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     }
     if (threadIdx.x == 0) {
       P.piece = p;
+      sh_newcase = newcase ? 1 : 0;
       P.pbegin = pc.begin;
       P.tr0 = pc.tr0;
       P.tc0 = pc.tc0;
@@ -1503,7 +1544,15 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) sh_eq[threadIdx.x * NMV_MAX_INPUTS + j] = 0;
     }
     if (lane == 0) {
-      W->tA = W->tR = W->wA = W->wR = W->ga = W->gr = -1.f;
+      // A block takes the pieces of a case in ascending order, so the
+      // warp's own thresholds from its earlier pieces of the case bound
+      // maxima held at lower indices and carry over; a new case starts
+      // from nothing.
+      if (sh_newcase) W->wA = W->wR = -1.f;
+      W->cA = W->wA;
+      W->cR = W->wR;
+      W->ga = W->gr = -1.f;
+      merge_thr(W->wA, W->wR, W->ga, W->gr, W->tA, W->tR);
       W->pubA = W->pubR = 0;
       W->mism = 0;
       for (int k = 0; k < 9; ++k) W->st[k] = 0;
@@ -1525,7 +1574,8 @@ __global__ void __launch_bounds__(kThreads, 2)
     for (int j = 0; j < (NIN > 0 ? NIN : 1); ++j) R.eq[j] = 0;
     R.cpat = sh_pat[0];
     R.rpat = sh_pat[1];
-    R.tA = R.tR = R.tRq = R.ga = R.gr = -1.f;
+    R.ga = R.gr = -1.f;
+    reload_thr(R, W);
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
@@ -1542,25 +1592,25 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (W->st[k]) atomicAdd(&stats[k], W->st[k]);
 
     // ---- lanes -> warps -> the piece's partial
-    const Best a = best_warp(abs_best64(L)), r = best_warp(rel_best64(L));
+    const Best a = best_warp(abs_best64(L)), r = rel_best_warp(L);
     const double sse = warp_reduce(R.sse.acc, [](double x, double y) { return __dadd_rn(x, y); });
     const uint32_t cacc = warp_reduce(R.cacc | L->cacc, [](uint32_t x, uint32_t y) { return x | y; });
     const uint32_t racc = warp_reduce(R.racc | L->racc, [](uint32_t x, uint32_t y) { return x | y; });
     int eqs[NMV_MAX_INPUTS];
 #pragma unroll
     for (int j = 0; j < NMV_MAX_INPUTS; ++j) {
-      int v = 0;
-      if constexpr (NIN != 0) v = sh_eq[threadIdx.x * NMV_MAX_INPUTS + j];
-      if constexpr (NIN > 0) {
-        if (j < NIN) v += R.eq[j < NIN ? j : 0];
+      eqs[j] = 0;
+      if constexpr (NIN != 0) {
+        int v = sh_eq[threadIdx.x * NMV_MAX_INPUTS + j];
+        if constexpr (NIN > 0) {
+          if (j < NIN) v += R.eq[j < NIN ? j : 0];
+        }
+        eqs[j] = warp_reduce(v, [](int x, int y) { return x + y; });
       }
-      eqs[j] = warp_reduce(v, [](int x, int y) { return x + y; });
     }
-    int64_t mism = 0;
     if (lane == 0) {
-      mism = W->mism_tot;
       Partial &w = red[warp];
-      w.cnt[0] = mism;
+      w.cnt[0] = W->mism_tot;
       w.best_abs = a.v;
       w.arg_abs = a.i;
       w.best_rel = r.v;
@@ -1572,44 +1622,78 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) w.eq[j] = eqs[j];
     }
     __syncthreads();
-    if (P.wr > 0) {
-      for (int64_t t = threadIdx.x; t < (int64_t)P.wr * P.wc; t += kThreads) {
-        const int v = P.sh_hist[t];
-        if (v) {
-          const int64_t tr = P.tr0 + t / P.wc, tc = P.tc0 + t % P.wc;
-          gl_add(&P.g_hist[tr * P.cd.GC + tc], (unsigned long long)v);
+    if (warp != 0) {
+      // warps 1.. flush the localisation maps to the case's arrays
+      const int tid = threadIdx.x - 32, nt = kThreads - 32;
+      if (P.wr > 0) {
+        for (int64_t t = tid; t < (int64_t)P.wr * P.wc; t += nt) {
+          const int v = P.sh_hist[t];
+          if (v) {
+            const int64_t tr = P.tr0 + t / P.wc, tc = P.tc0 + t % P.wc;
+            gl_add(&P.g_hist[tr * P.cd.GC + tc], (unsigned long long)v);
+          }
         }
       }
-    }
-    if (P.prof_smem) {
-      for (int64_t t = threadIdx.x; t < P.cd.th; t += kThreads)
-        if (P.sh_row[t]) gl_add(&P.g_row[t], (unsigned long long)P.sh_row[t]);
-      for (int64_t t = threadIdx.x; t < P.cd.tw; t += kThreads)
-        if (P.sh_col[t]) gl_add(&P.g_col[t], (unsigned long long)P.sh_col[t]);
-    }
-    if (threadIdx.x == 0) {
-      Partial Q;
-      Q.cnt[0] = 0;
-      for (int k = 1; k < 8; ++k) Q.cnt[k] = smem[k - 1];
-      Best ba = {-1.0, INT64_MAX}, br = {-1.0, INT64_MAX};
-      Q.sse = 0.0;
-      Q.cacc = 0;
-      Q.racc = 0;
-      for (int j = 0; j < NMV_MAX_INPUTS; ++j) Q.eq[j] = 0;
-      for (int w = 0; w < kWarps; ++w) {
-        Q.cnt[0] += red[w].cnt[0];
-        best_offer(ba, red[w].best_abs, red[w].arg_abs);
-        best_offer(br, red[w].best_rel, red[w].arg_rel);
-        Q.sse = __dadd_rn(Q.sse, red[w].sse);
-        Q.cacc |= red[w].cacc;
-        Q.racc |= red[w].racc;
-        for (int j = 0; j < NMV_MAX_INPUTS; ++j) Q.eq[j] += red[w].eq[j];
+      if (P.prof_smem) {
+        for (int64_t t = tid; t < P.cd.th; t += nt)
+          if (P.sh_row[t]) gl_add(&P.g_row[t], (unsigned long long)P.sh_row[t]);
+        for (int64_t t = tid; t < P.cd.tw; t += nt)
+          if (P.sh_col[t]) gl_add(&P.g_col[t], (unsigned long long)P.sh_col[t]);
       }
-      Q.best_abs = ba.v;
-      Q.arg_abs = ba.i;
-      Q.best_rel = br.v;
-      Q.arg_rel = br.i;
-      partials[piece_base + P.piece] = Q;
+    } else {
+      // warp 0 combines the warps' parts: lanes 0..kWarps-1 hold one each,
+      // then a fixed tree (the same on every run)
+      int64_t m = 0;
+      Best ba = {-1.0, INT64_MAX}, br = {-1.0, INT64_MAX};
+      double s = 0.0;
+      uint32_t ca = 0, ra = 0;
+      int64_t eq[NMV_MAX_INPUTS];
+#pragma unroll
+      for (int j = 0; j < NMV_MAX_INPUTS; ++j) eq[j] = 0;
+      if (lane < kWarps) {
+        const Partial &w = red[lane];
+        m = w.cnt[0];
+        ba = {w.best_abs, w.arg_abs};
+        br = {w.best_rel, w.arg_rel};
+        s = w.sse;
+        ca = w.cacc;
+        ra = w.racc;
+        if constexpr (NIN != 0) {
+#pragma unroll
+          for (int j = 0; j < NMV_MAX_INPUTS; ++j) eq[j] = w.eq[j];
+        }
+      }
+      static_assert(kWarps == 8, "three rounds");
+#pragma unroll
+      for (int o = kWarps / 2; o; o >>= 1) {
+        m += __shfl_xor_sync(0xffffffffu, m, o);
+        best_offer(ba, __shfl_xor_sync(0xffffffffu, ba.v, o), __shfl_xor_sync(0xffffffffu, ba.i, o));
+        best_offer(br, __shfl_xor_sync(0xffffffffu, br.v, o), __shfl_xor_sync(0xffffffffu, br.i, o));
+        // lanes below the partner add the partner's value second, lanes
+        // above first, so both hold the same bits
+        const double s2 = __shfl_xor_sync(0xffffffffu, s, o);
+        s = (lane & o) ? __dadd_rn(s2, s) : __dadd_rn(s, s2);
+        ca |= __shfl_xor_sync(0xffffffffu, ca, o);
+        ra |= __shfl_xor_sync(0xffffffffu, ra, o);
+        if constexpr (NIN != 0) {
+#pragma unroll
+          for (int j = 0; j < NMV_MAX_INPUTS; ++j) eq[j] += __shfl_xor_sync(0xffffffffu, eq[j], o);
+        }
+      }
+      if (lane == 0) {
+        Partial Q;
+        Q.cnt[0] = m;
+        for (int k = 1; k < 8; ++k) Q.cnt[k] = smem[k - 1];
+        Q.best_abs = ba.v;
+        Q.arg_abs = ba.i;
+        Q.best_rel = br.v;
+        Q.arg_rel = br.i;
+        Q.sse = s;
+        Q.cacc = ca;
+        Q.racc = ra;
+        for (int j = 0; j < NMV_MAX_INPUTS; ++j) Q.eq[j] = eq[j];
+        partials[piece_base + P.piece] = Q;
+      }
     }
   }
 }
