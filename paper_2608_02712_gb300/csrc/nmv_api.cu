@@ -28,7 +28,7 @@ struct ScanOps {
                             unsigned long long *stats, uint32_t *err);
 };
 cudaError_t launch_finalize(const CaseDesc *, const Piece *, const Partial *, const int32_t *, uint8_t *,
-                            int, int, cudaStream_t);
+                            uint8_t *, uint8_t *, size_t, int, int, cudaStream_t);
 cudaError_t launch_sse64(const CaseDesc *cd, double *part, double *dst, cudaStream_t st);
 
 constexpr int kSseBlocksHost = 1024;  // scratch doubles of launch_sse64
@@ -119,13 +119,6 @@ struct Profile {
   cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
   int ev_dev = -1;
 } g_prof;
-
-// The packed results start with a call header holding the scan pass's
-// exact-path counters (filled when profiling is on) and, at byte
-// kCallErrOff, the scan kernel's error word (nonzero: a bulk copy into
-// shared memory did not complete within the kernel's wait limit).
-constexpr size_t kCallHeader = 256;
-constexpr size_t kCallErrOff = 128;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -464,6 +457,13 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.rowp_off = (int64_t)g.rowp_off;
   d.colp_off = (int64_t)g.colp_off;
   d.fk_off = (int64_t)g.fk_off;
+  d.hist_n = g.GR * g.GC;
+  d.rowp_n = c.tile_rows;
+  d.colp_n = c.tile_cols;
+  d.rank = c.cand.rank;
+  for (int k = 0; k < c.cand.rank && k < NMV_MAX_RANK; ++k)
+    d.sdiv[k] = c.cand.shape[k] > 0 ? make_div((uint64_t)c.cand.shape[k]) : Div64{0, 0};
+  d.coord_off = 0;
 }
 
 // The plan of the last call on each device: reused when the next call
@@ -480,6 +480,7 @@ struct PlanCache {
   int fin_helpers = 0;          // most finalize helper blocks of any case
   size_t out_size = 0;
   void *uploaded_ws = nullptr;  // workspace holding this plan's descriptors
+  void *zeroed_ws = nullptr;    // workspace whose accumulators the last finalize left zero
 };
 PlanCache g_plan[kMaxDevices];
 
@@ -586,6 +587,12 @@ int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo
     C.desc[i].piece_begin = C.desc[i].piece_end = 0;
     C.desc[i].batch_begin = C.desc[i].batch_end = 0;
   }
+  // the records' coordinates follow the packed results in the result block
+  size_t coord = out_size;
+  for (int64_t i = 0; i < n; ++i) {
+    C.desc[i].coord_off = (int64_t)coord;
+    coord += 8 * (size_t)cases[i].first_k * (size_t)cases[i].cand.rank;
+  }
   int64_t n_batches = 0;
   for (Group &G : C.groups) {
     for (size_t k = 0; k < G.plan.pieces.size(); ++k) {
@@ -614,6 +621,7 @@ int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo
   }
   C.out_size = out_size;
   C.uploaded_ws = nullptr;
+  C.zeroed_ws = nullptr;
   C.valid = true;
   return NMV_OK;
 }
@@ -647,7 +655,7 @@ void *arena_get(size_t bytes) {
   }
   void *p = nullptr;
   const size_t cap = std::max(bytes, (size_t)65536);
-  if (cudaHostAlloc(&p, cap, cudaHostAllocDefault) != cudaSuccess) {
+  if (cudaHostAlloc(&p, cap, cudaHostAllocMapped | cudaHostAllocPortable) != cudaSuccess) {
     cudaGetLastError();
     return nullptr;
   }
@@ -734,8 +742,10 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   if (rc) return rc;
   uint8_t *W = (uint8_t *)S->ws;
 
-  // ---- result block: the results, then the device's packed result, then
-  // the first-K coordinates
+  // ---- result block: the results, then the packed result, then the
+  // first-K coordinates.  The block is mapped pinned host memory: the
+  // finalize kernel writes the packed result and the coordinates into it
+  // directly, so no copy follows the kernels.
   const size_t res_bytes = align_up(sizeof(nmv_result) * n, 256);
   size_t coord_bytes = 0;
   for (int64_t i = 0; i < n; ++i) coord_bytes += 8 * (size_t)cases[i].first_k * (size_t)cases[i].cand.rank;
@@ -746,6 +756,13 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     ~ArenaGuard() { arena_put(p); }
   } guard{arena};
   uint8_t *HO = arena + res_bytes;
+  uint8_t *dHO = nullptr;
+  {
+    void *dp = nullptr;
+    const cudaError_t ep = cudaHostGetDevicePointer(&dp, arena, 0);
+    if (ep != cudaSuccess) return cuda_fail(ep, "cudaHostGetDevicePointer (result block)");
+    dHO = (uint8_t *)dp + res_bytes;
+  }
 
   cudaError_t e = cudaSuccess;
   const bool upload = C.uploaded_ws != S->ws;
@@ -757,8 +774,14 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
     C.uploaded_ws = S->ws;
   }
-  e = cudaMemsetAsync(W + o_thr, 0, sz_thr + out_size, st);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  // The accumulators (published maxima, piece counters, maps, counters) start
+  // at zero: the finalize of the previous call with this plan and workspace
+  // leaves them so, otherwise they are cleared here.
+  if (C.zeroed_ws != S->ws) {
+    e = cudaMemsetAsync(W + o_thr, 0, sz_thr + out_size, st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
+  }
+  C.zeroed_ws = nullptr;  // until this call completes
   const CaseDesc *d_cases = (const CaseDesc *)W;
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   unsigned long long *d_ctr = (unsigned long long *)(W + o_thr + sizeof(uint32_t) * 2 * n);
@@ -793,11 +816,9 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   }
   if (prof) cudaEventRecord(g_prof.ev[1], st);
   e = launch_finalize(d_cases, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc),
-                      W + o_out, (int)n, C.fin_helpers, st);
+                      W + o_out, dHO, W + o_thr, sz_thr, (int)n, C.fin_helpers, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   if (prof) cudaEventRecord(g_prof.ev[2], st);
-  e = cudaMemcpyAsync(HO, W + o_out, out_size, cudaMemcpyDeviceToHost, st);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (results)");
   e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   if (injected("d2h")) return fail(NMV_ECUDA, "injected copy-back failure");
@@ -808,11 +829,9 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   for (int64_t i = 0; i < n; ++i) {
     OutHeader *oh = (OutHeader *)(HO + C.desc[i].out_off);
     if (oh->max_abs > 0.0 && oh->max_abs < 0x1p-38) {
-      double *dst = (double *)(W + o_out + C.desc[i].out_off + offsetof(OutHeader, sse));
+      double *dst = (double *)(dHO + C.desc[i].out_off + offsetof(OutHeader, sse));
       e = launch_sse64(d_cases + i, (double *)(W + o_sse), dst, st);
       if (e != cudaSuccess) return cuda_fail(e, "fp64 SSE launch");
-      e = cudaMemcpyAsync(&oh->sse, dst, sizeof(double), cudaMemcpyDeviceToHost, st);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (fp64 SSE)");
       e = cudaStreamSynchronize(st);
       if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize (fp64 SSE)");
     }
@@ -842,7 +861,6 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
 
   // ---- results: scalar fields, arrays pointing into the packed copy
   nmv_result *res = (nmv_result *)arena;
-  int64_t *coords = (int64_t *)(HO + out_size);
   for (int64_t i = 0; i < n; ++i) {
     uint8_t *ob = HO + C.desc[i].out_off;
     OutHeader *oh = (OutHeader *)ob;
@@ -880,21 +898,13 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     r.fk_index = (int64_t *)(ob + g.fk_off);
     r.fk_cand = (double *)(r.fk_index + c.first_k);
     r.fk_ref = r.fk_cand + c.first_k;
-    r.fk_coords = coords;
-    for (int64_t t = 0; t < k; ++t) {
-      int64_t idx = r.fk_index[t];
-      for (int d = c.cand.rank - 1; d >= 0; --d) {
-        const int64_t sd = c.cand.shape[d];
-        coords[t * c.cand.rank + d] = sd > 0 ? idx % sd : 0;
-        idx = sd > 0 ? idx / sd : 0;
-      }
-    }
-    coords += (size_t)c.first_k * (size_t)c.cand.rank;
+    r.fk_coords = (int64_t *)(HO + C.desc[i].coord_off);  // written by the finalize
     r.n_inputs = c.n_inputs;
     r.passthrough_input = oh->passthrough;
     r.input_eq = oh->input_eq;
   }
   guard.p = nullptr;  // handed to the caller
+  C.zeroed_ws = S->ws;
   *out = res;
   g_err.clear();
   return NMV_OK;
@@ -1055,7 +1065,8 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   e = launch_finalize(d_case, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc), W + o_out,
-                      1, fin_helpers(g_na_desc.first_k, g_na_desc.batch_end - g_na_desc.batch_begin), st);
+                      nullptr, nullptr, 0, 1, fin_helpers(g_na_desc.first_k, g_na_desc.batch_end - g_na_desc.batch_begin),
+                      st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   const uint8_t *ob = W + o_out + kCallHeader;
   uint32_t kerr = 0;

@@ -24,21 +24,32 @@ __device__ __forceinline__ double widen_any(uint32_t b, int dt) {
 // What the record pass needs of one case, loaded once into registers.
 struct FkView {
   const char *cand, *ref;
-  int64_t *idx;          // record arrays of the packed result
+  int64_t *idx;          // record arrays of the packed result (device)
   double *c64, *r64;
+  uint8_t *hrec;         // the host result's record arrays (laid out as idx), or null
+  int64_t *coords;       // [first_k][rank] coordinates in the host result, or null
+  const Div64 *sdiv;     // the candidate's extents as divisors (rank entries)
+  int64_t first_k;
+  int32_t rank;
   double rtol, atol;
   float lo_r, lo_a, hi_r, hi_a;  // the fp32 pre-filter of the predicate
   int32_t ks;            // warp steps per batch
   int32_t vec_ok;
 };
 
-__device__ __forceinline__ FkView fk_view(const CaseDesc &cd, uint8_t *o) {
+// o: the case's device output; ho: its host result (or null).
+__device__ __forceinline__ FkView fk_view(const CaseDesc &cd, uint8_t *o, uint8_t *ho, uint8_t *hbase) {
   FkView F;
   F.cand = (const char *)cd.cand;
   F.ref = (const char *)cd.ref;
   F.idx = (int64_t *)(o + cd.fk_off);
   F.c64 = (double *)(F.idx + cd.first_k);
   F.r64 = F.c64 + cd.first_k;
+  F.hrec = ho ? ho + cd.fk_off : nullptr;
+  F.coords = hbase ? (int64_t *)(hbase + cd.coord_off) : nullptr;
+  F.sdiv = cd.sdiv;
+  F.first_k = cd.first_k;
+  F.rank = cd.rank;
   F.rtol = cd.rtol;
   F.atol = cd.atol;
   F.lo_r = cd.lo_r;
@@ -111,16 +122,48 @@ __device__ __forceinline__ int64_t block_excl_scan64(int64_t v, int64_t *total, 
   return sh[warp] + incl - v;
 }
 
+// Copy records [pos0, pos0 + n), written by this warp, from the device
+// arrays to the host result, with their row-major coordinates; lane t takes
+// records pos0 + t, pos0 + t + 32, ... so the stores coalesce.
+__device__ void publish_records(const FkView &F, int64_t pos0, int64_t n) {
+  __syncwarp();  // the warp's record stores are visible to its lanes
+  int64_t *hidx = (int64_t *)F.hrec;
+  double *hc = (double *)(hidx + F.first_k), *hr = hc + F.first_k;
+  for (int64_t t = threadIdx.x & 31; t < n; t += 32) {
+    const int64_t p = pos0 + t;
+    int64_t idx = F.idx[p];
+    hidx[p] = idx;
+    hc[p] = F.c64[p];
+    hr[p] = F.r64[p];
+    if (F.coords) {
+      int64_t *c = F.coords + p * F.rank;
+      for (int d = F.rank - 1; d >= 0; --d) {
+        const Div64 sd = F.sdiv[d];
+        if (sd.d == 0) {
+          c[d] = 0;
+          idx = 0;
+        } else {
+          const uint64_t q = div_q((uint64_t)idx, sd.d, sd.m);
+          c[d] = idx - (int64_t)(q * sd.d);
+          idx = (int64_t)q;
+        }
+      }
+    }
+  }
+}
+
 // Re-read elements [lo, hi) (one batch, lo batch-aligned) with one warp
 // and write the first `needed` mismatches at record positions pos0, pos0 +
 // 1, ...  Lane l takes the V elements at lo + u * 32V + lV of each warp step
-// u, as the scan does.  All of the batch's vectors are loaded up front and
-// put through the sure-pass filter together, so a batch costs one memory
+// u, as the scan does; only the steps the scan marked in sbits (those
+// holding mismatches) are read.  Their vectors are loaded up front and put
+// through the sure-pass filter together, so a batch costs one memory
 // latency and little more; only steps where some element is not surely
 // passing go through the full predicate and the warp-wide ordered
-// compaction that places their records.
+// compaction that places their records.  With a host result, the records
+// are then copied there with their coordinates.
 template <int DT>
-__device__ void reread_warp(const FkView &F, int64_t lo, int64_t hi, int64_t pos0, int64_t needed) {
+__device__ void reread_warp(const FkView &F, int64_t lo, int64_t hi, int64_t pos0, int64_t needed, uint32_t sbits) {
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
   constexpr int STEP = 32 * V;
@@ -130,7 +173,9 @@ __device__ void reread_warp(const FkView &F, int64_t lo, int64_t hi, int64_t pos
 #pragma unroll
   for (int u = 0; u < G; ++u) {
     const int64_t i0 = lo + u * STEP + lane * V;
-    if (F.vec_ok && i0 + V <= hi) {
+    if (!((sbits >> u) & 1u)) {
+      cv[u] = rv[u] = make_uint4(0, 0, 0, 0);  // no mismatch in this step
+    } else if (F.vec_ok && i0 + V <= hi) {
       cv[u] = ld_v4(F.cand + i0 * EB);
       rv[u] = ld_v4(F.ref + i0 * EB);
     } else {
@@ -158,9 +203,11 @@ __device__ void reread_warp(const FkView &F, int64_t lo, int64_t hi, int64_t pos
   for (int u = 0; u < G; ++u) {
     const int64_t i0 = lo + u * STEP + lane * V;
     uint32_t m = 0;
+    if ((sbits >> u) & 1u) {
 #pragma unroll
-    for (int k = 0; k < V; ++k)
-      if (i0 + k < hi && !sure_pass<DT>(F, vbits<DT>(cv[u], k), vbits<DT>(rv[u], k))) m |= 1u << k;
+      for (int k = 0; k < V; ++k)
+        if (i0 + k < hi && !sure_pass<DT>(F, vbits<DT>(cv[u], k), vbits<DT>(rv[u], k))) m |= 1u << k;
+    }
     open[u] = m;
   }
   int64_t found = 0;
@@ -192,6 +239,7 @@ __device__ void reread_warp(const FkView &F, int64_t lo, int64_t hi, int64_t pos
     found += __shfl_sync(0xffffffffu, incl, 31);
     if (found >= needed) break;
   }
+  if (F.hrec) publish_records(F, pos0, found < needed ? found : needed);
 }
 
 // One round of the record pass over a run of at most kFinChunk consecutive
@@ -203,8 +251,9 @@ constexpr int kFinPer = 4;
 constexpr int kFinChunk = kFinThreads * kFinPer;
 
 struct FkItem {
-  int64_t pos;   // first record position
-  int64_t id;    // piece or batch
+  int64_t pos;     // first record position
+  int32_t id;      // piece (within the launch) or batch (within the piece)
+  uint32_t sbits;  // a batch's warp steps that hold mismatches
 };
 
 // Records of one piece whose first record has position pos0 (< K): its
@@ -221,12 +270,15 @@ __device__ void first_k_piece(const FkView &F, int dt, int nin, const Piece &pc,
   for (int64_t b0 = 0; b0 < nb && pos < K; b0 += kFinChunk) {
     const int64_t bt = b0 + (int64_t)threadIdx.x * kFinPer;
     int32_t n[kFinPer];
+    uint32_t sb[kFinPer];
     // records in the low 32 bits (a chunk holds at most kFinChunk * be),
     // nonzero counts in the high ones
     int64_t packed = 0;
 #pragma unroll
     for (int t = 0; t < kFinPer; ++t) {
-      n[t] = bt + t < nb ? batch_count[pc.batch_base + bt + t] : 0;
+      const uint32_t w = bt + t < nb ? (uint32_t)batch_count[pc.batch_base + bt + t] : 0u;
+      n[t] = (int32_t)(w & kBatchCountMask);
+      sb[t] = w >> kStepBitsShift;
       packed += (int64_t)n[t] + (n[t] > 0 ? (int64_t(1) << 32) : 0);
     }
     int64_t total;
@@ -238,7 +290,7 @@ __device__ void first_k_piece(const FkView &F, int dt, int nin, const Piece &pc,
 #pragma unroll
     for (int t = 0; t < kFinPer; ++t) {
       if (n[t] > 0) {
-        sh_item[slot] = {pre, bt + t};
+        sh_item[slot] = {pre, (int32_t)(bt + t), sb[t]};
         // the last batch starting below K ends at or beyond it
         if (pre < K && pre + n[t] >= K) *sh_cnt = slot + 1;
         ++slot;
@@ -253,15 +305,43 @@ __device__ void first_k_piece(const FkView &F, int dt, int nin, const Piece &pc,
       const int64_t hi = lo + be < pc.end ? lo + be : pc.end;
       const int64_t nxt = j + 1 < n_nz ? sh_item[j + 1].pos : end_pos;
       const int64_t need = nxt < K ? nxt - pre_j : K - pre_j;
+      const uint32_t sbits = sh_item[j].sbits;
       switch (dt) {
-        case NMV_F32: reread_warp<NMV_F32>(F, lo, hi, pre_j, need); break;
-        case NMV_F16: reread_warp<NMV_F16>(F, lo, hi, pre_j, need); break;
-        case NMV_BF16: reread_warp<NMV_BF16>(F, lo, hi, pre_j, need); break;
-        default: reread_warp<NMV_I32>(F, lo, hi, pre_j, need); break;
+        case NMV_F32: reread_warp<NMV_F32>(F, lo, hi, pre_j, need, sbits); break;
+        case NMV_F16: reread_warp<NMV_F16>(F, lo, hi, pre_j, need, sbits); break;
+        case NMV_BF16: reread_warp<NMV_BF16>(F, lo, hi, pre_j, need, sbits); break;
+        default: reread_warp<NMV_I32>(F, lo, hi, pre_j, need, sbits); break;
       }
     }
     __syncthreads();
     pos = end_pos;
+  }
+}
+
+// Move n 8-byte words (n even or not; src and dst 16-byte aligned) from the
+// device to the host result and leave zeros behind, block `part` of
+// `parts`: each thread moves 16-byte pairs four at a time, loads first.
+__device__ void move_words(uint8_t *src, uint8_t *dst, int64_t n, int part, int parts) {
+  uint4 *s = (uint4 *)src, *d = (uint4 *)dst;
+  const int64_t n2 = n / 2;
+  const int64_t stride = (int64_t)parts * kFinThreads;
+  for (int64_t t0 = (int64_t)part * kFinThreads + threadIdx.x; t0 < n2; t0 += 4 * stride) {
+    uint4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) v[u] = t0 + u * stride < n2 ? s[t0 + u * stride] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (t0 + u * stride < n2) {
+        d[t0 + u * stride] = v[u];
+        if (v[u].x | v[u].y | v[u].z | v[u].w) s[t0 + u * stride] = make_uint4(0, 0, 0, 0);
+      }
+    }
+  }
+  if ((n & 1) && part == 0 && threadIdx.x == 0) {
+    unsigned long long *s1 = (unsigned long long *)src + (n - 1);
+    const unsigned long long v = *s1;
+    ((unsigned long long *)dst)[n - 1] = v;
+    if (v) *s1 = 0ull;
   }
 }
 
@@ -287,15 +367,33 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
                                                                const Piece *__restrict__ pieces,
                                                                const Partial *__restrict__ partials,
                                                                const int32_t *__restrict__ batch_count,
-                                                               uint8_t *out) {
+                                                               uint8_t *out, uint8_t *hout, uint8_t *zthr,
+                                                               size_t zthr_bytes) {
   const CaseDesc &cd = cases[blockIdx.x];
   // block 0 of the case reduces; with helpers, blocks 1 .. helpers write the
   // records meanwhile, else block 0 writes them afterwards
   const int helpers = fin_helpers(cd.first_k, cd.batch_end - cd.batch_begin);
   const int y = blockIdx.y;
   if (y > helpers) return;
+  // o: the case's part of the device output (the scan's accumulators); ho:
+  // where the packed result goes (the host result block when hout is set)
   uint8_t *o = out + cd.out_off;
-  OutHeader *H = (OutHeader *)o;
+  uint8_t *ho = hout ? hout + cd.out_off : o;
+  OutHeader *H = (OutHeader *)ho;
+  if (hout) {
+    // The maps go to the host block and their accumulators back to zero for
+    // the next call, shared over the case's blocks; block (0, 0) does the
+    // same for the call's counters and error word and clears the published
+    // maxima and piece counters.
+    const int nb = helpers + 1;
+    move_words(o + cd.hist_off, ho + cd.hist_off, cd.hist_n, y, nb);
+    move_words(o + cd.rowp_off, ho + cd.rowp_off, cd.rowp_n, y, nb);
+    move_words(o + cd.colp_off, ho + cd.colp_off, cd.colp_n, y, nb);
+    if (blockIdx.x == 0 && y == 0) {
+      move_words(out, hout, kCallHeader / 8, 0, 1);
+      for (size_t t = threadIdx.x; t < zthr_bytes / 8; t += kFinThreads) ((unsigned long long *)zthr)[t] = 0ull;
+    }
+  }
   __shared__ int64_t sh_scan[kFinThreads / 32 + 1];
   __shared__ int64_t sh_mism;
   __shared__ FkItem sh_need[kFinChunk], sh_item[kFinChunk];
@@ -406,9 +504,10 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
   // re-read by one warp of the case's record blocks.
   const int64_t K = cd.first_k;
   if (K == 0) return;
-  const FkView F = fk_view(cd, o);
+  const FkView F = fk_view(cd, o, hout ? ho : nullptr, hout);
   const int dt = cd.dtype, nin = nin_class_of(cd.n_elig);
-  const int gw = (helpers > 0 ? y - 1 : 0) * (kFinThreads / 32) + (threadIdx.x >> 5);
+  // items go round the blocks first, so a few items land on different SMs
+  const int gw = helpers > 0 ? (y - 1) + helpers * (threadIdx.x >> 5) : (threadIdx.x >> 5);
   const int nw = (helpers > 0 ? helpers : 1) * (kFinThreads / 32);
   int64_t base = 0;  // records in the pieces before this round
   for (int64_t q0 = cd.piece_begin; q0 < cd.piece_end && base < K; q0 += kFinChunk) {
@@ -425,7 +524,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
     int64_t slot = block_excl_scan64(nz, &n_nz, sh_scan);
 #pragma unroll
     for (int t = 0; t < kFinPer; ++t) {
-      if (n[t] > 0) sh_need[slot++] = {pre, qt + t};
+      if (n[t] > 0) sh_need[slot++] = {pre, (int32_t)(qt + t), 0u};
       pre += n[t];
     }
     __syncthreads();
@@ -480,11 +579,14 @@ __global__ void sse64_final(const double *part, int n, double *dst) {
 }
 
 // Grid: one column of 1 + max_helpers blocks per case (fin_helpers).
+// With hout set (a device pointer to mapped host memory laid out like
+// out), the packed results go there directly, the accumulators in out are
+// left zero, and so are the zthr_bytes (a multiple of 8) at zthr.
 cudaError_t launch_finalize(const CaseDesc *cases, const Piece *pieces, const Partial *partials,
-                            const int32_t *batch_count, uint8_t *out, int n_cases, int max_helpers,
-                            cudaStream_t st) {
+                            const int32_t *batch_count, uint8_t *out, uint8_t *hout, uint8_t *zthr,
+                            size_t zthr_bytes, int n_cases, int max_helpers, cudaStream_t st) {
   finalize_kernel<<<dim3(n_cases, 1 + max_helpers), kFinThreads, 0, st>>>(cases, pieces, partials, batch_count,
-                                                                          out);
+                                                                          out, hout, zthr, zthr_bytes);
   return cudaGetLastError();
 }
 

@@ -69,7 +69,21 @@ struct CaseDesc {
   int64_t batch_begin, batch_end;      // this case's batches (global batch indices)
   int64_t out_off;                     // byte offset of this case's packed result
   int64_t hist_off, rowp_off, colp_off, fk_off;  // byte offsets inside the packed result
+  int64_t hist_n, rowp_n, colp_n;      // entries of the histogram and the profiles
+  // the candidate's shape as divisors, for the records' coordinates
+  // (written at byte coord_off of the host result when the finalize writes
+  // there; a zero extent has d = 0)
+  int32_t rank, pad1;
+  Div64 sdiv[NMV_MAX_RANK];
+  int64_t coord_off;
 };
+
+// The packed results start with a call header holding the scan pass's
+// exact-path counters (filled when profiling is on) and, at byte
+// kCallErrOff, the scan kernel's error word (nonzero: a bulk copy into
+// shared memory did not complete within the kernel's wait limit).
+constexpr size_t kCallHeader = 256;
+constexpr size_t kCallErrOff = 128;
 
 // A contiguous element range of one case processed by one block.  It is
 // cut into batches of batch_elems(dtype) elements (the last one may be
@@ -121,6 +135,10 @@ struct OutHeader {
 constexpr int kMaxSteps = 8;
 NMV_CHD int batch_steps(int nin) { return nin == 1 ? 4 : 8; }
 NMV_CHD int stage_steps(int nin) { return batch_steps(nin) / 2; }
+// A batch's entry in the batch-count array: its mismatch count (below 2^24)
+// in the low bits, and from bit kStepBitsShift the warp steps that hold them.
+constexpr int kStepBitsShift = 24;
+constexpr uint32_t kBatchCountMask = (1u << kStepBitsShift) - 1;
 NMV_CHD int stage_bytes(int nin) { return 32 * 16 * stage_steps(nin); }  // one tensor's bytes per stage
 NMV_CHD int nin_class_of(int n_elig) { return n_elig == 0 ? 0 : (n_elig == 1 ? 1 : -1); }
 NMV_HD int64_t batch_elems(int dt, int nin) { return (int64_t)32 * vec_elems(dt) * batch_steps(nin); }

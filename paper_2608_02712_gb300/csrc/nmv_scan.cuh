@@ -310,6 +310,7 @@ struct WarpSh {
   float ga, gr;       // the case-wide part at the last merge (-1: none)
   uint32_t pubA, pubR;
   int64_t mism;       // mismatches so far in this batch
+  uint32_t sbits;     // steps of this batch that hold mismatches (bit u: warp step u)
   int64_t mism_tot;   // mismatches in the warp's batches of this piece
   uint32_t stage_b[4];  // batch held by each ring stage (kNoBatch: none)
   unsigned long long st[9];  // the warp's profile counters (layout of PieceSh::stats)
@@ -512,7 +513,13 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
   if (total == 0) return;
   const int64_t mism0 = W->mism;
   __syncwarp();
-  if (lane == 0) W->mism = mism0 + total;
+  if (lane == 0) {
+    // lane 0's element is the step's first: its warp step within the batch
+    // (32 V elements per warp step: V is 4 or 8; batch_steps is a power of two)
+    const int64_t step = (idx0 - P->pbegin) >> (V == 8 ? 8 : 7);
+    W->mism = mism0 + total;
+    W->sbits |= 1u << (uint32_t)(step & (batch_steps(nin_class_of(P->cd.n_elig)) - 1));
+  }
   const CaseDesc &cd = P->cd;
   const uint64_t N = cd.dN.d, th = cd.dth.d, tw = cd.dtw.d;
   uint64_t row = 0, col = 0, tr = 0, rp = 0, tc = 0, cp = 0;
@@ -1275,7 +1282,10 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     if (b == kNoBatch) break;
     const uint32_t erel = b * BATCH;  // element offset of the batch in the piece
     __syncwarp();
-    if (lane == 0) W->mism = 0;
+    if (lane == 0) {
+      W->mism = 0;
+      W->sbits = 0;
+    }
     if ((j + warp) % kPoll == 0) {
       if (lane == 0) {
         sh_max(&P->cta_thr[0], (uint32_t)gAR);
@@ -1350,7 +1360,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       __syncwarp();  // every lane is done with the stage before it is refilled
     }
     if (lane == 0) {
-      bcount[b] = (int32_t)W->mism;
+      bcount[b] = (int32_t)((uint32_t)W->mism | (W->sbits << kStepBitsShift));
       W->mism_tot += W->mism;
     }
     if (R.track_c | R.track_r) {
