@@ -369,6 +369,9 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
                                                                const int32_t *__restrict__ batch_count,
                                                                uint8_t *out, uint8_t *hout, uint8_t *zthr,
                                                                size_t zthr_bytes) {
+  // launched as the scan's programmatic dependent: wait until the scan grid
+  // has completed and its writes are visible (a no-op otherwise)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const CaseDesc &cd = cases[blockIdx.x];
   // block 0 of the case reduces; with helpers, blocks 1 .. helpers write the
   // records meanwhile, else block 0 writes them afterwards
@@ -582,11 +585,25 @@ __global__ void sse64_final(const double *part, int n, double *dst) {
 // With hout set (a device pointer to mapped host memory laid out like
 // out), the packed results go there directly, the accumulators in out are
 // left zero, and so are the zthr_bytes (a multiple of 8) at zthr.
+// Launched with programmatic stream serialization: its blocks may start
+// while the scan kernel before it on the stream drains, and wait for it
+// inside (griddepcontrol.wait).
 cudaError_t launch_finalize(const CaseDesc *cases, const Piece *pieces, const Partial *partials,
                             const int32_t *batch_count, uint8_t *out, uint8_t *hout, uint8_t *zthr,
                             size_t zthr_bytes, int n_cases, int max_helpers, cudaStream_t st) {
-  finalize_kernel<<<dim3(n_cases, 1 + max_helpers), kFinThreads, 0, st>>>(cases, pieces, partials, batch_count,
-                                                                          out, hout, zthr, zthr_bytes);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_cases, 1 + max_helpers);
+  cfg.blockDim = dim3(kFinThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, finalize_kernel, cases, pieces, partials, batch_count, out, hout,
+                                           zthr, zthr_bytes);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -1433,6 +1433,10 @@ __global__ void __launch_bounds__(kThreads, 2)
   constexpr int EB = Tr<DT>::EB;
   constexpr int NST = ring_stages(NIN);
   constexpr int STAGE = ring_streams(NIN) * stage_bytes(NIN);
+  // the finalize kernel, launched as this launch's programmatic dependent,
+  // may be scheduled as blocks of this one finish (it waits for the whole
+  // grid before it reads anything this kernel writes)
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   extern __shared__ __align__(128) uint8_t dsm[];
   __shared__ PieceSh P;
   __shared__ LaneSh lanes[kThreads];
