@@ -369,10 +369,17 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
                                                                const int32_t *__restrict__ batch_count,
                                                                uint8_t *out, uint8_t *hout, uint8_t *zthr,
                                                                size_t zthr_bytes) {
+  const CaseDesc &cd = cases[blockIdx.x];
+  // the inputs' first elements (for the degenerate-output flags) do not
+  // depend on the scan: read before waiting for it
+  uint32_t c0 = 0, r0 = 0;
+  if (blockIdx.y == 0 && threadIdx.x == 0 && cd.numel >= 1) {
+    c0 = ld_elem(cd.cand, 0, cd.dtype);
+    r0 = ld_elem(cd.ref, 0, cd.dtype);
+  }
   // launched as the scan's programmatic dependent: wait until the scan grid
   // has completed and its writes are visible (a no-op otherwise)
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  const CaseDesc &cd = cases[blockIdx.x];
   // block 0 of the case reduces; with helpers, blocks 1 .. helpers write the
   // records meanwhile, else block 0 writes them afterwards
   const int helpers = fin_helpers(cd.first_k, cd.batch_end - cd.batch_begin);
@@ -415,17 +422,39 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
       a.sse = 0.0;
       a.cacc = a.racc = 0;
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] = 0;
-      for (int64_t p = cd.piece_begin + threadIdx.x; p < cd.piece_end; p += kFinThreads) {
-        const Partial &Q = partials[p];
-        Red b;
-        for (int k = 0; k < 8; ++k) b.cnt[k] = Q.cnt[k];
-        b.ba = {Q.best_abs, Q.arg_abs};
-        b.br = {Q.best_rel, Q.arg_rel};
-        b.sse = Q.sse;
-        b.cacc = Q.cacc;
-        b.racc = Q.racc;
-        for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = Q.eq[j];
-        red_add(a, b);
+      const bool has_eq = cd.n_elig > 0;
+      // partials four at a time per thread, all loads before the adds (the
+      // order of the adds is the thread's pieces in ascending order)
+      for (int64_t p0 = cd.piece_begin + threadIdx.x; p0 < cd.piece_end; p0 += 4 * kFinThreads) {
+        Red b[4];
+  #pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t p = p0 + (int64_t)u * kFinThreads;
+          if (p < cd.piece_end) {
+            const Partial &Q = partials[p];
+  #pragma unroll
+            for (int k = 0; k < 8; ++k) b[u].cnt[k] = Q.cnt[k];
+            b[u].ba = {Q.best_abs, Q.arg_abs};
+            b[u].br = {Q.best_rel, Q.arg_rel};
+            b[u].sse = Q.sse;
+            b[u].cacc = Q.cacc;
+            b[u].racc = Q.racc;
+  #pragma unroll
+            for (int j = 0; j < NMV_MAX_INPUTS; ++j) b[u].eq[j] = has_eq ? Q.eq[j] : 0;
+          } else {
+  #pragma unroll
+            for (int k = 0; k < 8; ++k) b[u].cnt[k] = 0;
+            b[u].ba = {-1.0, INT64_MAX};
+            b[u].br = {-1.0, INT64_MAX};
+            b[u].sse = 0.0;
+            b[u].cacc = b[u].racc = 0;
+  #pragma unroll
+            for (int j = 0; j < NMV_MAX_INPUTS; ++j) b[u].eq[j] = 0;
+          }
+        }
+  #pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (p0 + (int64_t)u * kFinThreads < cd.piece_end) red_add(a, b[u]);
       }
   #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
@@ -439,8 +468,13 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
         b.sse = __shfl_xor_sync(0xffffffffu, a.sse, off);
         b.cacc = __shfl_xor_sync(0xffffffffu, a.cacc, off);
         b.racc = __shfl_xor_sync(0xffffffffu, a.racc, off);
+        if (has_eq) {
   #pragma unroll
-        for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = __shfl_xor_sync(0xffffffffu, a.eq[j], off);
+          for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = __shfl_xor_sync(0xffffffffu, a.eq[j], off);
+        } else {
+  #pragma unroll
+          for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = 0;
+        }
         // lanes below the partner add the partner's value second, lanes above
         // first, so both hold the same bits
         if ((threadIdx.x & off) == 0) {
@@ -481,8 +515,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
       }
       if (cd.numel >= 1) {
         const bool two = elem_bytes(cd.dtype) == 2;
-        const uint32_t c0 = ld_elem(cd.cand, 0, cd.dtype), r0 = ld_elem(cd.ref, 0, cd.dtype);
-        const uint32_t mag = cd.dtype == NMV_I32 ? 0xffffffffu : (two ? 0x7fffu : 0x7fffffffu);
+          const uint32_t mag = cd.dtype == NMV_I32 ? 0xffffffffu : (two ? 0x7fffu : 0x7fffffffu);
         const uint32_t cfold = two ? ((a.cacc | (a.cacc >> 16)) & 0xffffu) : a.cacc;
         const uint32_t rfold = two ? ((a.racc | (a.racc >> 16)) & 0xffffu) : a.racc;
         if ((c0 & mag) == 0 && (cfold & mag) == 0) flags |= NMV_FLAG_CAND_ALL_ZERO;
