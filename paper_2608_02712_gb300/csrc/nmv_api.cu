@@ -436,6 +436,10 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.dN = make_div((uint64_t)d.N);
   d.dth = make_div((uint64_t)d.th);
   d.dtw = make_div((uint64_t)d.tw);
+  d.idx32 = (g.numel <= (int64_t)0xffffffffll && d.N <= (int64_t)0xffffffffll) ? 1u : 0u;
+  d.m32N = d.idx32 ? 0xffffffffu / (uint32_t)d.N : 0u;
+  d.m32th = 0xffffffffu / (uint32_t)d.th;
+  d.m32tw = 0xffffffffu / (uint32_t)d.tw;
   d.rtol = c.rtol;
   d.atol = c.atol;
   // fp32 pre-filter coefficients (margins of 2^-20; see nmv_scan.cuh)

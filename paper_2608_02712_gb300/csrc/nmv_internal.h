@@ -60,6 +60,9 @@ struct CaseDesc {
   int32_t pad0;
   int64_t numel, M, N, th, tw, GR, GC;
   Div64 dN, dth, dtw;
+  // 32-bit reciprocals floor((2^32 - 1) / d) of N, th, tw, used when every
+  // element index fits in 32 bits (idx32 != 0)
+  uint32_t m32N, m32th, m32tw, idx32;
   double rtol, atol;
   // fp32 pre-filter of the predicate: sure-pass if |s| <= fma_rz(lo_r, |r|, lo_a),
   // sure-fail if |s| > fma_ru(hi_r, |r|, hi_a) (see nmv_scan.cuh).

@@ -68,6 +68,14 @@ __device__ __forceinline__ uint64_t div_q(uint64_t n, uint64_t d, uint64_t m) {
   return q;
 }
 
+// n / d for n < 2^32 with m = floor((2^32 - 1) / d): the product's high
+// word is the quotient or one below it.
+__device__ __forceinline__ uint32_t div_q32(uint32_t n, uint32_t d, uint32_t m) {
+  uint32_t q = __umulhi(n, m);
+  if (n - q * d >= d) q += 1;
+  return q;
+}
+
 __device__ __forceinline__ uint4 ld_v4(const void *p) {
   uint4 v;
   asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0,%1,%2,%3}, [%4];"
@@ -526,12 +534,24 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
   int64_t hbin = -1;
   bool single = false;
   if (mask) {
-    row = div_q((uint64_t)idx0, N, cd.dN.m);
-    col = (uint64_t)idx0 - row * N;
-    tr = div_q(row, th, cd.dth.m);
-    rp = row - tr * th;
-    tc = div_q(col, tw, cd.dtw.m);
-    cp = col - tc * tw;
+    if (cd.idx32) {
+      const uint32_t r32 = div_q32((uint32_t)idx0, (uint32_t)N, cd.m32N);
+      const uint32_t c32 = (uint32_t)idx0 - r32 * (uint32_t)N;
+      const uint32_t tr32 = div_q32(r32, (uint32_t)th, cd.m32th), tc32 = div_q32(c32, (uint32_t)tw, cd.m32tw);
+      row = r32;
+      col = c32;
+      tr = tr32;
+      rp = r32 - tr32 * (uint32_t)th;
+      tc = tc32;
+      cp = c32 - tc32 * (uint32_t)tw;
+    } else {
+      row = div_q((uint64_t)idx0, N, cd.dN.m);
+      col = (uint64_t)idx0 - row * N;
+      tr = div_q(row, th, cd.dth.m);
+      rp = row - tr * th;
+      tc = div_q(col, tw, cd.dtw.m);
+      cp = col - tc * tw;
+    }
     hbin = P->wr > 0 ? ((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0) : (int64_t)(tr * (uint64_t)cd.GC + tc);
     single = col + V <= N && cp + V <= tw;
   }
