@@ -149,7 +149,8 @@ typedef struct nmv_result {
 int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out);
 
 /* Validate n independent cases (a full-coverage sweep, Section 4.3) in one
- * call: one descriptor upload, one launch of each kernel, one copy back.
+ * call: one descriptor upload, one launch of each kernel, the results
+ * written by the finalize kernel straight into mapped host memory.
  * Results are identical, bit for bit, to n nmv_validate calls.  Every case
  * is checked before any work starts; an invalid case fails the whole call
  * (the message names its index).  On NMV_OK, *out points to an array of n
@@ -180,11 +181,12 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
  *    array whose size is 0 may be NULL).  The call fills them and every
  *    scalar field of *out, and leaves the pointers as they were.
  *
- * A case needs about: 4 bytes per batch of 1024 (16-bit types) or 512
+ * A case needs about: 4 bytes per batch of 2048 (16-bit types) or 1024
  * (32-bit types) elements (half that with one input of the candidate's type
  * and size), 8 bytes per histogram bin, 8 * (tile_rows + tile_cols) + 24 *
- * first_k bytes, and under 1 MiB of descriptors and partials.  A case that does not fit fails with NMV_EINVAL and a message
- * giving the bytes it needs (nmv_validate has no such limit).
+ * first_k bytes, and under 1 MiB of descriptors and partials.  A case that
+ * does not fit fails with NMV_EINVAL and a message giving the bytes it needs
+ * (nmv_validate has no such limit).
  *
  * The first call on each device looks up the scratch array's device address
  * (cudaGetSymbolAddress, with that device current); make that first call
@@ -200,8 +202,8 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
 int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out);
 
 /* Release what one nmv_validate / nmv_validate_batch call returned.  NULL
- * is accepted.  (The block is pinned host memory, which the library keeps
- * for reuse by later calls.) */
+ * is accepted.  (The block is mapped pinned host memory, which the library
+ * keeps for reuse by later calls.) */
 void nmv_result_free(nmv_result *r);
 
 /* Static text for a status code. */
