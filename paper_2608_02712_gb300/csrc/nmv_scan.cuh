@@ -530,6 +530,42 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
   }
   const CaseDesc &cd = P->cd;
   const uint64_t N = cd.dN.d, th = cd.dth.d, tw = cd.dtw.d;
+  if (cd.idx32) {
+    // The first element of the first lane holding a mismatch, computed by
+    // every lane alike: when the lanes from it to the last one holding a
+    // mismatch lie in one row and one tile, the maps need no further vote.
+    const unsigned act = __ballot_sync(0xffffffffu, mask != 0);
+    const int lead = __ffs(act) - 1, span = 32 - __clz(act) - lead;
+    const uint32_t b0 = (uint32_t)idx0 + (uint32_t)((lead - lane) * V);
+    const uint32_t r0 = div_q32(b0, (uint32_t)N, cd.m32N);
+    const uint32_t c0 = b0 - r0 * (uint32_t)N;
+    const uint32_t tc0 = div_q32(c0, (uint32_t)tw, cd.m32tw);
+    const uint32_t cp0 = c0 - tc0 * (uint32_t)tw;
+    if ((uint64_t)c0 + span * V <= N && (uint64_t)cp0 + span * V <= tw) {
+      if (lane == lead) {
+        const uint32_t tr0 = div_q32(r0, (uint32_t)th, cd.m32th);
+        const uint32_t rp0 = r0 - tr0 * (uint32_t)th;
+        const int64_t hb = P->wr > 0 ? ((int64_t)tr0 - P->tr0) * P->wc + ((int64_t)tc0 - P->tc0)
+                                     : (int64_t)((uint64_t)tr0 * (uint64_t)cd.GC + tc0);
+        if (P->wr > 0) sh_add(&P->sh_hist[hb], total);
+        else gl_add(&P->g_hist[hb], (unsigned long long)total);
+        if (P->prof_smem) sh_add(&P->sh_row[rp0], total);
+        else gl_add(&P->g_row[rp0], (unsigned long long)total);
+      }
+      if (mask) {
+        const uint32_t cp = cp0 + (uint32_t)((lane - lead) * V);  // lane >= lead here
+        if (P->prof_smem) {
+          const uint32_t base = (uint32_t)__cvta_generic_to_shared(P->sh_col + cp);
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            if (k < V && ((mask >> k) & 1u)) sh_add_at(base + 4 * k, 1);
+        } else {
+          for (uint32_t m = mask; m; m &= m - 1) gl_add(&P->g_col[cp + __ffs(m) - 1], 1ull);
+        }
+      }
+      return;
+    }
+  }
   uint64_t row = 0, col = 0, tr = 0, rp = 0, tc = 0, cp = 0;
   int64_t hbin = -1;
   bool single = false;
