@@ -359,9 +359,11 @@ __device__ __forceinline__ float abs_lb(const LaneSh *L) {
   return L->a_x ? L->a_f : __double2float_rd(L->a_v);
 }
 
+// (the exact fraction rounded down, so a maximum that fp32 holds exactly is
+// its own bound; an fp64 quotient, itself rounded, gets the 2^-20 margin)
 __device__ __forceinline__ float rel_lb(const LaneSh *L) {
   if (L->r_i == INT64_MAX) return -1.f;
-  return L->r_x ? quot_lb(L->r_n, L->r_d) : __double2float_rd(L->r_v);
+  return L->r_x ? __fdiv_rd(L->r_n, L->r_d) : __fmul_rz(__double2float_rd(L->r_v), kMarginLo);
 }
 
 // The lane's maximum |d| as fp64 (for the reduction at the end of a piece).
@@ -683,7 +685,11 @@ static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask,
 //        batches of a piece in ascending order), so ties with the warp's
 //        own maximum leave the fast path alone.  An inexact difference whose
 //        rounded |s| equals it may exceed it and stays a candidate;
-//   rel: fl_rd(max) (1 - 2^-20) rounded toward zero.
+//   rel: the largest fraction held, rounded down (the maximum itself when
+//        fp32 holds it exactly; an fp64 quotient keeps a 2^-20 margin), by
+//        the same argument; an inexact difference whose rounded |s| meets
+//        the threshold may lie above it, so the exact and dense steps
+//        compare those against the threshold less 2^-20.
 static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpSh *W) {
   const int lane = threadIdx.x & 31;
   const float fa = warp_reduce(abs_lb(L), [](float x, float y) { return fmaxf(x, y); });
@@ -691,7 +697,7 @@ static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, W
   __syncwarp();
   if (lane == 0) {
     W->wA = fmaxf(W->cA, fa < 0.f ? -1.f : fa);
-    W->wR = fmaxf(W->cR, fr < 0.f ? -1.f : __fmul_rz(fr, kMarginLo));
+    W->wR = fmaxf(W->cR, fr < 0.f ? -1.f : fr);
     // Publish improvements to the block, and to the case when they raise
     // the block's value (the block's value came from the case or from a
     // warp that published it there).
@@ -787,7 +793,8 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
         candA |= 1u << k;
         mA = fmaxf(mA, as);
       }
-      if (ar != 0.f && !(as <= __fmul_rz(tR, ar))) {
+      // (an inexact difference may lie above its rounded as: a margin)
+      if (ar != 0.f && !(as <= __fmul_rz(e[k] == 0.f ? tR : __fmul_rz(tR, kMarginLo), ar))) {
         candR |= 1u << k;
         rel[k] = rel32(as, ar);
         mR = fmaxf(mR, rel[k]);
@@ -983,8 +990,11 @@ __device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     const float2 t2 = __fmul2_rz(ar2, tR2);
     const float as0 = fabsf(s2.x), as1 = fabsf(s2.y);
     // (an inexact difference rounded onto tA may lie above it)
-    dense &= (as0 <= a2.x || as0 > h2.x) && (as0 < tA || (as0 == tA && e[j].x == 0.f)) && as0 <= t2.x;
-    dense &= (as1 <= a2.y || as1 > h2.y) && (as1 < tA || (as1 == tA && e[j].y == 0.f)) && as1 <= t2.y;
+    // (and one rounded onto tR |r|: a margin)
+    dense &= (as0 <= a2.x || as0 > h2.x) && (as0 < tA || (as0 == tA && e[j].x == 0.f)) &&
+             as0 <= (e[j].x == 0.f ? t2.x : __fmul_rz(t2.x, kMarginLo));
+    dense &= (as1 <= a2.y || as1 > h2.y) && (as1 < tA || (as1 == tA && e[j].y == 0.f)) &&
+             as1 <= (e[j].y == 0.f ? t2.y : __fmul_rz(t2.y, kMarginLo));
     if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
     if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
   }

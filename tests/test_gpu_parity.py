@@ -258,3 +258,20 @@ def test_max_abs_ties_everywhere_bf16():
     want = oracle.validate(cand, ref, rtol=1.6e-2, atol=1e-3, tile=(128, 128), first_k=64)
     got = validate(cand.cuda(), ref.cuda(), rtol=1.6e-2, atol=1e-3, tile=(128, 128), first_k=64)
     assert_same(got, want, "bf16 ties")
+
+
+def test_max_rel_tie_with_an_inexact_difference():
+    # Element A (index 5) has the exact relative error 2^24 (c - r = 1 with
+    # |r| = 2^-24); element B (index 15 * 1024 + 5, a later batch of the same
+    # warp) has fl32(c - r) = 1 too, but its exact difference 1 + 2^-24 makes
+    # its relative error 2^24 + 1: the larger, whatever the warp already holds.
+    n = 1 << 24
+    ref = torch.linspace(1.0, 2.0, n)
+    cand = ref.clone()
+    a, b = 5, 15 * 1024 + 5
+    ref[a], cand[a] = -(2.0 ** -24), 1.0 - 2.0 ** -24
+    ref[b], cand[b] = -(2.0 ** -24), 1.0
+    want = oracle.validate(cand, ref, rtol=1e-3, atol=1e-6, tile=(1, 4096), first_k=8)
+    got = validate(cand.cuda(), ref.cuda(), rtol=1e-3, atol=1e-6, tile=(1, 4096), first_k=8)
+    assert_same(got, want, "inexact rel tie")
+    assert got["argmax_rel"] == b and got["argmax_abs"] == b
