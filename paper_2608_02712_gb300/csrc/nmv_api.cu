@@ -619,9 +619,9 @@ int make_call_plan(const nmv_case *cases, int64_t n, const std::vector<Geo> &geo
   C.n_batches = n_batches;
   C.fin_helpers = 0;
   for (int64_t i = 0; i < n; ++i) {
-    const CaseDesc &d = C.desc[i];
-    const int h = fin_helpers(d.first_k, d.batch_end - d.batch_begin);
-    if (h > C.fin_helpers) C.fin_helpers = h;
+    CaseDesc &d = C.desc[i];
+    d.fin_help = fin_helpers(d.first_k, d.batch_end - d.batch_begin, n);
+    if (d.fin_help > C.fin_helpers) C.fin_helpers = d.fin_help;
   }
   C.out_size = out_size;
   C.uploaded_ws = nullptr;
@@ -1029,6 +1029,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   }
   g_na_desc.batch_begin = 0;
   g_na_desc.batch_end = n_batches;
+  g_na_desc.fin_help = fin_helpers(g_na_desc.first_k, n_batches, 1);
 
   // ---- scratch layout (the same regions as the workspace of nmv_validate)
   const size_t sz_cases = align_up(sizeof(CaseDesc), 256);
@@ -1069,8 +1070,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
   }
   e = launch_finalize(d_case, d_pieces, (const Partial *)(W + o_part), (const int32_t *)(W + o_segc), W + o_out,
-                      nullptr, nullptr, 0, 1, fin_helpers(g_na_desc.first_k, g_na_desc.batch_end - g_na_desc.batch_begin),
-                      st);
+                      nullptr, nullptr, 0, 1, g_na_desc.fin_help, st);
   if (e != cudaSuccess) return cuda_fail(e, "finalize kernel launch");
   const uint8_t *ob = W + o_out + kCallHeader;
   uint32_t kerr = 0;

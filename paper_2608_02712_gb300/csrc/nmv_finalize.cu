@@ -345,13 +345,31 @@ __device__ void move_words(uint8_t *src, uint8_t *dst, int64_t n, int part, int 
   }
 }
 
+// What the first block reduces of the partials (the pass-through counts
+// are summed separately, only for cases with inputs).
 struct Red {
   int64_t cnt[8];
   Best ba, br;
   double sse;
   uint32_t cacc, racc;
-  int64_t eq[NMV_MAX_INPUTS];
 };
+
+__device__ __forceinline__ void red_clear(Red &a) {
+  for (int k = 0; k < 8; ++k) a.cnt[k] = 0;
+  a.ba = {-1.0, INT64_MAX};
+  a.br = {-1.0, INT64_MAX};
+  a.sse = 0.0;
+  a.cacc = a.racc = 0;
+}
+
+__device__ __forceinline__ void red_load(Red &a, const Partial &Q) {
+  for (int k = 0; k < 8; ++k) a.cnt[k] = Q.cnt[k];
+  a.ba = {Q.best_abs, Q.arg_abs};
+  a.br = {Q.best_rel, Q.arg_rel};
+  a.sse = Q.sse;
+  a.cacc = Q.cacc;
+  a.racc = Q.racc;
+}
 
 __device__ __forceinline__ void red_add(Red &a, const Red &b) {
   for (int k = 0; k < 8; ++k) a.cnt[k] += b.cnt[k];
@@ -360,31 +378,31 @@ __device__ __forceinline__ void red_add(Red &a, const Red &b) {
   a.sse = __dadd_rn(a.sse, b.sse);
   a.cacc |= b.cacc;
   a.racc |= b.racc;
-  for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] += b.eq[j];
 }
 
-__global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *__restrict__ cases,
+__global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(const CaseDesc *__restrict__ cases,
                                                                const Piece *__restrict__ pieces,
                                                                const Partial *__restrict__ partials,
                                                                const int32_t *__restrict__ batch_count,
                                                                uint8_t *out, uint8_t *hout, uint8_t *zthr,
                                                                size_t zthr_bytes) {
   const CaseDesc &cd = cases[blockIdx.x];
+  // block 0 of the case reduces; with helpers, blocks 1 .. helpers write the
+  // records meanwhile, else block 0 writes them afterwards (the descriptors
+  // were uploaded before the scan started)
+  const int helpers = cd.fin_help;
+  const int y = blockIdx.y;
+  if (y > helpers) return;
   // the inputs' first elements (for the degenerate-output flags) do not
   // depend on the scan: read before waiting for it
   uint32_t c0 = 0, r0 = 0;
-  if (blockIdx.y == 0 && threadIdx.x == 0 && cd.numel >= 1) {
+  if (y == 0 && threadIdx.x == 0 && cd.numel >= 1) {
     c0 = ld_elem(cd.cand, 0, cd.dtype);
     r0 = ld_elem(cd.ref, 0, cd.dtype);
   }
   // launched as the scan's programmatic dependent: wait until the scan grid
   // has completed and its writes are visible (a no-op otherwise)
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  // block 0 of the case reduces; with helpers, blocks 1 .. helpers write the
-  // records meanwhile, else block 0 writes them afterwards
-  const int helpers = fin_helpers(cd.first_k, cd.batch_end - cd.batch_begin);
-  const int y = blockIdx.y;
-  if (y > helpers) return;
   // o: the case's part of the device output (the scan's accumulators); ho:
   // where the packed result goes (the host result block when hout is set)
   uint8_t *o = out + cd.out_off;
@@ -409,6 +427,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
   __shared__ FkItem sh_need[kFinChunk], sh_item[kFinChunk];
   __shared__ int sh_cnt;
   __shared__ Red sh_red[kFinThreads / 32];
+  __shared__ int64_t sh_eq[NMV_MAX_INPUTS];
 
   if (y == 0) {
     // ---- 1. reduce the partials: thread t takes pieces t, t + kFinThreads,
@@ -416,45 +435,16 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
     // order (the same tree on every run).
     {
       Red a;
-      for (int k = 0; k < 8; ++k) a.cnt[k] = 0;
-      a.ba = {-1.0, INT64_MAX};
-      a.br = {-1.0, INT64_MAX};
-      a.sse = 0.0;
-      a.cacc = a.racc = 0;
-      for (int j = 0; j < NMV_MAX_INPUTS; ++j) a.eq[j] = 0;
-      const bool has_eq = cd.n_elig > 0;
-      // partials four at a time per thread, all loads before the adds (the
+      red_clear(a);
+      // partials two at a time per thread, both loads before the adds (the
       // order of the adds is the thread's pieces in ascending order)
-      for (int64_t p0 = cd.piece_begin + threadIdx.x; p0 < cd.piece_end; p0 += 4 * kFinThreads) {
-        Red b[4];
-  #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int64_t p = p0 + (int64_t)u * kFinThreads;
-          if (p < cd.piece_end) {
-            const Partial &Q = partials[p];
-  #pragma unroll
-            for (int k = 0; k < 8; ++k) b[u].cnt[k] = Q.cnt[k];
-            b[u].ba = {Q.best_abs, Q.arg_abs};
-            b[u].br = {Q.best_rel, Q.arg_rel};
-            b[u].sse = Q.sse;
-            b[u].cacc = Q.cacc;
-            b[u].racc = Q.racc;
-  #pragma unroll
-            for (int j = 0; j < NMV_MAX_INPUTS; ++j) b[u].eq[j] = has_eq ? Q.eq[j] : 0;
-          } else {
-  #pragma unroll
-            for (int k = 0; k < 8; ++k) b[u].cnt[k] = 0;
-            b[u].ba = {-1.0, INT64_MAX};
-            b[u].br = {-1.0, INT64_MAX};
-            b[u].sse = 0.0;
-            b[u].cacc = b[u].racc = 0;
-  #pragma unroll
-            for (int j = 0; j < NMV_MAX_INPUTS; ++j) b[u].eq[j] = 0;
-          }
-        }
-  #pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (p0 + (int64_t)u * kFinThreads < cd.piece_end) red_add(a, b[u]);
+      for (int64_t p0 = cd.piece_begin + threadIdx.x; p0 < cd.piece_end; p0 += 2 * kFinThreads) {
+        const int64_t p1 = p0 + kFinThreads;
+        Red b0, b1;
+        red_load(b0, partials[p0]);
+        if (p1 < cd.piece_end) red_load(b1, partials[p1]);
+        red_add(a, b0);
+        if (p1 < cd.piece_end) red_add(a, b1);
       }
   #pragma unroll
       for (int off = 16; off > 0; off >>= 1) {
@@ -468,13 +458,6 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
         b.sse = __shfl_xor_sync(0xffffffffu, a.sse, off);
         b.cacc = __shfl_xor_sync(0xffffffffu, a.cacc, off);
         b.racc = __shfl_xor_sync(0xffffffffu, a.racc, off);
-        if (has_eq) {
-  #pragma unroll
-          for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = __shfl_xor_sync(0xffffffffu, a.eq[j], off);
-        } else {
-  #pragma unroll
-          for (int j = 0; j < NMV_MAX_INPUTS; ++j) b.eq[j] = 0;
-        }
         // lanes below the partner add the partner's value second, lanes above
         // first, so both hold the same bits
         if ((threadIdx.x & off) == 0) {
@@ -485,7 +468,26 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
         }
       }
       if ((threadIdx.x & 31) == 0) sh_red[threadIdx.x >> 5] = a;
+      // the pass-through counts (integers: any order)
+      if (threadIdx.x < NMV_MAX_INPUTS) sh_eq[threadIdx.x] = 0;
       __syncthreads();
+      if (cd.n_elig > 0) {
+        int64_t e[NMV_MAX_INPUTS];
+  #pragma unroll
+        for (int j = 0; j < NMV_MAX_INPUTS; ++j) e[j] = 0;
+        for (int64_t p = cd.piece_begin + threadIdx.x; p < cd.piece_end; p += kFinThreads) {
+  #pragma unroll
+          for (int j = 0; j < NMV_MAX_INPUTS; ++j)
+            if (j < cd.n_elig) e[j] += partials[p].eq[j];
+        }
+  #pragma unroll
+        for (int j = 0; j < NMV_MAX_INPUTS; ++j) {
+          if (j < cd.n_elig) {
+            const int64_t t = warp_reduce(e[j], [](int64_t x, int64_t y) { return x + y; });
+            if ((threadIdx.x & 31) == 0) atomicAdd((unsigned long long *)&sh_eq[j], (unsigned long long)t);
+          }
+        }
+      }
       if (threadIdx.x == 0) {
         for (int w = 1; w < kFinThreads / 32; ++w) red_add(sh_red[0], sh_red[w]);
       }
@@ -505,7 +507,7 @@ __global__ void __launch_bounds__(kFinThreads) finalize_kernel(const CaseDesc *_
       uint32_t flags = 0;
       int32_t pt = -1;
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) H->input_eq[j] = -1;
-      for (int j = 0; j < cd.n_elig; ++j) H->input_eq[cd.in_slot[j]] = a.eq[j];
+      for (int j = 0; j < cd.n_elig; ++j) H->input_eq[cd.in_slot[j]] = sh_eq[j];
       const int64_t thr = cd.numel >= 100 ? (cd.numel + 99) / 100 : 1;
       for (int j = 0; j < cd.n_inputs; ++j) {
         if (H->input_eq[j] >= thr) {
@@ -614,7 +616,7 @@ __global__ void sse64_final(const double *part, int n, double *dst) {
   }
 }
 
-// Grid: one column of 1 + max_helpers blocks per case (fin_helpers).
+// Grid: one column of 1 + max_helpers blocks per case (CaseDesc::fin_help).
 // With hout set (a device pointer to mapped host memory laid out like
 // out), the packed results go there directly, the accumulators in out are
 // left zero, and so are the zthr_bytes (a multiple of 8) at zthr.

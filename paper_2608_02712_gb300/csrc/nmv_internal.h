@@ -57,7 +57,7 @@ struct CaseDesc {
   int32_t dtype;
   int32_t vec_ok;                      // all buffers 16-byte aligned
   int32_t filter_ok;                   // the fp32 pre-filter of the predicate is valid
-  int32_t pad0;
+  int32_t fin_help;                    // finalize helper blocks of this case (fin_helpers)
   int64_t numel, M, N, th, tw, GR, GC;
   Div64 dN, dth, dtw;
   // 32-bit reciprocals floor((2^32 - 1) / d) of N, th, tw, used when every
@@ -150,15 +150,24 @@ NMV_HD int64_t piece_batches(int64_t begin, int64_t end, int dt, int nin) {
   return (end - begin + be - 1) / be;
 }
 
-// Finalize blocks of one case beyond the first: a case with records to write
-// and at least kFinHelperBatches batches gets one helper block per that many
-// batches (at most kFinMaxHelpers); the helpers then write the records while
-// the first block reduces the partials.
+// Finalize blocks of one case beyond the first.  A case with records to
+// write gets one helper block per kFinHelperBatches batches; in a call of at
+// most kFinFewCases cases (whose finalize grid is otherwise small) also one
+// per kFinHelperItems batches that may hold records (min(first_k,
+// batches)), so that sparse mismatches, one or two per batch, are re-read by
+// many warps at once.  At most kFinMaxHelpers; the helpers then write the
+// records while the first block reduces the partials.
 constexpr int kFinMaxHelpers = 16;
 constexpr int64_t kFinHelperBatches = 4096;
-NMV_HD int fin_helpers(int64_t first_k, int64_t n_batches) {
-  if (first_k <= 0 || n_batches < kFinHelperBatches) return 0;
-  const int64_t h = n_batches / kFinHelperBatches;
+constexpr int64_t kFinHelperItems = 16;
+constexpr int64_t kFinFewCases = 16;
+NMV_HD int fin_helpers(int64_t first_k, int64_t n_batches, int64_t n_cases) {
+  if (first_k <= 0) return 0;
+  int64_t h = n_batches / kFinHelperBatches;
+  if (n_cases <= kFinFewCases) {
+    const int64_t items = first_k < n_batches ? first_k : n_batches;
+    if (items / kFinHelperItems > h) h = items / kFinHelperItems;
+  }
   return h < kFinMaxHelpers ? (int)h : kFinMaxHelpers;
 }
 

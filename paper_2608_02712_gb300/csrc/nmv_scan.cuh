@@ -20,10 +20,11 @@
 //  * predicate: lo_* are the fp32 round-down of (1 - 2^-20) {rtol, atol}; the
 //    margin absorbs every fp32 rounding, so the element provably passes the
 //    fp64 test fl(|fl(c-r)|) <= fl(atol + fl(rtol |r|)).
-//  * max |d|/|r|: tR lies below the best relative error held, so the element
-//    provably is no new maximum (strictly below a maximum published by any
-//    warp of the case, or not above one held earlier in this warp's
-//    ascending sweep, whose index is lower).
+//  * max |d|/|r|: no fraction |d|/|r| of such an element lies between tR
+//    and the best relative error held, so the element provably is no new
+//    maximum (strictly below a maximum published by any warp of the case,
+//    or not above one held earlier in this warp's ascending sweep, whose
+//    index is lower).
 //  * max |d|: the same with tA, which is also capped at 2^56 (SSE range).
 //  * |s| <= |r|/4 gives |c - r| < min(|c|, |r|), so c - r is exact in fp32
 //    (Sterbenz's lemma): d = s exactly and d^2 = p + pe with p = fl(s*s),
@@ -285,7 +286,8 @@ struct PieceSh {
   int64_t piece;   // the piece's index in the launch
   int64_t pbegin;  // the piece's first element
   int64_t tr0, tc0;
-  int32_t wr, wc, prof_smem, pad;
+  int32_t wr, wc, prof_smem;
+  int32_t rel_ru;  // 16-bit element type: exact fractions up to 1/4 round up (rel_thr)
   int32_t *sh_cls, *sh_row, *sh_col, *sh_hist;
   unsigned long long *g_hist, *g_row, *g_col;
   uint32_t *g_thr;
@@ -359,11 +361,22 @@ __device__ __forceinline__ float abs_lb(const LaneSh *L) {
   return L->a_x ? L->a_f : __double2float_rd(L->a_v);
 }
 
-// (the exact fraction rounded down, so a maximum that fp32 holds exactly is
-// its own bound; an fp64 quotient, itself rounded, gets the 2^-20 margin)
-__device__ __forceinline__ float rel_lb(const LaneSh *L) {
+// The warp's own threshold from a lane's maximum |d|/|r| (-1 when none
+// held): a value t such that an element whose exact fraction is at most t
+// is at most the maximum.  An exact fraction n/d is rounded down (the
+// maximum itself when fp32 holds it exactly), an fp64 quotient, itself
+// rounded, gets the 2^-20 margin.  For fp16 and bf16 an exact fraction
+// q = n/d <= 1/4 is rounded up instead: with |c - r| <= |r|/4, c lies within
+// one binade of r, so q = M / (2R) for integers R < 2^11 (r's significand)
+// and M <= R/2; two such fractions q < q' differ by q' - q >= 1 / (2 R R'),
+// i.e. by more than 2^-21 q relative, while (q, ru(q)] is narrower than one
+// fp32 ulp of q (2^-23 q).  So no element the fast path can pass (|s| <=
+// |r|/4, c - r exact) has a fraction in (q, ru(q)], and ties with the
+// maximum stay on the fast path.
+__device__ __forceinline__ float rel_thr(const PieceSh *P, const LaneSh *L) {
   if (L->r_i == INT64_MAX) return -1.f;
-  return L->r_x ? __fdiv_rd(L->r_n, L->r_d) : __fmul_rz(__double2float_rd(L->r_v), kMarginLo);
+  if (!L->r_x) return __fmul_rz(__double2float_rd(L->r_v), kMarginLo);
+  return P->rel_ru && L->r_n <= 0.25f * L->r_d ? __fdiv_ru(L->r_n, L->r_d) : __fdiv_rd(L->r_n, L->r_d);
 }
 
 // The lane's maximum |d| as fp64 (for the reduction at the end of a piece).
@@ -685,15 +698,15 @@ static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask,
 //        batches of a piece in ascending order), so ties with the warp's
 //        own maximum leave the fast path alone.  An inexact difference whose
 //        rounded |s| equals it may exceed it and stays a candidate;
-//   rel: the largest fraction held, rounded down (the maximum itself when
-//        fp32 holds it exactly; an fp64 quotient keeps a 2^-20 margin), by
-//        the same argument; an inexact difference whose rounded |s| meets
-//        the threshold may lie above it, so the exact and dense steps
-//        compare those against the threshold less 2^-20.
+//   rel: rel_thr of the largest fraction held (rounded down, or for fp16
+//        and bf16 up where no other fraction can fall in between), by the
+//        same argument; an inexact difference whose rounded |s| meets the
+//        threshold may lie above it, so the exact and dense steps compare
+//        those against the threshold less 2^-20.
 static __device__ __noinline__ void refresh(const PieceSh *P, const LaneSh *L, WarpSh *W) {
   const int lane = threadIdx.x & 31;
   const float fa = warp_reduce(abs_lb(L), [](float x, float y) { return fmaxf(x, y); });
-  const float fr = warp_reduce(rel_lb(L), [](float x, float y) { return fmaxf(x, y); });
+  const float fr = warp_reduce(rel_thr(P, L), [](float x, float y) { return fmaxf(x, y); });
   __syncwarp();
   if (lane == 0) {
     W->wA = fmaxf(W->cA, fa < 0.f ? -1.f : fa);
@@ -1581,6 +1594,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       P.wr = pc.wr;
       P.wc = pc.wc;
       P.prof_smem = pc.prof_smem;
+      P.rel_ru = EB == 2 && !Tr<DT>::kInt;
       P.sh_row = smem + kShHead;
       P.sh_col = P.sh_row + (pc.prof_smem ? P.cd.th : 0);
       P.sh_hist = P.sh_col + (pc.prof_smem ? P.cd.tw : 0);

@@ -275,3 +275,47 @@ def test_max_rel_tie_with_an_inexact_difference():
     got = validate(cand.cuda(), ref.cuda(), rtol=1e-3, atol=1e-6, tile=(1, 4096), first_k=8)
     assert_same(got, want, "inexact rel tie")
     assert got["argmax_rel"] == b and got["argmax_abs"] == b
+
+
+def _closest_fractions(dt):
+    """The two closest distinct relative errors |c - r| / |r| <= 1/4 over
+    values c, r of type dt with r in [1, 2) (every binade alike), the
+    smaller one not an fp32 value: (c, r) of each."""
+    v = torch.arange(0, 1 << 16, dtype=torch.int32).to(torch.int16).view(dt).double().numpy()
+    vals = np.unique(v[np.isfinite(v) & (v >= 0.75) & (v < 2.5)])
+    C, R = np.meshgrid(vals, vals[(vals >= 1.0) & (vals < 2.0)])
+    q = np.abs(C - R) / R
+    m = (q > 0) & (np.abs(C - R) <= R / 4)
+    q, C, R = q[m], C[m], R[m]
+    o = np.argsort(q, kind="stable")
+    q, C, R = q[o], C[o], R[o]
+    gap = np.diff(q) / q[:-1]
+    gap[(gap == 0) | (q[:-1].astype(np.float32).astype(np.float64) == q[:-1])] = np.inf
+    i = int(np.argmin(gap))
+    return (C[i], R[i]), (C[i + 1], R[i + 1])
+
+
+@pytest.mark.parametrize("dt", [torch.bfloat16, torch.float16], ids=["bf16", "f16"])
+@pytest.mark.parametrize("order", ["larger_late", "larger_first", "ties_only"])
+def test_max_rel_closest_fractions_16bit(dt, order):
+    # For 16-bit types a warp's own relative-error threshold may be the
+    # maximum rounded up to fp32; the next larger relative error any pair
+    # of such values can have is farther away than that rounding, so it is
+    # still found.  The two closest fractions of the type, the smaller held
+    # many times (also earlier in the warp that meets the larger one).
+    (c1, r1), (c2, r2) = _closest_fractions(dt)
+    n = 1 << 20
+    ref = torch.ones(n, dtype=dt)
+    cand = ref.clone()
+    late = 600_000
+    small_at = [3, 5000, 100_000, late - 8 * 2048, late - 8 * 1024, late - 256, late + 1, 900_000]
+    for i in small_at:
+        cand[i], ref[i] = c1, r1
+    if order == "larger_late":
+        cand[late], ref[late] = c2, r2
+    elif order == "larger_first":
+        cand[1], ref[1] = c2, r2
+    want = oracle.validate(cand, ref, rtol=1e-3, atol=1e-3, tile=(1, 4096), first_k=16)
+    got = validate(cand.cuda(), ref.cuda(), rtol=1e-3, atol=1e-3, tile=(1, 4096), first_k=16)
+    assert_same(got, want, "closest fractions %s %s" % (dt, order))
+    assert got["argmax_rel"] == {"larger_late": late, "larger_first": 1, "ties_only": 3}[order]
