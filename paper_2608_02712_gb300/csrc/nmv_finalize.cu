@@ -256,66 +256,67 @@ struct FkItem {
   uint32_t sbits;  // a batch's warp steps that hold mismatches
 };
 
-// Records of one piece whose first record has position pos0 (< K): its
-// batch counts are taken kFinChunk at a time, and each batch holding
-// records below K is re-read by one warp of the nw warps of the case's
-// record blocks (this warp is number gw of them).  Called by the whole block
-// with uniform arguments.
-__device__ void first_k_piece(const FkView &F, int dt, int nin, const Piece &pc, const int32_t *batch_count,
-                              int64_t pos0, int64_t K, int gw, int nw, int64_t *sh_scan, FkItem *sh_item,
-                              int *sh_cnt) {
+// One round of the batch level of the record pass: the counts of the
+// case's batches b0, b0 + 1, ... (global indices; at most kFinChunk, up to
+// the case's last batch), the first of which starts at record position pos
+// (< K).  A block scan gives each batch its first record position, and
+// every batch holding records below K is re-read by one warp of the nw
+// warps of the case's record blocks (this warp is number gw of them).  The
+// case's pieces are contiguous and cut at batch boundaries, so batch b
+// starts at element (b - batch_begin) * batch_elems.  Returns the position
+// after the round's batches.  Called by the whole block with uniform
+// arguments.
+__device__ int64_t first_k_batches(const FkView &F, const CaseDesc &cd, int dt, int nin,
+                                   const int32_t *batch_count, int64_t b0, int64_t pos, int64_t K, int gw, int nw,
+                                   int64_t *sh_scan, FkItem *sh_item, int *sh_cnt) {
   const int64_t be = batch_elems(dt, nin);
-  const int64_t nb = piece_batches(pc.begin, pc.end, dt, nin);
-  int64_t pos = pos0;
-  for (int64_t b0 = 0; b0 < nb && pos < K; b0 += kFinChunk) {
-    const int64_t bt = b0 + (int64_t)threadIdx.x * kFinPer;
-    int32_t n[kFinPer];
-    uint32_t sb[kFinPer];
-    // records in the low 32 bits (a chunk holds at most kFinChunk * be),
-    // nonzero counts in the high ones
-    int64_t packed = 0;
+  const int64_t bt = b0 + (int64_t)threadIdx.x * kFinPer;
+  int32_t n[kFinPer];
+  uint32_t sb[kFinPer];
+  // records in the low 32 bits (a round holds at most kFinChunk * be),
+  // nonzero counts in the high ones
+  int64_t packed = 0;
 #pragma unroll
-    for (int t = 0; t < kFinPer; ++t) {
-      const uint32_t w = bt + t < nb ? (uint32_t)batch_count[pc.batch_base + bt + t] : 0u;
-      n[t] = (int32_t)(w & kBatchCountMask);
-      sb[t] = w >> kStepBitsShift;
-      packed += (int64_t)n[t] + (n[t] > 0 ? (int64_t(1) << 32) : 0);
-    }
-    int64_t total;
-    const int64_t ex = block_excl_scan64(packed, &total, sh_scan);
-    const int64_t end_pos = pos + (total & 0xffffffffll);
-    const int n_nz = (int)(total >> 32);
-    int64_t pre = pos + (ex & 0xffffffffll);
-    int slot = (int)(ex >> 32);
-#pragma unroll
-    for (int t = 0; t < kFinPer; ++t) {
-      if (n[t] > 0) {
-        sh_item[slot] = {pre, (int32_t)(bt + t), sb[t]};
-        // the last batch starting below K ends at or beyond it
-        if (pre < K && pre + n[t] >= K) *sh_cnt = slot + 1;
-        ++slot;
-      }
-      pre += n[t];
-    }
-    __syncthreads();
-    const int items = end_pos < K ? n_nz : *sh_cnt;
-    for (int j = gw; j < items; j += nw) {
-      const int64_t pre_j = sh_item[j].pos;
-      const int64_t lo = pc.begin + sh_item[j].id * be;
-      const int64_t hi = lo + be < pc.end ? lo + be : pc.end;
-      const int64_t nxt = j + 1 < n_nz ? sh_item[j + 1].pos : end_pos;
-      const int64_t need = nxt < K ? nxt - pre_j : K - pre_j;
-      const uint32_t sbits = sh_item[j].sbits;
-      switch (dt) {
-        case NMV_F32: reread_warp<NMV_F32>(F, lo, hi, pre_j, need, sbits); break;
-        case NMV_F16: reread_warp<NMV_F16>(F, lo, hi, pre_j, need, sbits); break;
-        case NMV_BF16: reread_warp<NMV_BF16>(F, lo, hi, pre_j, need, sbits); break;
-        default: reread_warp<NMV_I32>(F, lo, hi, pre_j, need, sbits); break;
-      }
-    }
-    __syncthreads();
-    pos = end_pos;
+  for (int t = 0; t < kFinPer; ++t) {
+    const uint32_t w = bt + t < cd.batch_end ? (uint32_t)batch_count[bt + t] : 0u;
+    n[t] = (int32_t)(w & kBatchCountMask);
+    sb[t] = w >> kStepBitsShift;
+    packed += (int64_t)n[t] + (n[t] > 0 ? (int64_t(1) << 32) : 0);
   }
+  int64_t total;
+  const int64_t ex = block_excl_scan64(packed, &total, sh_scan);
+  const int64_t end_pos = pos + (total & 0xffffffffll);
+  const int n_nz = (int)(total >> 32);
+  int64_t pre = pos + (ex & 0xffffffffll);
+  int slot = (int)(ex >> 32);
+#pragma unroll
+  for (int t = 0; t < kFinPer; ++t) {
+    if (n[t] > 0) {
+      sh_item[slot] = {pre, (int32_t)(threadIdx.x * kFinPer + t), sb[t]};
+      // the last batch starting below K ends at or beyond it
+      if (pre < K && pre + n[t] >= K) *sh_cnt = slot + 1;
+      ++slot;
+    }
+    pre += n[t];
+  }
+  __syncthreads();
+  const int items = end_pos < K ? n_nz : *sh_cnt;
+  for (int j = gw; j < items; j += nw) {
+    const int64_t pre_j = sh_item[j].pos;
+    const int64_t lo = (b0 + sh_item[j].id - cd.batch_begin) * be;
+    const int64_t hi = lo + be < cd.numel ? lo + be : cd.numel;
+    const int64_t nxt = j + 1 < n_nz ? sh_item[j + 1].pos : end_pos;
+    const int64_t need = nxt < K ? nxt - pre_j : K - pre_j;
+    const uint32_t sbits = sh_item[j].sbits;
+    switch (dt) {
+      case NMV_F32: reread_warp<NMV_F32>(F, lo, hi, pre_j, need, sbits); break;
+      case NMV_F16: reread_warp<NMV_F16>(F, lo, hi, pre_j, need, sbits); break;
+      case NMV_BF16: reread_warp<NMV_BF16>(F, lo, hi, pre_j, need, sbits); break;
+      default: reread_warp<NMV_I32>(F, lo, hi, pre_j, need, sbits); break;
+    }
+  }
+  __syncthreads();
+  return end_pos;
 }
 
 // Move n 8-byte words (n even or not; src and dst 16-byte aligned) from the
@@ -534,12 +535,13 @@ __global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(const CaseDesc
     if (helpers > 0 || cd.first_k == 0 || sh_mism == 0) return;
   }
 
-  // ---- 2. first-K records.  Pieces are taken kFinChunk at a time; block
-  // scans of their mismatch counts and of their nonzero flags give each
-  // piece its first record position and each nonzero piece its slot, in
-  // order.  The pieces holding records below K are then scanned the same
-  // way over their batch counts, and every batch holding records below K is
-  // re-read by one warp of the case's record blocks.
+  // ---- 2. first-K records, in two levels.  The pieces' mismatch counts
+  // are taken kFinChunk at a time: block scans of them and of their nonzero
+  // flags give each piece its first record position and each nonzero piece
+  // its slot, in order.  From the first piece holding records below K, the
+  // batch counts are then scanned kFinChunk batches at a time across piece
+  // boundaries (first_k_batches), jumping over runs of pieces without
+  // records, until K records are placed.
   const int64_t K = cd.first_k;
   if (K == 0) return;
   const FkView F = fk_view(cd, o, hout ? ho : nullptr, hout);
@@ -547,8 +549,10 @@ __global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(const CaseDesc
   // items go round the blocks first, so a few items land on different SMs
   const int gw = helpers > 0 ? (y - 1) + helpers * (threadIdx.x >> 5) : (threadIdx.x >> 5);
   const int nw = (helpers > 0 ? helpers : 1) * (kFinThreads / 32);
-  int64_t base = 0;  // records in the pieces before this round
-  for (int64_t q0 = cd.piece_begin; q0 < cd.piece_end && base < K; q0 += kFinChunk) {
+  int64_t base = 0;               // records in the pieces before this round
+  int64_t cur = cd.batch_begin;   // first batch not scanned yet
+  int64_t pos = 0;                // records before batch cur
+  for (int64_t q0 = cd.piece_begin; q0 < cd.piece_end && base < K && pos < K; q0 += kFinChunk) {
     const int64_t qt = q0 + (int64_t)threadIdx.x * kFinPer;
     int64_t n[kFinPer], s = 0, nz = 0;
 #pragma unroll
@@ -566,11 +570,20 @@ __global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(const CaseDesc
       pre += n[t];
     }
     __syncthreads();
-    for (int64_t j = 0; j < n_nz; ++j) {
+    for (int64_t j = 0; j < n_nz && pos < K; ++j) {
       const int64_t pos0 = sh_need[j].pos;
       if (pos0 >= K) break;
-      first_k_piece(F, dt, nin, pieces[sh_need[j].id], batch_count, pos0, K, gw, nw, sh_scan, sh_item,
-                    &sh_cnt);
+      const Piece &pc = pieces[sh_need[j].id];
+      const int64_t pend = pc.batch_base + piece_batches(pc.begin, pc.end, dt, nin);
+      if (pend <= cur) continue;  // scanned with an earlier piece
+      if (pc.batch_base > cur) {
+        cur = pc.batch_base;      // the batches before hold no records
+        pos = pos0;
+      }
+      while (cur < pend && pos < K) {
+        pos = first_k_batches(F, cd, dt, nin, batch_count, cur, pos, K, gw, nw, sh_scan, sh_item, &sh_cnt);
+        cur = cur + kFinChunk < cd.batch_end ? cur + kFinChunk : cd.batch_end;
+      }
     }
     base += total;
     __syncthreads();
