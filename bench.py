@@ -47,11 +47,21 @@ def parse():
     ap.add_argument("--c2-batch", type=int, default=8,
                     help="leading dimension of the c2 workload (8 = full size); smaller "
                          "values give the small cases used for profiler captures")
+    ap.add_argument("--c5-rows", type=int, default=32768,
+                    help="rows of the c5 workload (32768 = full size, 65536 columns)")
+    ap.add_argument("--no-inputs", action="store_true",
+                    help="drop the cases' inputs (c5 as a plain cand/ref pair, same data)")
     return ap.parse_args()
 
 
 # ------------------------------------------------------------- workloads
-def make_cases(config: str, device, seed_shift: int = 0, c2_batch: int = 8):
+def make_cases(config: str, device, seed_shift: int = 0, c2_batch: int = 8, c5_rows: int = 32768,
+               no_inputs: bool = False):
+    cases = _make_cases(config, device, seed_shift, c2_batch, c5_rows)
+    return [dict(c, inputs=[]) for c in cases] if no_inputs else cases
+
+
+def _make_cases(config, device, seed_shift, c2_batch, c5_rows):
     from paper_2608_02712_gb300 import workloads as W
     if config == "c1":
         return [W.c1(seed=0 + seed_shift, device=device)]
@@ -61,7 +71,7 @@ def make_cases(config: str, device, seed_shift: int = 0, c2_batch: int = 8):
         return W.c3(seed=2 + seed_shift, device=device)
     if config == "c4":
         return [W.c4(seed=3 + seed_shift, device=device)]
-    return [W.c5(seed=4 + seed_shift, device=device)]
+    return [W.c5(seed=4 + seed_shift, device=device, shape=(c5_rows, 65536))]
 
 
 def case_bytes(c, with_inputs=False):
@@ -164,6 +174,11 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def full_size(args) -> bool:
+    """The workload at the size and with the inputs that the benchmark names."""
+    return args.c2_batch == 8 and args.c5_rows == 32768 and not args.no_inputs
+
+
 def profiled_traffic(config: str):
     """DRAM bytes per scan launch from the committed ncu summary, when it was
     taken on the current kernel source (else None)."""
@@ -184,17 +199,42 @@ def profiled_traffic(config: str):
 
 
 # ------------------------------------------------------------ reference
-def oracle_step_time(cases, rows):
-    """Run the oracle on the first `rows` rows of the [M, N] view of case 0."""
+def sample_units(cases):
+    """What a bounded oracle sample counts: rows of the [M, N] view of a single
+    case, or whole cases of a batch."""
+    if len(cases) > 1:
+        return len(cases)
+    c = cases[0]["cand"]
+    return c.reshape(-1, c.shape[-1]).shape[0] if c.dim() else 1
+
+
+def sample_text(cases, units, nbytes):
+    what = "cases of the batch" if len(cases) > 1 else "rows of the [M, N] view"
+    return "first %d %s (%d bytes of cand+ref)" % (units, what, nbytes)
+
+
+def oracle_step_time(cases, units):
+    """Run the oracle on a sample: the first `units` rows of the [M, N] view
+    of a single case (its inputs cut to the same elements), or the first
+    `units` cases of a batch."""
     import oracle
-    c = cases[0]
-    n = c["cand"].shape[-1]
-    cv = c["cand"].reshape(-1, n)[:rows]
-    rv = c["ref"].reshape(-1, n)[:rows]
     t0 = time.perf_counter()
-    oracle.validate(cv, rv, rtol=c["rtol"], atol=c["atol"], tile=c["tile"],
-                    first_k=c["first_k"])
-    return time.perf_counter() - t0, cv.numel() * cv.element_size() * 2
+    nbytes = 0
+    if len(cases) > 1:
+        for c in cases[:units]:
+            oracle.validate(c["cand"], c["ref"], inputs=c["inputs"], rtol=c["rtol"], atol=c["atol"],
+                            tile=c["tile"], first_k=c["first_k"])
+            nbytes += case_bytes(c)
+    else:
+        c = cases[0]
+        n = c["cand"].shape[-1] if c["cand"].dim() else 1
+        cv = c["cand"].reshape(-1, n)[:units]
+        rv = c["ref"].reshape(-1, n)[:units]
+        xs = [x.reshape(-1)[:cv.numel()] for x in c["inputs"]]
+        oracle.validate(cv, rv, inputs=xs, rtol=c["rtol"], atol=c["atol"], tile=c["tile"],
+                        first_k=c["first_k"])
+        nbytes = cv.numel() * cv.element_size() * 2
+    return time.perf_counter() - t0, nbytes
 
 
 def host_copy(cases):
@@ -204,14 +244,13 @@ def host_copy(cases):
 
 def cpu_baseline(cases_host, budget_s=12.0):
     """The oracle as it stands, on one host core, on a bounded row sample."""
-    n_rows = cases_host[0]["cand"].reshape(-1, cases_host[0]["cand"].shape[-1]).shape[0]
-    rows = min(n_rows, 256)
-    t, b = oracle_step_time(cases_host, rows)
-    rows = int(min(n_rows, max(rows, rows * budget_s / max(t, 1e-6))))
-    t, b = oracle_step_time(cases_host, rows)
+    n = sample_units(cases_host)
+    units = min(n, 4 if len(cases_host) > 1 else 256)
+    t, b = oracle_step_time(cases_host, units)
+    units = int(min(n, max(units, units * budget_s / max(t, 1e-6))))
+    t, b = oracle_step_time(cases_host, units)
     return {"value": b / t / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": "first %d rows of the [M, N] view (%d bytes of cand+ref), one pass, "
-                      "%.1f s" % (rows, b, t)}
+            "sample": "%s, one pass, %.1f s" % (sample_text(cases_host, units, b), t)}
 
 
 def run_reference(args, rank, world):
@@ -219,21 +258,22 @@ def run_reference(args, rank, world):
     if rank != 0:
         return None
     dev = "cuda" if torch.cuda.is_available() else "cpu"
-    cases = host_copy(make_cases(args.config if args.config != "c3" else "c2", dev,
-                                 c2_batch=args.c2_batch))
-    n_rows = cases[0]["cand"].reshape(-1, cases[0]["cand"].shape[-1]).shape[0]
-    t, _ = oracle_step_time(cases, 64)
+    cases = host_copy(make_cases(args.config, dev, c2_batch=args.c2_batch, c5_rows=args.c5_rows,
+                                 no_inputs=args.no_inputs))
+    n = sample_units(cases)
+    probe = min(n, 4 if len(cases) > 1 else 64)
+    t, _ = oracle_step_time(cases, probe)
     per_step = 150.0 / max(1, args.steps + args.warmup)
-    rows = int(min(n_rows, max(1, 64 * per_step / max(t, 1e-6))))
+    units = int(min(n, max(1, probe * per_step / max(t, 1e-6))))
     for _ in range(args.warmup):
-        oracle_step_time(cases, rows)
+        oracle_step_time(cases, units)
     times, nbytes = [], 0
     for _ in range(args.steps):
-        dt, nbytes = oracle_step_time(cases, rows)
+        dt, nbytes = oracle_step_time(cases, units)
         times.append(dt)
     total = sum(times)
     value = nbytes * args.steps / total / 1e9
-    sample = "first %d rows of the [M, N] view per step (%d bytes of cand+ref)" % (rows, nbytes)
+    sample = sample_text(cases, units, nbytes) + " per step"
     return {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
@@ -254,7 +294,8 @@ def run_ours(args, rank, world, local_rank):
     from paper_2608_02712_gb300 import nmv as nmvmod
 
     torch.cuda.set_device(local_rank)
-    cases = make_cases(args.config, "cuda", seed_shift=0, c2_batch=args.c2_batch)
+    cases = make_cases(args.config, "cuda", seed_shift=0, c2_batch=args.c2_batch, c5_rows=args.c5_rows,
+                       no_inputs=args.no_inputs)
     torch.cuda.synchronize()
     nbytes = sum(case_bytes(c) for c in cases)
     algo_bytes = sum(case_bytes(c, with_inputs=True) for c in cases)
@@ -361,7 +402,7 @@ def run_ours(args, rank, world, local_rank):
                        parallelism="replicas" if world > 1 else "1 GPU",
                        pct_of_hbm_peak=100.0 * value / world / peak),
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": profiled_traffic(args.config),
+                     "frac": achieved / peak, "traffic": profiled_traffic(args.config) if full_size(args) else None,
                      "kernel": "scan_kernel", "peak_source": peak_src,
                      "algorithmic_bytes_per_launch": algo_bytes,
                      "scan_ms_mean": scan_mean, "scan_ms_min": min(scan_ms),
