@@ -198,6 +198,24 @@ def profiled_traffic(config: str):
         return None
 
 
+# ------------------------------------------------------------ ranks
+def max_over_ranks(value: float, world: int, device) -> float:
+    """The slowest rank's figure (every rank passes its own; all get the max)."""
+    if world <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_gbs(nbytes_per_rank: int, world: int, ms: float) -> float:
+    """Whole-job throughput: every rank's bytes over the slowest rank's time
+    (replicas: each rank validates its own copy of the workload)."""
+    return world * nbytes_per_rank / (ms * 1e-3) / 1e9
+
+
 # ------------------------------------------------------------ reference
 def sample_units(cases):
     """What a bounded oracle sample counts: rows of the [M, N] view of a single
@@ -333,18 +351,14 @@ def run_ours(args, rank, world, local_rank):
         ev1.record(stream)
         torch.cuda.synchronize()
     barrier()
-    elapsed_ms = ev0.elapsed_time(ev1)
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(ev0.elapsed_time(ev1), world, "cuda")
     ms_per_step = elapsed_ms / args.steps
     # one more call with the exact-path counters (kept out of the timed loop)
     nmvmod.profile_enable(nmvmod.PROFILE_TIMING | nmvmod.PROFILE_COUNTERS)
     prep.call()
     pr = nmvmod.profile_last()
     nmvmod.profile_enable(False)
-    value = world * nbytes / (ms_per_step * 1e-3) / 1e9
+    value = job_gbs(nbytes, world, ms_per_step)
 
     # e2e: pinned host buffers -> device copies -> validate -> results back
     host = [dict(c, cand=c["cand"].cpu().pin_memory(), ref=c["ref"].cpu().pin_memory(),
@@ -379,11 +393,7 @@ def run_ours(args, rank, world, local_rank):
     e1.record(stream)
     torch.cuda.synchronize()
     barrier()
-    e2e_ms = e0.elapsed_time(e1) / ke
-    if world > 1:
-        t = torch.tensor([e2e_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / ke, world, "cuda")
 
     if rank != 0:
         return None
@@ -409,7 +419,7 @@ def run_ours(args, rank, world, local_rank):
                      "slow_steps": pr["slow_steps"], "light_steps": pr["light_steps"],
                      "exact_abs": pr["exact_abs"],
                      "exact_rel": pr["exact_rel"], "exact_pred": pr["exact_pred"]},
-        "e2e": {"value": world * nbytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
+        "e2e": {"value": job_gbs(nbytes, world, e2e_ms), "unit": "GB/s",
                 "h2d_bytes_per_step": copied + lib_h2d, "d2h_bytes_per_step": lib_d2h,
                 "ms_per_step": e2e_ms},
         "gpu_launches": launches,
