@@ -415,3 +415,83 @@ def test_c5_full_size():
     np.testing.assert_array_equal(got["tile_hist"], p["hist"])
     np.testing.assert_array_equal(got["row_prof"], p["rowp"])
     np.testing.assert_array_equal(got["col_prof"], p["colp"])
+
+
+def test_concurrent_calls_from_threads():
+    """Four host threads, each on its own stream with its own case, call the
+    library in turns that interleave: every result equals that case's
+    single-threaded result, bit for bit."""
+    import threading
+
+    cases = [workloads.fuzz(5000 + i, device="cuda") for i in range(4)]
+    want = [_gpu(c) for c in cases]
+    errors = []
+
+    def worker(i):
+        try:
+            s = torch.cuda.Stream()
+            c = cases[i]
+            for _ in range(10):
+                got = validate(c["cand"], c["ref"], inputs=c["inputs"], rtol=c["rtol"],
+                               atol=c["atol"], tile=c["tile"], first_k=c["first_k"], stream=s)
+                for k, a in got.items():
+                    b = want[i][k]
+                    same = (a.dtype == b.dtype and np.array_equal(a.view(np.uint8), b.view(np.uint8))
+                            if isinstance(a, np.ndarray) else (a == b or (a != a and b != b)))
+                    if not same:
+                        errors.append((i, k))
+        except Exception as e:  # noqa: BLE001 - reported below
+            errors.append((i, repr(e)))
+
+    threads = [threading.Thread(target=worker, args=(i,)) for i in range(4)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors[:5]
+
+
+@pytest.mark.parametrize("shape", [((1 << 32) + 4099,), (2, (1 << 31) + 4099)], ids=["1d", "2d"])
+def test_indices_beyond_32_bits(shape):
+    """More than 2^32 elements (bf16, 8 GiB per tensor): the scan's 64-bit
+    index path.  Planted errors on both sides of 2^32 give every output in
+    closed form: the records, their coordinates, the maxima and their
+    indices, the histogram bins, the profiles and the SSE."""
+    free, _ = torch.cuda.mem_get_info()
+    if free < (40 << 30):
+        pytest.skip("needs 40 GiB of free device memory")
+    numel = int(np.prod(shape))
+    ref = torch.ones(shape, dtype=torch.bfloat16, device="cuda")
+    cand = ref.clone()
+    small = [5, (1 << 32) - 1, 1 << 32, (1 << 32) + 777, numel - 1]
+    big = (1 << 32) + 999
+    cf = cand.view(-1)
+    for i in small:
+        cf[i] = 1.5
+    cf[big] = 3.0
+    th, tw = 2, 4096
+    got = validate(cand, ref, rtol=1e-2, atol=0.0, tile=(th, tw), first_k=8)
+    planted = sorted(small + [big])
+    assert got["mismatch"] == 6 and not got["pass"]
+    assert got["k_out"] == 6
+    np.testing.assert_array_equal(got["fk_index"], planted)
+    np.testing.assert_array_equal(got["fk_coords"], np.stack(np.unravel_index(planted, shape), 1))
+    np.testing.assert_array_equal(got["fk_cand"], [3.0 if i == big else 1.5 for i in planted])
+    np.testing.assert_array_equal(got["fk_ref"], [1.0] * 6)
+    assert got["max_abs"] == 2.0 and got["argmax_abs"] == big
+    assert got["max_rel"] == 2.0 and got["argmax_rel"] == big
+    assert got["sse"] == 5 * 0.25 + 4.0
+    assert got["n_finite_pairs"] == numel
+    N = shape[-1]
+    hist = np.zeros_like(got["tile_hist"])
+    rowp = np.zeros(th, np.int64)
+    colp = np.zeros(tw, np.int64)
+    for i in planted:
+        r, c = divmod(i, N)
+        hist[r // th, c // tw] += 1
+        rowp[r % th] += 1
+        colp[c % tw] += 1
+    np.testing.assert_array_equal(got["tile_hist"], hist)
+    np.testing.assert_array_equal(got["row_prof"], rowp)
+    np.testing.assert_array_equal(got["col_prof"], colp)
+    assert got["flags"] == 16  # NMV_FLAG_REF_CONSTANT: the reference is all ones
