@@ -149,8 +149,9 @@ typedef struct nmv_result {
 int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out);
 
 /* Validate n independent cases (a full-coverage sweep, Section 4.3) in one
- * call: one descriptor upload, one launch of each kernel, the results
- * written by the finalize kernel straight into mapped host memory.
+ * call: one descriptor upload, one launch of the scan kernel per element
+ * type and input class present, one launch of the finalize kernel, the
+ * results written by the finalize kernel straight into mapped host memory.
  * Results are identical, bit for bit, to n nmv_validate calls.  Every case
  * is checked before any work starts; an invalid case fails the whole call
  * (the message names its index).  On NMV_OK, *out points to an array of n
