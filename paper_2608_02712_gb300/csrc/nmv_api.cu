@@ -21,7 +21,7 @@ template <int DT>
 struct ScanOps {
   static cudaError_t prepare(int nin, size_t smem);
   static int occupancy(int nin, size_t smem);
-  static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
+  static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, bool pdl, const CaseDesc *cases,
                             const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,
                             int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
@@ -51,22 +51,22 @@ int scan_occupancy(int dt, int nin, size_t smem) {
   }
 }
 
-cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
+cudaError_t launch_scan(int dt, int nin, int grid, size_t smem, cudaStream_t st, bool pdl, const CaseDesc *cases,
                         const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
                         Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                         unsigned long long *stats, uint32_t *err) {
   switch (dt) {
     case NMV_F32:
-      return ScanOps<NMV_F32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
+      return ScanOps<NMV_F32>::launch(nin, grid, smem, st, pdl, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
     case NMV_F16:
-      return ScanOps<NMV_F16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
+      return ScanOps<NMV_F16>::launch(nin, grid, smem, st, pdl, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
     case NMV_BF16:
-      return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
+      return ScanOps<NMV_BF16>::launch(nin, grid, smem, st, pdl, cases, pieces, piece_ctr, n_pieces, piece_base,
                                        partials, batch_count, out, g_thr, stats, err);
     default:
-      return ScanOps<NMV_I32>::launch(nin, grid, smem, st, cases, pieces, piece_ctr, n_pieces, piece_base,
+      return ScanOps<NMV_I32>::launch(nin, grid, smem, st, pdl, cases, pieces, piece_ctr, n_pieces, piece_base,
                                       partials, batch_count, out, g_thr, stats, err);
   }
 }
@@ -813,7 +813,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   }
   for (size_t gi = 0; gi < groups.size(); ++gi) {
     const Group &G = groups[gi];
-    e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, d_cases, d_pieces + G.piece_base, d_ctr + gi,
+    e = launch_scan(G.dt, G.nin, G.grid, G.smem, st, gi > 0, d_cases, d_pieces + G.piece_base, d_ctr + gi,
                     (int64_t)G.plan.pieces.size(), G.piece_base, (Partial *)(W + o_part), (int32_t *)(W + o_segc),
                     W + o_out, (uint32_t *)(W + o_thr), d_stats, (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");
@@ -1064,7 +1064,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   const CaseDesc *d_case = (const CaseDesc *)W;
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   if (grid > 0) {
-    e = launch_scan(g.dt, nin, grid, smem, st, d_case, d_pieces, (unsigned long long *)(W + o_thr + 8), n_pieces, 0,
+    e = launch_scan(g.dt, nin, grid, smem, st, false, d_case, d_pieces, (unsigned long long *)(W + o_thr + 8), n_pieces, 0,
                     (Partial *)(W + o_part), (int32_t *)(W + o_segc), W + o_out, (uint32_t *)(W + o_thr), nullptr,
                     (uint32_t *)(W + o_out + kCallErrOff));
     if (e != cudaSuccess) return cuda_fail(e, "scan kernel launch");

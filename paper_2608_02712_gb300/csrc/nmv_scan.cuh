@@ -1790,6 +1790,11 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
     }
   }
+  // A later launch of a batch call (another element type) may run as this
+  // grid's programmatic dependent, overlapping its drain; each grid then
+  // ends only after the one before it, so the finalize kernel, which waits
+  // for the last, sees all of them (a no-op for a grid launched normally).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // Launch helpers of one element type (defined in nmv_scan_<dtype>.cu).  The
@@ -1799,7 +1804,7 @@ template <int DT>
 struct ScanOps {
   static cudaError_t prepare(int nin, size_t smem);
   static int occupancy(int nin, size_t smem);
-  static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases,
+  static cudaError_t launch(int nin, int grid, size_t smem, cudaStream_t st, bool pdl, const CaseDesc *cases,
                             const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces, int64_t piece_base,
                             Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr,
                             unsigned long long *stats, uint32_t *err);
@@ -1828,20 +1833,35 @@ struct ScanOps {
     return e == cudaSuccess ? n : 0;                                                                     \
   }                                                                                                      \
   template <>                                                                                            \
-  cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, const CaseDesc *cases, \
-                                  const Piece *pieces, unsigned long long *piece_ctr, int64_t n_pieces,  \
-                                  int64_t piece_base,                                                     \
-                                  Partial *partials, int32_t *batch_count, uint8_t *out, uint32_t *g_thr, \
+  cudaError_t ScanOps<DT>::launch(int nin, int grid, size_t smem, cudaStream_t st, bool pdl,             \
+                                  const CaseDesc *cases, const Piece *pieces, unsigned long long *piece_ctr, \
+                                  int64_t n_pieces, int64_t piece_base, Partial *partials,                \
+                                  int32_t *batch_count, uint8_t *out, uint32_t *g_thr,                    \
                                   unsigned long long *stats, uint32_t *err) {                            \
-    if (nin == 0)                                                                                        \
-      NMV_SCAN_FN(DT, 0)<<<grid, kThreads, NMV_SCAN_SMEM(0, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
-    else if (nin == 1)                                                                                   \
-      NMV_SCAN_FN(DT, 1)<<<grid, kThreads, NMV_SCAN_SMEM(1, smem), st>>>(                               \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
-    else                                                                                                 \
-      NMV_SCAN_FN(DT, -1)<<<grid, kThreads, NMV_SCAN_SMEM(-1, smem), st>>>(                              \
-          cases, pieces, piece_ctr, n_pieces, piece_base, partials, batch_count, out, g_thr, stats, err);        \
+    cudaLaunchConfig_t cfg = {};                                                                         \
+    cfg.gridDim = dim3(grid);                                                                            \
+    cfg.blockDim = dim3(kThreads);                                                                       \
+    cfg.stream = st;                                                                                     \
+    cudaLaunchAttribute attr[1];                                                                         \
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;                                     \
+    attr[0].val.programmaticStreamSerializationAllowed = 1;                                              \
+    cfg.attrs = attr;                                                                                    \
+    cfg.numAttrs = pdl ? 1 : 0;                                                                          \
+    cudaError_t e;                                                                                       \
+    if (nin == 0) {                                                                                      \
+      cfg.dynamicSmemBytes = NMV_SCAN_SMEM(0, smem);                                                     \
+      e = cudaLaunchKernelEx(&cfg, NMV_SCAN_FN(DT, 0), cases, pieces, piece_ctr, n_pieces, piece_base,   \
+                             partials, batch_count, out, g_thr, stats, err);                             \
+    } else if (nin == 1) {                                                                               \
+      cfg.dynamicSmemBytes = NMV_SCAN_SMEM(1, smem);                                                     \
+      e = cudaLaunchKernelEx(&cfg, NMV_SCAN_FN(DT, 1), cases, pieces, piece_ctr, n_pieces, piece_base,   \
+                             partials, batch_count, out, g_thr, stats, err);                             \
+    } else {                                                                                             \
+      cfg.dynamicSmemBytes = NMV_SCAN_SMEM(-1, smem);                                                    \
+      e = cudaLaunchKernelEx(&cfg, NMV_SCAN_FN(DT, -1), cases, pieces, piece_ctr, n_pieces, piece_base,  \
+                             partials, batch_count, out, g_thr, stats, err);                             \
+    }                                                                                                    \
+    if (e != cudaSuccess) return e;                                                                      \
     return cudaGetLastError();                                                                           \
   }
 
