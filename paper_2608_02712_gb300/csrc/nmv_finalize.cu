@@ -129,42 +129,23 @@ __device__ void publish_records(const FkView &F, int64_t pos0, int64_t n) {
   __syncwarp();  // the warp's record stores are visible to its lanes
   int64_t *hidx = (int64_t *)F.hrec;
   double *hc = (double *)(hidx + F.first_k), *hr = hc + F.first_k;
-  // four records per lane in flight: every load of a round before its stores
-  constexpr int U = 4;
-  for (int64_t t0 = threadIdx.x & 31; t0 < n; t0 += 32 * U) {
-    int64_t idx[U];
-    double cv[U], rv[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int64_t p = pos0 + t0 + 32 * u;
-      idx[u] = 0;
-      cv[u] = rv[u] = 0.0;
-      if (t0 + 32 * u < n) {
-        idx[u] = F.idx[p];
-        cv[u] = F.c64[p];
-        rv[u] = F.r64[p];
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (t0 + 32 * u >= n) break;
-      const int64_t p = pos0 + t0 + 32 * u;
-      int64_t i = idx[u];
-      hidx[p] = i;
-      hc[p] = cv[u];
-      hr[p] = rv[u];
-      if (F.coords) {
-        int64_t *c = F.coords + p * F.rank;
-        for (int d = F.rank - 1; d >= 0; --d) {
-          const Div64 sd = F.sdiv[d];
-          if (sd.d == 0) {
-            c[d] = 0;
-            i = 0;
-          } else {
-            const uint64_t q = div_q((uint64_t)i, sd.d, sd.m);
-            c[d] = i - (int64_t)(q * sd.d);
-            i = (int64_t)q;
-          }
+  for (int64_t t = threadIdx.x & 31; t < n; t += 32) {
+    const int64_t p = pos0 + t;
+    int64_t idx = F.idx[p];
+    hidx[p] = idx;
+    hc[p] = F.c64[p];
+    hr[p] = F.r64[p];
+    if (F.coords) {
+      int64_t *c = F.coords + p * F.rank;
+      for (int d = F.rank - 1; d >= 0; --d) {
+        const Div64 sd = F.sdiv[d];
+        if (sd.d == 0) {
+          c[d] = 0;
+          idx = 0;
+        } else {
+          const uint64_t q = div_q((uint64_t)idx, sd.d, sd.m);
+          c[d] = idx - (int64_t)(q * sd.d);
+          idx = (int64_t)q;
         }
       }
     }
