@@ -495,3 +495,20 @@ def test_indices_beyond_32_bits(shape):
     np.testing.assert_array_equal(got["row_prof"], rowp)
     np.testing.assert_array_equal(got["col_prof"], colp)
     assert got["flags"] == 16  # NMV_FLAG_REF_CONSTANT: the reference is all ones
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+def test_first_k_records_across_far_apart_pieces(dt):
+    """Records in a few batches far apart (first, middle, last, and a ragged
+    last batch), K larger than the mismatch count: the record pass skips the
+    runs of pieces without records and still places every record."""
+    n = (1 << 26) + 37
+    ref = torch.ones(n, dtype=dt)
+    cand = ref.clone()
+    where = [0, 1, 2, 31, 4097, n // 2, n // 2 + 1, n - 40, n - 2, n - 1]
+    for i in where:
+        cand[i] = 3.0
+    want = oracle.validate(cand, ref, rtol=1e-3, atol=0.0, tile=(1, 1024), first_k=64)
+    got = validate(cand.cuda(), ref.cuda(), rtol=1e-3, atol=0.0, tile=(1, 1024), first_k=64)
+    assert_same(got, want, "far-apart records %s" % dt)
+    np.testing.assert_array_equal(got["fk_index"], where)
