@@ -51,3 +51,26 @@ def test_max_over_ranks_and_job_value_gloo():
 def test_single_rank_is_identity():
     assert bench.max_over_ranks(3.25, 1, "cpu") == 3.25
     assert bench.job_gbs(537_000_000, 1, 1.0) == pytest.approx(537.0)
+
+
+def test_oracle_sample_units_and_bytes():
+    """The reference arm's bounded sample: rows of a single case (its inputs
+    cut to the same elements), whole cases of a batch."""
+    from paper_2608_02712_gb300 import workloads
+    single = [workloads.c5(shape=(64, 256), first_k=16)]
+    assert bench.sample_units(single) == 64
+    t, nbytes = bench.oracle_step_time(single, 8)
+    assert t > 0 and nbytes == 8 * 256 * 4 * 2
+    batch = [workloads.fuzz(s) for s in range(3)]
+    assert bench.sample_units(batch) == 3
+    t, nbytes = bench.oracle_step_time(batch, 2)
+    assert nbytes == sum(bench.case_bytes(c) for c in batch[:2])
+    assert "cases of the batch" in bench.sample_text(batch, 2, nbytes)
+
+
+def test_full_size_flags():
+    class A:
+        c2_batch, c5_rows, no_inputs = 8, 32768, False
+    assert bench.full_size(A)
+    A.c5_rows = 4096
+    assert not bench.full_size(A)
