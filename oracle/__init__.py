@@ -1,7 +1,7 @@
 """CPU oracle for numerical validation with failure forensics.
 
 TEST INFRASTRUCTURE ONLY: the test suite, ``__graft_entry__.smoke()`` and the
-CPU-baseline leg of ``bench.py`` are the only callers.  The product path (the
+CPU-baseline leg and reference arm of ``bench.py`` are the only callers.  The product path (the
 CUDA library and its binding in ``paper_2608_02712_gb300``) never imports this
 package, and this package imports nothing from it.
 

@@ -3,7 +3,7 @@
  * validation with failure forensics.
  *
  * TEST INFRASTRUCTURE ONLY.  Only the test suite, the smoke check and the
- * benchmark's CPU-baseline leg may load this library.  The product path
+ * benchmark's CPU-baseline leg and reference arm may load this library.  The product path
  * (the CUDA library and its Python binding) never calls it, includes it or
  * shares a line of code, a header or a table with it.
  *
