@@ -52,6 +52,11 @@ extern "C" {
 #define NMV_ECUDA (-3)        /* a CUDA call failed (no device, bad stream,
                                  a kernel error); see nmv_last_error()      */
 #define NMV_EUNSUPPORTED (-4) /* the device is not sm_103                   */
+#define NMV_ETIMEOUT (-5)     /* a kernel gave up waiting (its bulk copies into
+                                 shared memory did not complete within its
+                                 2 s wait limit); the call's results are void,
+                                 nothing stays allocated and the CUDA context
+                                 remains usable                             */
 
 /* ---- element types ----------------------------------------------------- */
 typedef enum nmv_dtype {
@@ -139,6 +144,10 @@ typedef struct nmv_result {
     int32_t n_inputs;
     int32_t passthrough_input;  /* lowest input that raised CAND_EQ_INPUT, or -1 */
     int64_t *input_eq;          /* [n_inputs]; -1 for an input of another dtype or numel */
+    /* The numerical match rate of full-coverage evaluation (Section 4.3,
+     * Table S4 "x% matched cases" per case): (numel - mismatch) / numel,
+     * one fp64 division of the two exact integers; 1.0 when numel == 0.    */
+    double match_fraction;
 } nmv_result;
 
 /* Validate one case on `cuda_stream` (a cudaStream_t; NULL = the legacy
@@ -194,7 +203,8 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
  * before any stream capture.  All calls share the one array and find the
  * previous call's contents in it; each call clears what must start at zero.
  * Calls made through this library are serialised by its lock and return
- * only after their stream work has finished; calls that did overlap on the
+ * only after their stream work has finished, also when they fail; calls
+ * that did overlap on the
  * GPU would race on the array.  Profiling (nmv_profile_enable) does not
  * apply to this entry point.  On error *out's scalar fields are unspecified.
  */
@@ -243,6 +253,11 @@ typedef struct nmv_profile {
     int64_t dense_steps;       /* warp steps that only counted and localised
                                   mismatches (no maximum candidates)         */
     int64_t dense_cycles;      /* SM clock cycles warps spent in those steps */
+    int64_t workspace_allocs;  /* device workspace allocations on this device
+                                  since the library was loaded (the workspace
+                                  grows by doubling, so a rising sequence of
+                                  case sizes allocates O(log n) times)       */
+    int64_t workspace_bytes;   /* the device workspace's current size        */
 } nmv_profile;
 
 void nmv_profile_enable(int mode);

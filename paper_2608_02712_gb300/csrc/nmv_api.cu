@@ -104,6 +104,7 @@ struct DeviceState {
   size_t smem_set[4][3] = {};  // dynamic smem opted in per kernel instantiation
   void *ws = nullptr;
   size_t ws_size = 0;
+  int64_t ws_allocs = 0;  // workspace allocations so far (nmv_profile.workspace_allocs)
   void *pinned = nullptr;
   size_t pinned_size = 0;
 };
@@ -135,6 +136,13 @@ float f32_up(double x) {
 }
 
 bool valid_dtype(int32_t dt) { return dt >= NMV_F32 && dt <= NMV_I32; }
+
+// The numerical match rate (Section 4.3, Table S4): matching elements over
+// all elements, one rounding of the exact integer quotient; 1.0 for an
+// empty case.
+double match_fraction(int64_t numel, int64_t mismatch) {
+  return numel == 0 ? 1.0 : (double)(numel - mismatch) / (double)numel;
+}
 
 // numel of a tensor, or -1 if its shape is invalid.
 int64_t tensor_numel(const nmv_tensor &t) {
@@ -251,10 +259,13 @@ int probe_device(int *dev_out, DeviceState **st_out) {
 int ensure_workspace(DeviceState &s, size_t ws, size_t pinned) {
   if (injected("alloc")) return fail(NMV_ENOMEM, "injected allocation failure");
   if (ws > s.ws_size) {
+    // grow geometrically, so a rising sequence of case sizes reallocates
+    // O(log n) times
+    const size_t want = std::max(ws, s.ws_size * 2);
     if (s.ws) cudaFree(s.ws);
     s.ws = nullptr;
     s.ws_size = 0;
-    size_t want = std::max(ws, s.ws_size * 2);
+    ++s.ws_allocs;
     cudaError_t e = cudaMalloc(&s.ws, want);
     if (e != cudaSuccess) {
       cudaGetLastError();
@@ -264,10 +275,10 @@ int ensure_workspace(DeviceState &s, size_t ws, size_t pinned) {
     s.ws_size = want;
   }
   if (pinned > s.pinned_size) {
+    const size_t want = std::max(pinned, s.pinned_size * 2);
     if (s.pinned) cudaFreeHost(s.pinned);
     s.pinned = nullptr;
     s.pinned_size = 0;
-    size_t want = std::max(pinned, s.pinned_size * 2);
     cudaError_t e = cudaHostAlloc(&s.pinned, want, cudaHostAllocDefault);
     if (e != cudaSuccess) {
       cudaGetLastError();
@@ -768,6 +779,19 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     dHO = (uint8_t *)dp + res_bytes;
   }
 
+  // From the first enqueue on, an error return waits for the work already
+  // queued (status ignored), so the next call, perhaps on another stream,
+  // does not race with it on the workspace.
+  struct DrainOnError {
+    cudaStream_t st;
+    bool armed = true;
+    ~DrainOnError() {
+      if (armed) {
+        cudaStreamSynchronize(st);
+        cudaGetLastError();
+      }
+    }
+  } drain{st};
   cudaError_t e = cudaSuccess;
   const bool upload = C.uploaded_ws != S->ws;
   if (upload) {
@@ -827,7 +851,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   if (injected("d2h")) return fail(NMV_ECUDA, "injected copy-back failure");
   if (*(const uint32_t *)(HO + kCallErrOff) != 0)
-    return fail(NMV_ECUDA, "scan kernel: a bulk copy into shared memory did not complete in time");
+    return fail(NMV_ETIMEOUT, "scan kernel: a bulk copy into shared memory did not complete in time");
   // Cases whose differences are all tiny (max |d| < 2^-38): the fp32 squares
   // of the scan pass may have lost terms, so their SSE is recomputed in fp64.
   for (int64_t i = 0; i < n; ++i) {
@@ -860,6 +884,8 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     P.light_cycles = (int64_t)st4[6];
     P.dense_steps = (int64_t)st4[7];
     P.dense_cycles = (int64_t)st4[8];
+    P.workspace_allocs = S->ws_allocs;
+    P.workspace_bytes = (int64_t)S->ws_size;
     g_prof.valid = true;
   }
 
@@ -906,8 +932,10 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     r.n_inputs = c.n_inputs;
     r.passthrough_input = oh->passthrough;
     r.input_eq = oh->input_eq;
+    r.match_fraction = match_fraction(g.numel, r.mismatch);
   }
   guard.p = nullptr;  // handed to the caller
+  drain.armed = false;
   C.zeroed_ws = S->ws;
   *out = res;
   g_err.clear();
@@ -1051,6 +1079,20 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   }
 
   // ---- upload, clear, launch
+  // From the first enqueue on, an error return first waits for the work
+  // already queued on the stream (its status ignored): the header promises
+  // that a call's stream work has finished when it returns, and a later call
+  // on another stream would otherwise race with it on the shared scratch.
+  struct DrainOnError {
+    cudaStream_t st;
+    bool armed = true;
+    ~DrainOnError() {
+      if (armed) {
+        cudaStreamSynchronize(st);
+        cudaGetLastError();
+      }
+    }
+  } drain{st};
   cudaError_t e = cudaMemcpyAsync(W, &g_na_desc, sizeof(CaseDesc), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess && n_pieces > 0)
     e = cudaMemcpyAsync(W + sz_cases, g_na_pieces, sizeof(Piece) * (size_t)n_pieces, cudaMemcpyHostToDevice, st);
@@ -1078,7 +1120,7 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   if (e == cudaSuccess) e = cudaMemcpyAsync(&kerr, W + o_out + kCallErrOff, 4, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(st);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (result header)");
-  if (kerr != 0) return fail(NMV_ECUDA, "scan kernel: a bulk copy into shared memory did not complete in time");
+  if (kerr != 0) return fail(NMV_ETIMEOUT, "scan kernel: a bulk copy into shared memory did not complete in time");
   if (g_na_head.max_abs > 0.0 && g_na_head.max_abs < 0x1p-38) {
     // the fp64 SSE re-pass for cases whose differences are all tiny
     double *dst = (double *)(W + o_out + kCallHeader + offsetof(OutHeader, sse));
@@ -1140,6 +1182,8 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
   out->n_inputs = c->n_inputs;
   out->passthrough_input = oh.passthrough;
   for (int j = 0; j < c->n_inputs; ++j) out->input_eq[j] = oh.input_eq[j];
+  out->match_fraction = match_fraction(g.numel, out->mismatch);
+  drain.armed = false;  // the last synchronize above covered every copy
   g_err.clear();
   return NMV_OK;
 }
@@ -1171,6 +1215,7 @@ const char *nmv_status_string(int status) {
     case NMV_ENOMEM: return "out of memory";
     case NMV_ECUDA: return "CUDA error";
     case NMV_EUNSUPPORTED: return "unsupported device";
+    case NMV_ETIMEOUT: return "kernel wait limit reached";
     default: return "unknown status";
   }
 }

@@ -17,7 +17,7 @@ import torch
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libnmv.so")
 
-NMV_OK, NMV_EINVAL, NMV_ENOMEM, NMV_ECUDA, NMV_EUNSUPPORTED = 0, -1, -2, -3, -4
+NMV_OK, NMV_EINVAL, NMV_ENOMEM, NMV_ECUDA, NMV_EUNSUPPORTED, NMV_ETIMEOUT = 0, -1, -2, -3, -4, -5
 MAX_RANK, MAX_INPUTS = 8, 8
 DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2, torch.int32: 3}
 FLAGS = {"CAND_EQ_INPUT": 1, "CAND_ALL_ZERO": 2, "CAND_CONSTANT": 4,
@@ -40,7 +40,8 @@ class Profile(ctypes.Structure):
                 ("exact_abs", ctypes.c_int64), ("exact_rel", ctypes.c_int64),
                 ("exact_pred", ctypes.c_int64), ("slow_cycles", ctypes.c_int64),
                 ("light_cycles", ctypes.c_int64), ("dense_steps", ctypes.c_int64),
-                ("dense_cycles", ctypes.c_int64)]
+                ("dense_cycles", ctypes.c_int64), ("workspace_allocs", ctypes.c_int64),
+                ("workspace_bytes", ctypes.c_int64)]
 
 
 class Case(ctypes.Structure):
@@ -66,7 +67,7 @@ class Result(ctypes.Structure):
                 ("col_prof", _i64p), ("k_out", ctypes.c_int64), ("fk_index", _i64p),
                 ("fk_coords", _i64p), ("fk_cand", _f64p), ("fk_ref", _f64p),
                 ("n_inputs", ctypes.c_int32), ("passthrough_input", ctypes.c_int32),
-                ("input_eq", _i64p)]
+                ("input_eq", _i64p), ("match_fraction", ctypes.c_double)]
 
 
 _lock = threading.Lock()
@@ -169,7 +170,7 @@ def result_to_dict(r: Result) -> dict:
     k = int(r.k_out)
     return {
         "pass": bool(r.pass_), "numel": numel, "rank": int(r.rank), "mismatch": mismatch,
-        "match_fraction": 1.0 if numel == 0 else (numel - mismatch) / numel,
+        "match_fraction": float(r.match_fraction),
         "cand_nan": int(r.cand_nan), "cand_posinf": int(r.cand_posinf),
         "cand_neginf": int(r.cand_neginf), "ref_nan": int(r.ref_nan),
         "ref_posinf": int(r.ref_posinf), "ref_neginf": int(r.ref_neginf),

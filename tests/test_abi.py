@@ -76,7 +76,20 @@ def test_status_strings(lib):
     assert lib.nmv_status_string(0) == b"ok"
     assert lib.nmv_status_string(-1) == b"invalid argument"
     assert lib.nmv_status_string(-3) == b"CUDA error"
+    assert lib.nmv_status_string(-4) == b"unsupported device"
+    assert lib.nmv_status_string(-5) == b"kernel wait limit reached"
     assert lib.nmv_status_string(12345) == b"unknown status"
+
+
+def test_status_codes_match_header():
+    from paper_2608_02712_gb300 import nmv
+    text = open(HEADER).read()
+    codes = {m.group(1): int(m.group(2)) for m in
+             re.finditer(r"#define (NMV_E\w+|NMV_OK) \(?(-?\d+)\)?", text)}
+    assert codes == {"NMV_OK": 0, "NMV_EINVAL": -1, "NMV_ENOMEM": -2, "NMV_ECUDA": -3,
+                     "NMV_EUNSUPPORTED": -4, "NMV_ETIMEOUT": -5}
+    for name, v in codes.items():
+        assert getattr(nmv, name) == v, name
 
 
 def _host_case(nmv, n=16, dtype=0, **over):

@@ -512,3 +512,27 @@ def test_first_k_records_across_far_apart_pieces(dt):
     got = validate(cand.cuda(), ref.cuda(), rtol=1e-3, atol=0.0, tile=(1, 1024), first_k=64)
     assert_same(got, want, "far-apart records %s" % dt)
     np.testing.assert_array_equal(got["fk_index"], where)
+
+
+def test_workspace_grows_geometrically():
+    """A rising sequence of case sizes (each 10% above the last, 40 calls)
+    reallocates the device workspace O(log n) times: it grows by doubling."""
+    from paper_2608_02712_gb300 import nmv as m
+    m.profile_enable(m.PROFILE_TIMING)
+    try:
+        allocs, sizes = [], []
+        n = 100_000
+        for _ in range(40):
+            x = torch.zeros(n, device="cuda")
+            # one-element tiles: the histogram (8 bytes per element) dominates
+            validate(x, x, rtol=0.0, atol=0.0, tile=(1, 1), first_k=0)
+            p = m.profile_last()
+            allocs.append(p["workspace_allocs"])
+            sizes.append(p["workspace_bytes"])
+            n = int(n * 1.1)
+    finally:
+        m.profile_enable(0)
+    assert all(b >= a for a, b in zip(sizes, sizes[1:]))
+    grew = allocs[-1] - allocs[0]
+    # 1.1^40 = 45x: at most ceil(log2(45)) + 1 = 7 doublings
+    assert grew <= 7, (grew, allocs)
