@@ -314,3 +314,132 @@ def fuzz(seed: int, device="cpu", max_dim: int = 300, allow_empty: bool = True):
     tw = int(torch.randint(1, 70, (1,), generator=g))
     k = int(torch.randint(0, 300, (1,), generator=g))
     return _case("fuzz_%d" % seed, cand, ref, rtol, atol, (th, tw), k, inputs)
+
+
+# Tolerances at the edges of the scan's fp32 proofs: rtol around 1/4 and
+# 1/2 (the exactness and pre-filter limits), atol from 0 up past 2^100.
+EDGE_RTOL = (0.0, 0.25, 0.5, math.nextafter(0.5, 1.0), 2.0)
+EDGE_ATOL = (0.0, 1e-50, 2.0 ** 100, 2.0 ** 101, 1e300)
+EDGE_FAMILIES = ("tolerance", "sterbenz", "subnormal", "big_tiles", "global_hist", "large")
+
+
+def _bits_of(t: torch.Tensor) -> torch.Tensor:
+    return t.contiguous().view(_INT_VIEW[t.dtype]).to(torch.int64)
+
+
+def _from_bits(b: torch.Tensor, dt) -> torch.Tensor:
+    width = 32 if dt == torch.float32 else 16
+    b = b & ((1 << width) - 1)
+    b = torch.where(b >= (1 << (width - 1)), b - (1 << width), b)
+    return b.to(_INT_VIEW[dt]).view(dt)
+
+
+def _ulp_step(t: torch.Tensor, k: torch.Tensor) -> torch.Tensor:
+    """Move each element k[i] representable values up (k > 0) or down, in
+    the order of the real line (through zero)."""
+    width = 32 if t.dtype == torch.float32 else 16
+    b = _bits_of(t) & ((1 << width) - 1)
+    sign = b >> (width - 1)
+    mag = b & ((1 << (width - 1)) - 1)
+    key = torch.where(sign == 1, -mag, mag)          # ordered integer key (-0 -> 0)
+    key = key + k
+    nb = torch.where(key < 0, (1 << (width - 1)) | (-key), key)
+    return _from_bits(nb, t.dtype).reshape(t.shape)
+
+
+def edge(seed: int, device="cpu"):
+    """One case at an edge of the fast path's proofs or of the launch plan,
+    by family (seed % 6):
+
+    * tolerance: rtol in {0, 1/4, 1/2, the double after 1/2, 2} and atol in
+      {0, 1e-50, 2^100, 2^101, 1e300} (the pre-filter is off above rtol 1/2
+      or atol 2^100);
+    * sterbenz: differences planted at |c - r| = |r|/4 and 1-2 values either
+      side (c near 5r/4 and 3r/4), where c - r stops being provably exact;
+    * subnormal: references (and candidates) in the subnormal range of the
+      type, a few representable values apart;
+    * big_tiles: row or column tiles above 4096 (profiles not privatised in
+      shared memory);
+    * global_hist: a tile grid wider than the shared-memory histogram window
+      (8192 bins), with mismatches;
+    * large: 2-6 million elements, so the case spans many pieces and blocks.
+    """
+    g = torch.Generator().manual_seed(50_000 + seed)
+    gd = _gen(60_000 + seed, device)
+    fam = EDGE_FAMILIES[seed % len(EDGE_FAMILIES)]
+    floats = (torch.float32, torch.float16, torch.bfloat16)
+    pick = lambda seq: seq[int(torch.randint(0, len(seq), (1,), generator=g))]
+    dt = pick(floats)
+    rtol, atol = DEFAULT_TOL[dt]
+    tile = (int(torch.randint(1, 70, (1,), generator=g)), int(torch.randint(1, 70, (1,), generator=g)))
+    k = int(torch.randint(0, 600, (1,), generator=g))
+    if fam == "big_tiles":
+        m, n = pick(((300, 10000), (5001, 600), (700, 4099)))
+        tile = pick(((5000, 10000), (4097, 64), (64, 4097), (m, n), (4096, 4096)))
+    elif fam == "global_hist":
+        m, n = pick(((40, 100000), (20, 65536 + 3), (2000, 3000)))
+        tile = pick(((1, 8), (1, 1), (2, 4)))
+    elif fam == "large":
+        numel = int(torch.randint(2_000_000, 6_000_000, (1,), generator=g))
+        n = pick((1, 7, 4096, 4099, 65536))
+        m = max(1, numel // n)
+        dt = pick(floats + (torch.int32,))
+        k = int(torch.randint(0, 5000, (1,), generator=g))
+    else:
+        m = int(torch.randint(1, 600, (1,), generator=g))
+        n = int(torch.randint(1, 3000, (1,), generator=g))
+    shape = (m, n)
+    if dt == torch.int32:
+        ref = torch.randint(-(1 << 20), 1 << 20, shape, generator=gd, device=device, dtype=torch.int32)
+        cand = ref.clone()
+        hit = torch.rand(shape, generator=gd, device=device) < 0.01
+        cand = torch.where(hit, cand + torch.randint(-2, 3, shape, generator=gd, device=device,
+                                                     dtype=torch.int32), cand)
+        rtol, atol = pick(((0.0, 0.0), (1e-6, 1.0), (0.5, 0.0)))
+        return _case("edge_%d_%s_int32" % (seed, fam), cand, ref, rtol, atol, tile, k)
+
+    x = torch.randn(shape, generator=gd, device=device)
+    if fam == "subnormal":
+        width = 32 if dt == torch.float32 else 16
+        mant = (1 << 23) if dt == torch.float32 else (1 << 10 if dt == torch.float16 else 1 << 7)
+        mag = torch.randint(0, mant, shape, generator=gd, device=device, dtype=torch.int64)
+        sgn = torch.randint(0, 2, shape, generator=gd, device=device, dtype=torch.int64)
+        ref = _from_bits((sgn << (width - 1)) | mag, dt).reshape(shape)
+        steps = torch.randint(-3, 4, shape, generator=gd, device=device, dtype=torch.int64)
+        steps = torch.where(torch.rand(shape, generator=gd, device=device) < 0.7, 0 * steps, steps)
+        cand = _ulp_step(ref, steps)
+        atol = pick((0.0, 1e-50, 1e-45, 6e-8, 1e-40, 1e-39))
+        rtol = pick((0.0, rtol, 0.25, 0.5))
+    else:
+        ref = (x * 10.0 ** float(torch.randint(-2, 3, (1,), generator=g))).to(dt)
+        if fam == "tolerance":
+            rtol, atol = pick(EDGE_RTOL), pick(EDGE_ATOL)
+            rel = torch.randn(shape, generator=gd, device=device) * pick((1e-3, 0.3, 1.0, 3.0))
+            cand = (ref.float() * (1.0 + rel)).to(dt)
+        elif fam == "sterbenz":
+            rtol = pick((0.2, 0.25, 0.3, 0.5, math.nextafter(0.5, 1.0)))
+            atol = pick((0.0, 1e-8, 1e-3))
+            f = torch.where(torch.rand(shape, generator=gd, device=device) < 0.5,
+                            torch.full(shape, 1.25, device=device), torch.full(shape, 0.75, device=device))
+            near = (ref.double() * f.double()).to(dt)
+            steps = torch.randint(-2, 3, shape, generator=gd, device=device, dtype=torch.int64)
+            near = _ulp_step(near, steps)
+            noisy = (ref.float() * (1.0 + torch.randn(shape, generator=gd, device=device) * 1e-3)).to(dt)
+            cand = torch.where(torch.rand(shape, generator=gd, device=device) < 0.3, near, noisy)
+        else:
+            rel = torch.randn(shape, generator=gd, device=device) * rtol * 2.0
+            cand = (ref.float() * (1.0 + rel)).to(dt)
+            if fam == "global_hist":
+                band = torch.rand(shape, generator=gd, device=device) < 0.2
+                cand = torch.where(band, (cand.float() + 1.0).to(dt), cand)
+            elif fam == "large":
+                r0 = int(torch.randint(0, m, (1,), generator=g))
+                cand.view(m, n)[r0: r0 + max(1, m // 50)] += 1
+    cf, rf = cand.view(-1), ref.view(-1)
+    nsp = int(torch.randint(0, 9, (1,), generator=g))
+    sp = SPECIALS[dt]
+    for _ in range(nsp):
+        p = int(torch.randint(0, cf.numel(), (1,), generator=g))
+        cf[p] = sp[int(torch.randint(0, len(sp), (1,), generator=g))]
+    return _case("edge_%d_%s_%s_%dx%d" % (seed, fam, str(dt).split(".")[-1], m, n), cand, ref,
+                 rtol, atol, tile, k)

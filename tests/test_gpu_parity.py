@@ -321,60 +321,17 @@ def test_max_rel_closest_fractions_16bit(dt, order):
     assert got["argmax_rel"] == {"larger_late": late, "larger_first": 1, "ties_only": 3}[order]
 
 
-def _props_fp32(c, r, x, rtol, atol, th, tw, chunk_rows=2048):
-    """Whole-tensor properties of an fp32 [M, N] pair with one input, from
-    torch's fp64 elementwise ops (the predicate with its two roundings, no
-    fusion), in chunks of rows: counts, maxima with their first indices,
-    the SSE and the localisation maps."""
-    M, N = c.shape
-    out = {"mismatch": 0, "sse": 0.0, "max_abs": -1.0, "argmax_abs": -1, "max_rel": -1.0,
-           "argmax_rel": -1, "eq": 0}
-    hist = torch.zeros(-(-M // th), -(-N // tw), dtype=torch.int64, device=c.device)
-    rowp = torch.zeros(th, dtype=torch.int64, device=c.device)
-    colp = torch.zeros(tw, dtype=torch.int64, device=c.device)
-    xv = x.view(M, N)
-    for r0 in range(0, M, chunk_rows):
-        r1 = min(M, r0 + chunk_rows)
-        cc, rr = c[r0:r1].double(), r[r0:r1].double()
-        fin = torch.isfinite(cc) & torch.isfinite(rr)
-        d = (cc - rr).abs()
-        ok = (cc == rr) | (fin & (d <= atol + rtol * rr.abs()))
-        mis = ~ok
-        out["mismatch"] += int(mis.sum())
-        d = torch.where(fin, d, torch.full_like(d, -1.0))
-        out["sse"] += float(torch.where(fin, (cc - rr) * (cc - rr), torch.zeros_like(d)).sum())
-        m = float(d.max())
-        if m > out["max_abs"]:
-            out["max_abs"], out["argmax_abs"] = m, r0 * N + int(torch.nonzero(d.view(-1) == m)[0])
-        rel = torch.where(fin & (rr != 0), d / rr.abs(), torch.full_like(d, -1.0))
-        m = float(rel.max())
-        if m > out["max_rel"]:
-            out["max_rel"], out["argmax_rel"] = m, r0 * N + int(torch.nonzero(rel.view(-1) == m)[0])
-        cb, rb, xb = (t.view(torch.int32) for t in (c[r0:r1], r[r0:r1], xv[r0:r1]))
-        out["eq"] += int(((cb == xb) & (rb != xb)).sum())
-        mi = mis.to(torch.int64)
-        rows = torch.arange(r0, r1, device=c.device)
-        rowp.index_add_(0, rows % th, mi.sum(1))
-        colp.index_add_(0, torch.arange(N, device=c.device) % tw, mi.sum(0))
-        hist.index_add_(0, rows // th, torch.zeros(r1 - r0, hist.shape[1], dtype=torch.int64,
-                                                   device=c.device).index_add_(
-            1, torch.arange(N, device=c.device) // tw, mi))
-        del cc, rr, fin, d, ok, mis, rel, mi
-    out["hist"], out["rowp"], out["colp"] = hist.cpu().numpy(), rowp.cpu().numpy(), colp.cpu().numpy()
-    return out
-
-
 def test_c5_full_size():
     """C5 at its full size (fp32 [32768, 65536] plus a 2^31-element input,
-    24 GiB), in the launch configuration the benchmark times: the oracle on
-    the records' prefix and on two sampled tile rows, the planted closed
-    forms, and whole-tensor properties from independent fp64 arithmetic."""
+    24 GiB), in the launch configuration the benchmark times, against one
+    oracle pass over the whole tensors: every field, element by element,
+    plus run-to-run bit identity and the planted closed forms."""
     free, _ = torch.cuda.mem_get_info()
     if free < (64 << 30):
         pytest.skip("needs 64 GiB of free device memory")
     case = workloads.c5(device="cuda")
     c, r, x = case["cand"], case["ref"], case["inputs"][0]
-    rtol, atol, (th, tw), K = case["rtol"], case["atol"], case["tile"], case["first_k"]
+    K = case["first_k"]
     got = _gpu(case)
     again = _gpu(case)
     for k in got:
@@ -383,38 +340,15 @@ def test_c5_full_size():
             assert a.dtype == b.dtype and np.array_equal(a.view(np.uint8), b.view(np.uint8)), k
         else:
             assert a == b, k
-    M, N = c.shape
     # planted closed forms: 2147 distinct special positions, the first 1074 NaN
     assert got["cand_nan"] == 1074 and got["cand_neginf"] == 1073 and got["cand_posinf"] == 0
     assert got["ref_nan"] == got["ref_posinf"] == got["ref_neginf"] == 0
     assert got["flags"] & 1 and got["passthrough_input"] == 0  # NMV_FLAG_CAND_EQ_INPUT
     assert got["k_out"] == K
-    # the oracle on the prefix that holds the first K records
-    end = int(got["fk_index"][-1]) + 1
-    cf, rf, xf = c.view(-1), r.view(-1), x.view(-1)
-    pre = oracle.validate(cf[:end].cpu(), rf[:end].cpu(), inputs=[xf[:end].cpu()], rtol=rtol,
-                          atol=atol, tile=(1, tw), first_k=K)
-    assert pre["mismatch"] == K
-    np.testing.assert_array_equal(got["fk_index"], pre["fk_index"])
-    np.testing.assert_array_equal(got["fk_cand"].view(np.int64), pre["fk_cand"].view(np.int64))
-    np.testing.assert_array_equal(got["fk_ref"].view(np.int64), pre["fk_ref"].view(np.int64))
-    np.testing.assert_array_equal(got["fk_coords"], np.stack(np.unravel_index(got["fk_index"], (M, N)), 1))
-    # the oracle on two whole tile rows: one in the pass-through half, one in the noisy half
-    for t in (3, 200):
-        rows = slice(t * th, (t + 1) * th)
-        sub = oracle.validate(c[rows].cpu(), r[rows].cpu(), inputs=[x.view(M, N)[rows].reshape(-1).cpu()],
-                              rtol=rtol, atol=atol, tile=(th, tw), first_k=0)
-        np.testing.assert_array_equal(got["tile_hist"][t], sub["tile_hist"][0])
-    # whole-tensor properties
-    p = _props_fp32(c, r, x, rtol, atol, th, tw)
-    assert got["mismatch"] == p["mismatch"]
-    assert got["input_eq"][0] == p["eq"]
-    assert got["max_abs"] == p["max_abs"] and got["argmax_abs"] == p["argmax_abs"]
-    assert got["max_rel"] == p["max_rel"] and got["argmax_rel"] == p["argmax_rel"]
-    assert abs(got["sse"] - p["sse"]) <= 1e-9 * p["sse"]
-    np.testing.assert_array_equal(got["tile_hist"], p["hist"])
-    np.testing.assert_array_equal(got["row_prof"], p["rowp"])
-    np.testing.assert_array_equal(got["col_prof"], p["colp"])
+    host = dict(case, cand=c.cpu(), ref=r.cpu(), inputs=[x.cpu()])
+    del c, r, x, case
+    want = _oracle(host)
+    assert_same(got, want, host["name"])
 
 
 def test_concurrent_calls_from_threads():
