@@ -73,6 +73,9 @@ def _bind(path: str):
         fn.argtypes = [ctypes.c_uint32]
     lib.oracle_pass.restype = ctypes.c_int
     lib.oracle_pass.argtypes = [ctypes.c_double] * 4
+    lib.oracle_stats.restype = ctypes.c_int
+    lib.oracle_stats.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
+                                 ctypes.c_int64, ctypes.c_int64, i64p, f64p, i64p, i64p, f64p]
     return lib
 
 
@@ -104,6 +107,9 @@ class Oracle:
 
     def validate_batch(self, cases):
         return _validate_batch(self.validate, cases)
+
+    def stats(self, x, **kw):
+        return _stats(self.lib, x, **kw)
 
 
 def _decode(lib, bits: int, dtype: torch.dtype) -> float:
@@ -235,3 +241,47 @@ def _validate_batch(fn, cases) -> dict:
 def validate_batch(cases) -> dict:
     """P7: each case validated independently; the batch pass count is the sum."""
     return _validate_batch(validate, cases)
+
+
+STAT_COUNTS = ("n_finite", "n_nan", "n_posinf", "n_neginf", "n_zero")
+STAT_VALUES = ("min", "max", "sum", "sumsq", "mean", "std")
+
+
+def _stat_dict(cnt, f):
+    d = {k: int(v) for k, v in zip(STAT_COUNTS, cnt)}
+    d.update({k: float(v) for k, v in zip(STAT_VALUES, f)})
+    return d
+
+
+def stats(x: torch.Tensor, *, tile=(64, 64)) -> dict:
+    """Diagnostic tensor statistics of one CPU tensor (see oracle_stats in
+    nmv_oracle.c): the whole tensor, and every tile of the [M, N] view."""
+    return _stats(_load(), x, tile=tile)
+
+
+def _stats(lib, x: torch.Tensor, *, tile=(64, 64)) -> dict:
+    if x.dtype not in DTYPE_CODES:
+        raise ValueError("unsupported dtype %s" % x.dtype)
+    x = x.detach().cpu().contiguous()
+    shape = tuple(x.shape)
+    numel = x.numel()
+    m, n = view_2d(shape)
+    th, tw = int(tile[0]), int(tile[1])
+    gr = -(-m // th) if numel else 0
+    gc = -(-n // tw) if numel else 0
+    counts = np.zeros(5, np.int64)
+    f = np.zeros(6, np.float64)
+    first = np.zeros(2, np.int64)
+    tcnt = np.zeros(max(gr * gc, 1) * 5, np.int64)
+    tf = np.zeros(max(gr * gc, 1) * 6, np.float64)
+    rc = lib.oracle_stats(ctypes.c_void_p(x.data_ptr()), DTYPE_CODES[x.dtype], numel, max(n, 1),
+                          th, tw, _ptr(counts, ctypes.c_int64), _ptr(f, ctypes.c_double),
+                          _ptr(first, ctypes.c_int64), _ptr(tcnt, ctypes.c_int64),
+                          _ptr(tf, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments")
+    tiles = {k: tcnt[i:gr * gc * 5:5].reshape(gr, gc).copy() for i, k in enumerate(STAT_COUNTS)}
+    tiles.update({k: tf[i:gr * gc * 6:6].reshape(gr, gc).copy() for i, k in enumerate(STAT_VALUES)})
+    return {"numel": numel, "rank": len(shape), "all": _stat_dict(counts, f),
+            "first_nan": int(first[0]), "first_inf": int(first[1]),
+            "grid_rows": gr, "grid_cols": gc, "tile_rows": th, "tile_cols": tw, "tiles": tiles}

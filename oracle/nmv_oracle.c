@@ -306,3 +306,152 @@ int oracle_validate(const void *cand, const void *ref, int dtype, int64_t numel,
     passthrough[0] = pt;
     return 0;
 }
+
+/*
+ * ---- diagnostic tensor statistics (the instrumentation probe) -----------
+ *
+ * The engine's diagnostic instrumentation (Section 4.2, "Diagnostic
+ * instrumentation"; Figure 3 bottom-left; S5.1 "tensor-statistic
+ * instrumentation") records multi-level tensor statistics at pipeline
+ * boundaries so that diffuse precision failures can be localised.  The paper
+ * gives no list of statistics and no formula; the reading written out here:
+ *
+ *   levels: the whole tensor, and every tile of the same [M, N] view and
+ *           tile grid as the localisation maps (P4);
+ *   per level, over its elements x_i (widened to fp64 exactly):
+ *     n_finite, n_nan, n_posinf, n_neginf   class counts (int32: all finite)
+ *     n_zero                                #{x_i == 0 by value} (+0 and -0)
+ *     min, max                              over the finite x_i (0.0 if none)
+ *     sum   = sum of the finite x_i
+ *     sumsq = sum of x_i^2 over the finite x_i
+ *     mean  = sum / n_finite                (0.0 if n_finite == 0)
+ *     std   = sqrt(max(0, sumsq / n_finite - mean^2))   (0.0 if none)
+ *             (the population standard deviation written with the two
+ *             sums; each operation one fp64 rounding)
+ *   tensor level only: first_nan / first_inf = the lowest index holding a
+ *           NaN / an infinity of either sign, -1 if none.
+ *
+ * Sums: int32 elements are summed exactly (integers; x^2 in 128 bits) and
+ * rounded once to fp64; float elements with Neumaier's compensated
+ * summation in index order.
+ *
+ * Output layout: stat[11] = {n_finite, n_nan, n_posinf, n_neginf, n_zero}
+ * as int64 in counts[5] and {min, max, sum, sumsq, mean, std} as fp64 in
+ * f[6]; tile t (row-major on the tile grid) at counts + 5 t, f + 6 t.
+ */
+static void or_stat_finish(const int64_t *cnt, double *f)
+{
+    double n = (double)cnt[0];
+    if (cnt[0] == 0) {
+        f[0] = f[1] = f[2] = f[3] = f[4] = f[5] = 0.0;
+        return;
+    }
+    double mean = f[2] / n;
+    double ex2 = f[3] / n;
+    double var = ex2 - mean * mean;
+    f[4] = mean;
+    f[5] = var > 0.0 ? sqrt(var) : 0.0;
+}
+
+typedef struct {
+    int64_t cnt[5];
+    double mn, mx;
+    int have;
+    /* float sums: Neumaier (running value + correction) */
+    double s, sc, q, qc;
+    /* int32 sums: exact */
+    __int128 is, iq;
+} or_acc;
+
+static void or_acc_init(or_acc *a)
+{
+    memset(a, 0, sizeof(*a));
+}
+
+static void neumaier(double *sum, double *comp, double term)
+{
+    double t = *sum + term;
+    if (fabs(*sum) >= fabs(term)) *comp += (*sum - t) + term;
+    else *comp += (term - t) + *sum;
+    *sum = t;
+}
+
+static void or_acc_add(or_acc *a, uint32_t bits, int dtype)
+{
+    if (dtype == OR_I32) {
+        int64_t v = (int64_t)(int32_t)bits;
+        a->cnt[0]++;
+        if (v == 0) a->cnt[4]++;
+        double d = (double)v;
+        if (!a->have || d < a->mn) a->mn = d;
+        if (!a->have || d > a->mx) a->mx = d;
+        a->have = 1;
+        a->is += v;
+        a->iq += (__int128)(v * v);
+        return;
+    }
+    double x = decode(bits, dtype);
+    if (isnan(x)) { a->cnt[1]++; return; }
+    if (isinf(x)) { if (x > 0) a->cnt[2]++; else a->cnt[3]++; return; }
+    a->cnt[0]++;
+    if (x == 0.0) a->cnt[4]++;
+    if (!a->have || x < a->mn) a->mn = x;
+    if (!a->have || x > a->mx) a->mx = x;
+    a->have = 1;
+    neumaier(&a->s, &a->sc, x);
+    neumaier(&a->q, &a->qc, x * x);
+}
+
+static void or_acc_out(const or_acc *a, int dtype, int64_t *cnt, double *f)
+{
+    for (int k = 0; k < 5; ++k) cnt[k] = a->cnt[k];
+    f[0] = a->have ? a->mn : 0.0;
+    f[1] = a->have ? a->mx : 0.0;
+    if (dtype == OR_I32) {
+        f[2] = (double)a->is;   /* one rounding of the exact integer */
+        f[3] = (double)a->iq;
+    } else {
+        f[2] = a->s + a->sc;
+        f[3] = a->q + a->qc;
+    }
+    or_stat_finish(cnt, f);
+}
+
+int oracle_stats(const void *x, int dtype, int64_t numel, int64_t ncols, int64_t tile_rows,
+                 int64_t tile_cols, int64_t *counts, double *f, int64_t *first,
+                 int64_t *tile_counts, double *tile_f)
+{
+    if (ncols < 1 || tile_rows < 1 || tile_cols < 1 || numel < 0) return -1;
+    int64_t nrows = numel / ncols;
+    int64_t gr = numel ? (nrows + tile_rows - 1) / tile_rows : 0;
+    int64_t gc = numel ? (ncols + tile_cols - 1) / tile_cols : 0;
+    or_acc all;
+    or_acc_init(&all);
+    int64_t first_nan = -1, first_inf = -1;
+    /* whole tensor, in index order */
+    for (int64_t i = 0; i < numel; ++i) {
+        uint32_t b = load_bits(x, dtype, i);
+        or_acc_add(&all, b, dtype);
+        if (dtype != OR_I32) {
+            double v = decode(b, dtype);
+            if (isnan(v) && first_nan < 0) first_nan = i;
+            if (isinf(v) && first_inf < 0) first_inf = i;
+        }
+    }
+    or_acc_out(&all, dtype, counts, f);
+    first[0] = first_nan;
+    first[1] = first_inf;
+    /* every tile, its elements in index order */
+    for (int64_t tr = 0; tr < gr; ++tr) {
+        for (int64_t tc = 0; tc < gc; ++tc) {
+            or_acc a;
+            or_acc_init(&a);
+            for (int64_t r = tr * tile_rows; r < nrows && r < (tr + 1) * tile_rows; ++r)
+                for (int64_t c = tc * tile_cols; c < ncols && c < (tc + 1) * tile_cols; ++c)
+                    or_acc_add(&a, load_bits(x, dtype, r * ncols + c), dtype);
+            int64_t t = tr * gc + tc;
+            or_acc_out(&a, dtype, tile_counts + 5 * t, tile_f + 6 * t);
+        }
+    }
+    return 0;
+}

@@ -451,6 +451,15 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.m32N = d.idx32 ? 0xffffffffu / (uint32_t)d.N : 0u;
   d.m32th = 0xffffffffu / (uint32_t)d.th;
   d.m32tw = 0xffffffffu / (uint32_t)d.tw;
+  {
+    const int64_t step = 32 * (int64_t)g.vec;  // elements of one warp step
+    d.amode = 0;
+    d.a_shift = 0;
+    if (d.idx32 && g.numel > 0 && d.N % step == 0 && step % d.tw == 0 && d.tw % g.vec == 0) {
+      d.amode = 1;
+      while ((int64_t)g.vec << d.a_shift < d.tw) ++d.a_shift;
+    }
+  }
   d.rtol = c.rtol;
   d.atol = c.atol;
   // fp32 pre-filter coefficients (margins of 2^-20; see nmv_scan.cuh)

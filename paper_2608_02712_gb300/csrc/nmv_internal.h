@@ -73,6 +73,13 @@ struct CaseDesc {
   int64_t out_off;                     // byte offset of this case's packed result
   int64_t hist_off, rowp_off, colp_off, fk_off;  // byte offsets inside the packed result
   int64_t hist_n, rowp_n, colp_n;      // entries of the histogram and the profiles
+  // Aligned localisation (amode != 0): indices fit in 32 bits, N is a
+  // multiple of the warp step (32 vec_elems elements), and the tile width
+  // divides the warp step and is a multiple of vec_elems.  A warp step then
+  // lies in one row, and lane l's elements lie in one tile column at column
+  // offsets (l mod 2^a_shift) * vec_elems + k, with 2^a_shift = tw /
+  // vec_elems lanes per tile.
+  int32_t amode, a_shift;
   // the candidate's shape as divisors, for the records' coordinates
   // (written at byte coord_off of the host result when the finalize writes
   // there; a zero extent has d = 0)

@@ -293,6 +293,7 @@ struct PieceSh {
   uint32_t *g_thr;
   uint32_t *cta_thr;  // [2] the block's view of the case-wide maxima (float bits), in shared memory
   int32_t *sh_eq;  // [kThreads][NMV_MAX_INPUTS] pass-through counts of the exact paths (inputs only)
+  uint32_t lcol_sa;  // shared address of the lanes' private column counters ([kThreads][V], aligned mode)
   unsigned long long *stats;  // [exact steps, exact abs, exact rel, exact predicate, light steps,
                               //  SM cycles in exact steps, SM cycles in light steps,
                               //  dense steps, SM cycles in dense steps]
@@ -630,6 +631,61 @@ __device__ __forceinline__ void record_step(const PieceSh *P, WarpSh *W, uint32_
   if (mask) record_lane(P, mask, row, col, tr, rp, tc, cp);
 }
 
+// Localisation and the batch's mismatch count for one step of a case with
+// aligned geometry (CaseDesc::amode): the step (32 V elements from s0, a
+// multiple of the step) lies in one row, and lane l's elements lie in tile
+// column (s0 mod N) / tw + (l >> a_shift) at column offsets
+// (l mod 2^a_shift) V + k.  Every lane computes the row and tile from s0
+// alike (no vote), the first lane of each tile adds the tile's count to its
+// histogram bin, lane 0 adds the step's count to the row bin, and each lane
+// adds its column bits to its private counters in shared memory, which are
+// added to the column profile at the end of the piece.
+template <int V>
+__device__ __forceinline__ void record_step_aligned(const PieceSh *P, WarpSh *W, uint32_t mask, int64_t idx0) {
+  const int lane = threadIdx.x & 31;
+  const int cnt = __popc(mask);
+  const int total = __reduce_add_sync(0xffffffffu, (unsigned)cnt);
+  if (total == 0) return;
+  const CaseDesc &cd = P->cd;
+  const uint32_t N = (uint32_t)cd.dN.d, th = (uint32_t)cd.dth.d, tw = (uint32_t)cd.dtw.d;
+  const uint32_t s0 = (uint32_t)idx0 - (uint32_t)(lane * V);
+  const uint32_t row = div_q32(s0, N, cd.m32N);
+  const uint32_t col0 = s0 - row * N;
+  const uint32_t tr = div_q32(row, th, cd.m32th);
+  const uint32_t rp = row - tr * th;
+  const int sh = cd.a_shift;
+  const uint32_t tc = div_q32(col0, tw, cd.m32tw) + (uint32_t)(lane >> sh);
+  int gsum = cnt;
+  if (sh == 5) {
+    gsum = total;
+  } else {
+    for (int o = 1; o < (1 << sh); o <<= 1) gsum += __shfl_xor_sync(0xffffffffu, gsum, o);
+  }
+  if (gsum != 0 && (lane & ((1 << sh) - 1)) == 0) {
+    if (P->wr > 0) sh_add(&P->sh_hist[((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0)], gsum);
+    else gl_add(&P->g_hist[(int64_t)tr * cd.GC + tc], (unsigned long long)gsum);
+  }
+  if (lane == 0) {
+    if (P->prof_smem) sh_add(&P->sh_row[rp], total);
+    else gl_add(&P->g_row[rp], (unsigned long long)total);
+    W->mism += total;
+    W->sbits |= 1u << (((s0 - (uint32_t)P->pbegin) >> (V == 8 ? 8 : 7)) & (batch_steps(nin_class_of(cd.n_elig)) - 1));
+  }
+  if (mask) {
+    const uint32_t a = P->lcol_sa + (uint32_t)threadIdx.x * (V * 4);
+#pragma unroll
+    for (int j = 0; j < V; j += 4) {
+      int x, y, z, w;
+      asm volatile("ld.shared.v4.s32 {%0,%1,%2,%3}, [%4];" : "=r"(x), "=r"(y), "=r"(z), "=r"(w) : "r"(a + 4 * j));
+      x += (mask >> j) & 1u;
+      y += (mask >> (j + 1)) & 1u;
+      z += (mask >> (j + 2)) & 1u;
+      w += (mask >> (j + 3)) & 1u;
+      asm volatile("st.shared.v4.s32 [%0], {%1,%2,%3,%4};" ::"r"(a + 4 * j), "r"(x), "r"(y), "r"(z), "r"(w));
+    }
+  }
+}
+
 // The general case of record_step for one lane: walk its mismatches from
 // the coordinates of its first element, merging runs of equal bins.
 static __device__ __noinline__ void record_lane(const PieceSh *P, uint32_t mask, uint64_t row, uint64_t col,
@@ -880,7 +936,10 @@ __device__ __noinline__ SseAcc slow_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     if (kA >= 0) changed |= offer_abs(L, bA, xA, aA, idx0 + kA);
     if (kR >= 0) changed |= offer_rel(L, bRn, bRd, xR, aR, rR, bRq, idx0 + kR, n_rel);
   }
-  if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0, V);
+  if (__any_sync(0xffffffffu, mask != 0)) {
+    if (P->cd.amode) record_step_aligned<V>(P, W, mask, idx0);
+    else record_step(P, W, mask, idx0, V);
+  }
   if (__any_sync(0xffffffffu, changed)) refresh(P, L, W);
   if (P->stats) count_stats(W, 0, t_start, n_abs, n_rel, n_pred);
   return sse;
@@ -973,6 +1032,8 @@ __device__ __noinline__ SseAcc light_step(const PieceSh *P, LaneSh *L, WarpSh *W
 //    here; the SSE terms take the exact path's arithmetic (c - r as s + e by
 //    TwoSum, d^2 = p + pe + 2se), so the result does not depend on which path
 //    an element took;
+//  * a light step when every element provably passes, is finite and has an
+//    exact fp32 difference (only candidates for a maximum);
 //  * otherwise the exact step.
 template <int DT>
 __device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W, uint4 cv, uint4 rv,
@@ -1011,7 +1072,22 @@ __device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
     if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
   }
-  if (!__all_sync(0xffffffffu, dense)) return slow_step<DT>(P, L, W, cv, rv, idx0, V, sse);
+  if (!__all_sync(0xffffffffu, dense)) {
+    // Light or exact: a light step needs every element provably passing,
+    // finite and exact in fp32 (|s| <= min(fma_rz(lo_r, |r|, lo_a), |r|/4);
+    // the finite cap keeps infinities out).
+    bool other = false;
+#pragma unroll
+    for (int j = 0; j < V / 2; ++j) {
+      const float2 r2 = make_float2(vdec<DT>(rv, 2 * j), vdec<DT>(rv, 2 * j + 1));
+      const float2 ar2 = make_float2(fabsf(r2.x), fabsf(r2.y));
+      const float2 a2 = __ffma2_rz(ar2, lo_r2, lo_a2);
+      other |= !(fabsf(s[j].x) <= min3f(a2.x, __fmul_rz(0.25f, ar2.x), kHuge));
+      other |= !(fabsf(s[j].y) <= min3f(a2.y, __fmul_rz(0.25f, ar2.y), kHuge));
+    }
+    if (__any_sync(0xffffffffu, other)) return slow_step<DT>(P, L, W, cv, rv, idx0, V, sse);
+    return light_step<DT>(P, L, W, cv, rv, idx0, sse);
+  }
 #pragma unroll
   for (int j = 0; j < V / 2; ++j) {
     const float2 p = __fmul2_rn(s[j], s[j]);
@@ -1024,7 +1100,10 @@ __device__ __noinline__ SseAcc hard_step(const PieceSh *P, LaneSh *L, WarpSh *W,
     sse.lo = __fadd2_rn(sse.lo, __fadd2_rn(err, q));
     sse.hi = t;
   }
-  if (__any_sync(0xffffffffu, mask != 0)) record_step(P, W, mask, idx0, V);
+  if (__any_sync(0xffffffffu, mask != 0)) {
+    if (P->cd.amode) record_step_aligned<V>(P, W, mask, idx0);
+    else record_step(P, W, mask, idx0, V);
+  }
   if (P->stats) count_stats(W, 2, t_start, 0, 0, 0);
   return sse;
 }
@@ -1219,23 +1298,13 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
       for (int k = 0; k < V; k += 2) ff_pair<Tr<DT>::EB == 4>(R.sse, make_float2(s[k], s[k + 1]));
       return;
     }
-    // Which steps need more than a maximum update (a mismatch, a non-finite
-    // value, an inexact c - r, an undecided predicate; the finite cap keeps
-    // infinities out of the light path).
-    other = false;
-#pragma unroll
-    for (int k = 0; k < V; ++k) {
-      const float rf = vdec<DT>(rv, k);
-      const float a = __fmaf_rz(R.lo_r, fabsf(rf), R.lo_a);
-      other |= !(fabsf(s[k]) <= min3f(a, __fmul_rz(0.25f, fabsf(rf)), kHuge));
-    }
+    // dense, light or exact: decided out of line
+    R.sse = hard_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
+    reload_thr(R, W);
+    return;
   }
-  if (__any_sync(0xffffffffu, other)) {
-    if constexpr (Tr<DT>::kInt) R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
-    else R.sse = hard_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
-  } else {
-    R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
-  }
+  if (__any_sync(0xffffffffu, other)) R.sse = slow_step<DT>(P, L, W, cv, rv, P->pbegin + erel, V, R.sse);
+  else R.sse = light_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
   reload_thr(R, W);
 }
 
@@ -1523,6 +1592,8 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ Partial red[kWarps];
   __shared__ int32_t sh_eq[NIN != 0 ? kThreads * NMV_MAX_INPUTS : 1];
   __shared__ __align__(8) uint32_t cta_thr[2];
+  // each lane's column counters of an aligned case (record_step_aligned)
+  __shared__ __align__(16) int32_t lcol[kThreads * Tr<DT>::V];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   LaneSh *L = &lanes[threadIdx.x];
   WarpSh *W = &warps[warp];
@@ -1573,6 +1644,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         P.g_thr = g_thr + 2 * pc.case_id;
         P.sh_cls = smem;
         P.sh_eq = sh_eq;
+        P.lcol_sa = smem_addr(lcol);
         P.cta_thr = cta_thr;
         P.stats = stats;
         // the block's view starts from what the case has published so far
@@ -1634,6 +1706,10 @@ __global__ void __launch_bounds__(kThreads, 2)
     L->r_lo = -1.f;
     L->cacc = 0;
     L->racc = 0;
+    if (P.cd.amode) {
+#pragma unroll
+      for (int k = 0; k < Tr<DT>::V; ++k) lcol[threadIdx.x * Tr<DT>::V + k] = 0;
+    }
     if constexpr (NIN != 0) {
       for (int j = 0; j < NMV_MAX_INPUTS; ++j) sh_eq[threadIdx.x * NMV_MAX_INPUTS + j] = 0;
     }
@@ -1674,6 +1750,19 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
     sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
+    if (P.cd.amode) {
+      // this lane's column counters into the column profile
+      constexpr int V = Tr<DT>::V;
+      const int cp0 = (lane & ((1 << P.cd.a_shift) - 1)) * V;
+#pragma unroll
+      for (int k = 0; k < V; ++k) {
+        const int v = lcol[threadIdx.x * V + k];
+        if (v) {
+          if (P.prof_smem) sh_add(&P.sh_col[cp0 + k], v);
+          else gl_add(&P.g_col[cp0 + k], (unsigned long long)v);
+        }
+      }
+    }
     __syncwarp();
     if (lane == 0 && atomicAdd(&sh_done, 1) == 0) {
       // the first warp done claims the block's next piece

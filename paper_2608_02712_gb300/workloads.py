@@ -443,3 +443,42 @@ def edge(seed: int, device="cpu"):
         cf[p] = sp[int(torch.randint(0, len(sp), (1,), generator=g))]
     return _case("edge_%d_%s_%s_%dx%d" % (seed, fam, str(dt).split(".")[-1], m, n), cand, ref,
                  rtol, atol, tile, k)
+
+
+def stats_fuzz(seed: int, device="cpu", max_dim: int = 200):
+    """One random tensor for the diagnostic statistics: rank 0-4, any of the
+    four dtypes, values of a random scale and offset, sprinkled NaN/Inf and
+    zeros, a random tile.  Returns (tensor, tile)."""
+    g = torch.Generator().manual_seed(70_000 + seed)
+    gd = _gen(80_000 + seed, device)
+    dtypes = (torch.float32, torch.float16, torch.bfloat16, torch.int32)
+    dt = dtypes[int(torch.randint(0, 4, (1,), generator=g))]
+    rank = int(torch.randint(0, 5, (1,), generator=g))
+    shape, budget = [], 1 << 16
+    for _ in range(rank):
+        d = int(torch.randint(1, max(2, min(max_dim, budget)) + 1, (1,), generator=g))
+        if float(torch.rand(1, generator=g)) < 0.03:
+            d = 0
+        shape.append(d)
+        budget = max(1, budget // max(d, 1))
+    shape = tuple(shape)
+    if dt == torch.int32:
+        hi = (1 << 31) - 1 if float(torch.rand(1, generator=g)) < 0.5 else 1000
+        x = torch.randint(-hi, hi, shape, generator=gd, device=device, dtype=torch.int32)
+    else:
+        scale = 10.0 ** float(torch.randint(-3, 4, (1,), generator=g))
+        offset = float(torch.randn(1, generator=g)) * scale * 5
+        x = (torch.randn(shape, generator=gd, device=device) * scale + offset).to(dt)
+        n = x.numel()
+        if n:
+            ns = int(torch.randint(0, min(n, 16) + 1, (1,), generator=g))
+            pos = torch.randint(0, n, (ns,), generator=g).tolist()
+            sp = SPECIALS[dt]
+            which = torch.randint(0, len(sp), (ns,), generator=g).tolist()
+            xf = x.view(-1)
+            for p, w in zip(pos, which):
+                xf[p] = sp[w]
+    if x.numel() and float(torch.rand(1, generator=g)) < 0.3:
+        x.view(-1)[torch.rand(x.numel(), generator=gd, device=device) < 0.2] = 0
+    tile = (int(torch.randint(1, 70, (1,), generator=g)), int(torch.randint(1, 70, (1,), generator=g)))
+    return x, tile

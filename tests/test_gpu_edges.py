@@ -6,6 +6,8 @@ subnormal references; tiles above the shared-memory profile size; tile grids
 wider than the shared-memory histogram window; cases of millions of
 elements.  Each case is compared with the oracle field by field, alone, in
 one mixed batch, and through buffers that are not 16-byte aligned."""
+import zlib
+
 import pytest
 import torch
 
@@ -48,3 +50,55 @@ def test_edge_parity_unaligned(seed):
     got = validate(c, r, rtol=case["rtol"], atol=case["atol"], tile=case["tile"],
                    first_k=case["first_k"])
     assert_same(got, _oracle(case), case["name"] + " (unaligned)")
+
+
+def _aligned_case(dt, tw, th, n_steps, pattern, seed):
+    """A case whose last dimension is a multiple of the warp step (32 x 16
+    bytes) and whose tile width divides the step: the scan's aligned
+    localisation path."""
+    v = 8 if dt in (torch.float16, torch.bfloat16) else 4
+    n = 32 * v * n_steps
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    m = int(torch.randint(50, 400, (1,), generator=g, device="cuda"))
+    if dt == torch.int32:
+        ref = torch.randint(-1000, 1000, (m, n), generator=g, device="cuda", dtype=torch.int32)
+        wrong = ref + 1
+    else:
+        ref = torch.randn(m, n, generator=g, device="cuda").to(dt)
+        wrong = (ref.float() + 1.0).to(dt)
+    if pattern == "dense":
+        sel = torch.rand(m, n, generator=g, device="cuda") < 0.9
+    elif pattern == "sparse":
+        sel = torch.rand(m, n, generator=g, device="cuda") < 0.003
+    else:  # a band of columns in every other row
+        sel = torch.zeros(m, n, dtype=torch.bool, device="cuda")
+        sel[::2, n // 3: n // 3 + 40] = True
+    cand = torch.where(sel, wrong, ref)
+    rtol, atol = (0.0, 0.0) if dt == torch.int32 else (1e-2, 1e-3)
+    return cand, ref, rtol, atol
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.float16, torch.bfloat16, torch.int32],
+                         ids=["f32", "f16", "bf16", "i32"])
+@pytest.mark.parametrize("tw_mult", [1, 2, 8, 32])
+@pytest.mark.parametrize("th", [1, 7, 64, 5000])
+@pytest.mark.parametrize("pattern", ["dense", "sparse", "band"])
+def test_aligned_localisation(dt, tw_mult, th, pattern):
+    v = 8 if dt in (torch.float16, torch.bfloat16) else 4
+    tw = v * tw_mult
+    seed = zlib.crc32(("%s %d %d %s" % (dt, tw_mult, th, pattern)).encode()) % 10_000
+    cand, ref, rtol, atol = _aligned_case(dt, tw, th, 1 + seed % 5, pattern, seed)
+    got = validate(cand, ref, rtol=rtol, atol=atol, tile=(th, tw), first_k=300)
+    want = oracle.validate(cand.cpu(), ref.cpu(), rtol=rtol, atol=atol, tile=(th, tw), first_k=300)
+    assert_same(got, want, "aligned %s tw=%d th=%d %s" % (dt, tw, th, pattern))
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+def test_aligned_localisation_wide_grid(dt):
+    """Aligned steps whose tile grid is wider than the shared-memory
+    histogram window: the histogram goes to global memory."""
+    v = 8 if dt == torch.bfloat16 else 4
+    cand, ref, rtol, atol = _aligned_case(dt, v, 3, 300, "dense", 77)   # N / tw = 9600 tile columns
+    got = validate(cand, ref, rtol=rtol, atol=atol, tile=(3, v), first_k=50)
+    want = oracle.validate(cand.cpu(), ref.cpu(), rtol=rtol, atol=atol, tile=(3, v), first_k=50)
+    assert_same(got, want, "aligned wide grid %s" % dt)

@@ -14,6 +14,7 @@ import test_oracle_closed_forms as tc
 import test_oracle_decoders as td
 import test_oracle_golden as tg
 import test_oracle_predicate as tp
+import test_oracle_stats as ts
 from _golden import fixture_files
 
 SRC = os.path.join(os.path.dirname(oracle.__file__), "nmv_oracle.c")
@@ -42,6 +43,23 @@ MUTATIONS = {
     "all_zero_by_bits": ("if (!(c == 0.0)) cand_all_zero = 0;", "if (cb != 0) cand_all_zero = 0;"),
     "threshold_floor": ("int64_t threshold = (numel + 99) / 100;", "int64_t threshold = numel / 100;"),
     "first_k_one_short": ("if (k_out < first_k) {", "if (k_out + 1 < first_k) {"),
+    # diagnostic tensor statistics
+    "stats_negative_zero_not_zero": ("if (x == 0.0) a->cnt[4]++;", "if (bits == 0) a->cnt[4]++;"),
+    "stats_infinities_counted_finite": (
+        "if (isinf(x)) { if (x > 0) a->cnt[2]++; else a->cnt[3]++; return; }",
+        "if (isinf(x)) { if (x > 0) a->cnt[2]++; else a->cnt[3]++; }"),
+    "stats_sample_variance": ("double var = ex2 - mean * mean;",
+                              "double var = (ex2 - mean * mean) * n / (n - 1.0);"),
+    "stats_tile_transposed": ("int64_t t = tr * gc + tc;", "int64_t t = tc * gr + tr;"),
+    "stats_sum_uncompensated": ("f[2] = a->s + a->sc;", "f[2] = a->s;"),
+    "stats_int_square_in_32_bits": ("a->iq += (__int128)(v * v);",
+                                    "a->iq += (__int128)(int32_t)((int32_t)v * (int32_t)v);"),
+    "stats_first_inf_takes_nan": ("if (isinf(v) && first_inf < 0) first_inf = i;",
+                                  "if (!isfinite(v) && first_inf < 0) first_inf = i;"),
+    "stats_tile_row_overlap": ("r < nrows && r < (tr + 1) * tile_rows; ++r)",
+                               "r < nrows && r <= (tr + 1) * tile_rows; ++r)"),
+    "stats_min_includes_first_zero": ("if (!a->have || x < a->mn) a->mn = x;",
+                                      "if (x < a->mn) a->mn = x;"),
 }
 
 
@@ -58,6 +76,12 @@ def _pins(orc):
     yield lambda: tc.test_c1_closed_form(orc)
     yield lambda: td.test_decode_f16_exhaustive(orc)
     yield lambda: td.test_decode_bf16_exhaustive(orc)
+    yield lambda: [ts.test_stats_fuzz_against_brute_force(orc, s) for s in range(60)]
+    yield lambda: [ts.test_stats_arithmetic_sequence(orc, dt) for dt in (torch.int32, torch.float32)]
+    yield lambda: ts.test_stats_constant_and_specials(orc)
+    yield lambda: ts.test_stats_int32_sums_are_exact(orc)
+    yield lambda: ts.test_stats_float_sums_are_compensated(orc)
+    yield lambda: ts.test_stats_empty_and_rank0(orc)
 
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
