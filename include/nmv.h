@@ -212,10 +212,67 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
 
 int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out);
 
-/* Release what one nmv_validate / nmv_validate_batch call returned.  NULL
- * is accepted.  (The block is mapped pinned host memory, which the library
+/* ---- diagnostic tensor statistics ---------------------------------------
+ * The engine's diagnostic instrumentation (Section 4.2, "Diagnostic
+ * instrumentation"; Figure 3, bottom-left; S5.1): when a repair attempt fails
+ * on diffuse numerical deviation, the engine records multi-level tensor
+ * statistics of the buffers at the kernel's pipeline boundaries and re-runs
+ * forensics.  The paper gives no list of statistics; this library's reading:
+ * two levels, the whole tensor and every tile of the same [M, N] view and
+ * tile grid as the localisation maps, each with the statistics of nmv_stat.
+ * One call instruments n buffers (one per boundary).
+ *
+ * Values are widened to fp64 exactly.  Counts, min, max, first_nan and
+ * first_inf are exact.  int32 sums are exact integers rounded once to fp64,
+ * so every int32 field is bit-identical to that definition.  Float sums
+ * are accumulated in float-float pairs and fp64 and lie within 1e-12 of
+ * the sum of |x| (sum) and relative 1e-12 (sumsq) of the exact sums; mean
+ * and std are computed from them as stated in nmv_stat.  Results are
+ * bit-identical from run to run. */
+#define NMV_MAX_STAT_TILES (1LL << 22)  /* grid_rows * grid_cols per buffer  */
+
+typedef struct nmv_stats_case {
+    nmv_tensor x;               /* the buffer (borrowed, device-readable)    */
+    int64_t tile_rows;          /* tile of the [M, N] view, 1 .. NMV_MAX_TILE */
+    int64_t tile_cols;
+} nmv_stats_case;
+
+/* Statistics of one region (the tensor, or one tile), over its elements x:
+ * every element is finite for int32.  With no finite element, min, max,
+ * sum, sumsq, mean and std are 0.0. */
+typedef struct nmv_stat {
+    int64_t n_finite, n_nan, n_posinf, n_neginf;
+    int64_t n_zero;             /* x == 0 by value (+0 and -0)              */
+    double min, max;            /* over the finite x                        */
+    double sum, sumsq;          /* sum of x and of x^2 over the finite x    */
+    double mean;                /* sum / n_finite                            */
+    double std;                 /* sqrt(max(0, sumsq / n_finite - mean^2)),
+                                   each operation one fp64 rounding          */
+} nmv_stat;
+
+typedef struct nmv_stats_result {
+    int32_t status;             /* NMV_OK                                   */
+    int32_t rank;
+    int64_t numel;
+    nmv_stat all;               /* the whole tensor                         */
+    int64_t first_nan;          /* lowest index of a NaN, or -1             */
+    int64_t first_inf;          /* lowest index of +-Inf, or -1             */
+    int64_t grid_rows, grid_cols;   /* ceil(M/tile_rows), ceil(N/tile_cols); 0 when numel == 0 */
+    int64_t tile_rows, tile_cols;
+    nmv_stat *tiles;            /* [grid_rows * grid_cols] row-major        */
+} nmv_stats_result;
+
+/* Statistics of n buffers on `cuda_stream`, synchronous like nmv_validate.
+ * Every case is checked first (the message names a bad case's index).  On
+ * NMV_OK, *out points to an array of n results released by ONE
+ * nmv_result_free(*out) call; on error *out is NULL and nothing stays
+ * allocated. */
+int nmv_stats(const nmv_stats_case *cases, int64_t n, void *cuda_stream, nmv_stats_result **out);
+
+/* Release what one nmv_validate / nmv_validate_batch / nmv_stats call
+ * returned.  NULL is accepted.  (The block is mapped pinned host memory, which the library
  * keeps for reuse by later calls.) */
-void nmv_result_free(nmv_result *r);
+void nmv_result_free(void *r);
 
 /* Static text for a status code. */
 const char *nmv_status_string(int status);

@@ -1199,6 +1199,27 @@ int run_noalloc(const nmv_case *c, void *stream, nmv_result *out) {
 
 }  // namespace
 
+// ---- host services shared with the other entry points of the library
+// (declared in nmv_internal.h)
+namespace nmv {
+int host_fail(int code, const std::string &msg) { return fail(code, msg); }
+int host_cuda_fail(cudaError_t e, const char *what) { return cuda_fail(e, what); }
+void host_clear_error() { g_err.clear(); }
+std::mutex &host_mutex() { return g_mu; }
+int host_probe(int *dev, int *sms, size_t *smem_optin) {
+  DeviceState *S = nullptr;
+  const int rc = probe_device(dev, &S);
+  if (rc) return rc;
+  *sms = S->sms;
+  *smem_optin = S->smem_optin;
+  return NMV_OK;
+}
+int64_t host_tensor_numel(const nmv_tensor &t) { return tensor_numel(t); }
+void *host_arena_get(size_t bytes) { return arena_get(bytes); }
+void host_arena_put(void *p) { arena_put(p); }
+bool host_injected(const char *step) { return injected(step); }
+}  // namespace nmv
+
 extern "C" {
 
 int nmv_validate(const nmv_case *c, void *cuda_stream, nmv_result **out) {
@@ -1215,7 +1236,7 @@ int nmv_validate_noalloc(const nmv_case *c, void *cuda_stream, nmv_result *out) 
   return run_noalloc(c, cuda_stream, out);
 }
 
-void nmv_result_free(nmv_result *r) { arena_put(r); }
+void nmv_result_free(void *r) { arena_put(r); }
 
 const char *nmv_status_string(int status) {
   switch (status) {

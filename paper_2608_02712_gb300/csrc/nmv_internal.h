@@ -2,8 +2,12 @@
 // the kernels (nmv_scan.cuh, nmv_finalize.cu).  Not part of the public ABI.
 #pragma once
 
+#include <cuda_runtime.h>
+
 #include <cstddef>
 #include <cstdint>
+#include <mutex>
+#include <string>
 
 #include "../../include/nmv.h"
 
@@ -186,5 +190,18 @@ NMV_CHD int ring_streams(int nin) { return nin == 1 ? 3 : 2; }
 NMV_CHD size_t ring_bytes(int nin) {
   return (size_t)kWarps * ring_stages(nin) * ((size_t)ring_streams(nin) * stage_bytes(nin) + 8);
 }
+
+// Host services of nmv_api.cu used by the library's other entry points: the
+// thread-local error text (nmv_last_error), the library lock, the device
+// probe (sm_103 only), and the pool of mapped pinned result blocks.
+int host_fail(int code, const std::string &msg);
+int host_cuda_fail(cudaError_t e, const char *what);
+void host_clear_error();
+std::mutex &host_mutex();
+int host_probe(int *dev, int *sms, size_t *smem_optin);  // call with host_mutex() held
+int64_t host_tensor_numel(const nmv_tensor &t);          // -1 for an invalid shape
+void *host_arena_get(size_t bytes);                      // mapped pinned block, or NULL
+void host_arena_put(void *p);
+bool host_injected(const char *step);                    // NMV_FAULT_INJECT test hook
 
 }  // namespace nmv

@@ -70,6 +70,26 @@ class Result(ctypes.Structure):
                 ("input_eq", _i64p), ("match_fraction", ctypes.c_double)]
 
 
+class StatsCase(ctypes.Structure):
+    _fields_ = [("x", Tensor), ("tile_rows", ctypes.c_int64), ("tile_cols", ctypes.c_int64)]
+
+
+STAT_COUNTS = ("n_finite", "n_nan", "n_posinf", "n_neginf", "n_zero")
+STAT_VALUES = ("min", "max", "sum", "sumsq", "mean", "std")
+
+
+class Stat(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_int64) for k in STAT_COUNTS] + [(k, ctypes.c_double) for k in STAT_VALUES]
+
+
+class StatsResult(ctypes.Structure):
+    _fields_ = [("status", ctypes.c_int32), ("rank", ctypes.c_int32), ("numel", ctypes.c_int64),
+                ("all", Stat), ("first_nan", ctypes.c_int64), ("first_inf", ctypes.c_int64),
+                ("grid_rows", ctypes.c_int64), ("grid_cols", ctypes.c_int64),
+                ("tile_rows", ctypes.c_int64), ("tile_cols", ctypes.c_int64),
+                ("tiles", ctypes.POINTER(Stat))]
+
+
 _lock = threading.Lock()
 _lib = None
 
@@ -92,7 +112,10 @@ def load() -> ctypes.CDLL:
                                                ctypes.c_void_p,
                                                ctypes.POINTER(ctypes.POINTER(Result))]
             lib.nmv_result_free.restype = None
-            lib.nmv_result_free.argtypes = [ctypes.POINTER(Result)]
+            lib.nmv_result_free.argtypes = [ctypes.c_void_p]
+            lib.nmv_stats.restype = ctypes.c_int
+            lib.nmv_stats.argtypes = [ctypes.POINTER(StatsCase), ctypes.c_int64, ctypes.c_void_p,
+                                      ctypes.POINTER(ctypes.POINTER(StatsResult))]
             lib.nmv_status_string.restype = ctypes.c_char_p
             lib.nmv_status_string.argtypes = [ctypes.c_int]
             lib.nmv_last_error.restype = ctypes.c_char_p
@@ -308,6 +331,59 @@ class Prepared:
             return [result_to_dict(self.out[i]) for i in range(self.n)]
         finally:
             self.lib.nmv_result_free(self.out)
+
+
+def _stat_dict(st: Stat) -> dict:
+    return {k: getattr(st, k) for k, _ in Stat._fields_}
+
+
+def stats_result_to_dict(r: StatsResult) -> dict:
+    gr, gc = int(r.grid_rows), int(r.grid_cols)
+    n = gr * gc
+    tiles = {}
+    if n:
+        raw = np.ctypeslib.as_array(ctypes.cast(r.tiles, ctypes.POINTER(ctypes.c_uint8)),
+                                    shape=(n * ctypes.sizeof(Stat),)).copy()
+        rec = raw.view(np.dtype([(k, np.int64) for k in STAT_COUNTS] +
+                                [(k, np.float64) for k in STAT_VALUES]))
+        tiles = {k: rec[k].reshape(gr, gc).copy() for k in STAT_COUNTS + STAT_VALUES}
+    else:
+        tiles = {k: np.zeros((gr, gc), np.int64 if k in STAT_COUNTS else np.float64)
+                 for k in STAT_COUNTS + STAT_VALUES}
+    return {"numel": int(r.numel), "rank": int(r.rank), "all": _stat_dict(r.all),
+            "first_nan": int(r.first_nan), "first_inf": int(r.first_inf), "grid_rows": gr,
+            "grid_cols": gc, "tile_rows": int(r.tile_rows), "tile_cols": int(r.tile_cols),
+            "tiles": tiles}
+
+
+def stats_batch(items, stream=None) -> list:
+    """Diagnostic statistics of several buffers in one call (nmv_stats);
+    `items` holds (tensor, (tile_rows, tile_cols)) pairs."""
+    lib = load()
+    keep = _Keep()
+    structs = []
+    for x, tile in items:
+        c = StatsCase()
+        c.x = _tensor(x, keep)
+        c.tile_rows, c.tile_cols = int(tile[0]), int(tile[1])
+        keep.items.append(x)
+        structs.append(c)
+    arr = (StatsCase * max(len(structs), 1))(*structs)
+    out = ctypes.POINTER(StatsResult)()
+    rc = lib.nmv_stats(arr, len(structs), _stream_handle(stream), ctypes.byref(out))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    try:
+        return [stats_result_to_dict(out[i]) for i in range(len(structs))]
+    finally:
+        if out:
+            lib.nmv_result_free(out)
+
+
+def stats(x: torch.Tensor, *, tile=(64, 64), stream=None) -> dict:
+    """Diagnostic statistics of one buffer (nmv_stats): the whole tensor and
+    every tile of its [M, N] view."""
+    return stats_batch([(x, tile)], stream=stream)[0]
 
 
 PROFILE_TIMING = 1

@@ -41,7 +41,8 @@ def test_struct_layout_matches_header(tmp_path):
     from paper_2608_02712_gb300 import nmv
     prog = tmp_path / "layout.c"
     fields = {"nmv_tensor": nmv.Tensor, "nmv_case": nmv.Case, "nmv_result": nmv.Result,
-              "nmv_profile": nmv.Profile}
+              "nmv_profile": nmv.Profile, "nmv_stats_case": nmv.StatsCase, "nmv_stat": nmv.Stat,
+              "nmv_stats_result": nmv.StatsResult}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "nmv.h"', 'int main(void){']
     for cname, py in fields.items():
         lines.append('printf("%s sizeof %%zu\\n", sizeof(%s));' % (cname, cname))
@@ -176,3 +177,24 @@ def test_binding_refuses_host_tensors():
     from paper_2608_02712_gb300 import validate
     with pytest.raises(ValueError):
         validate(torch.zeros(4), torch.zeros(4), rtol=0, atol=0)
+
+
+def test_stats_rejects_bad_cases(lib):
+    from paper_2608_02712_gb300 import nmv
+    shape = (ctypes.c_int64 * 2)(4, 4)
+    buf = (ctypes.c_float * 16)()
+    t = nmv.Tensor(ctypes.cast(buf, ctypes.c_void_p), 0, 2, ctypes.cast(shape, ctypes.POINTER(ctypes.c_int64)))
+    good = nmv.StatsCase(t, 2, 2)
+    out = ctypes.POINTER(nmv.StatsResult)()
+    for bad in (nmv.StatsCase(t, 0, 2), nmv.StatsCase(t, 2, (1 << 24) + 1),
+                nmv.StatsCase(nmv.Tensor(t.data, 9, 2, t.shape), 2, 2),
+                nmv.StatsCase(nmv.Tensor(None, 0, 2, t.shape), 2, 2)):
+        arr = (nmv.StatsCase * 2)(good, bad)
+        assert lib.nmv_stats(arr, 2, None, ctypes.byref(out)) == nmv.NMV_EINVAL and not out
+        assert lib.nmv_last_error().startswith(b"case 1:")
+    big = (ctypes.c_int64 * 2)(1 << 12, 1 << 12)
+    huge = nmv.StatsCase(nmv.Tensor(t.data, 0, 2, ctypes.cast(big, ctypes.POINTER(ctypes.c_int64))), 1, 1)
+    assert lib.nmv_stats(ctypes.byref(huge), 1, None, ctypes.byref(out)) == nmv.NMV_EINVAL   # 2^24 tiles
+    assert lib.nmv_stats(None, 1, None, ctypes.byref(out)) == nmv.NMV_EINVAL
+    assert lib.nmv_stats(ctypes.byref(good), 1, None, None) == nmv.NMV_EINVAL
+    assert lib.nmv_stats(ctypes.byref(good), 0, None, ctypes.byref(out)) == nmv.NMV_OK and not out
