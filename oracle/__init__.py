@@ -73,6 +73,11 @@ def _bind(path: str):
         fn.argtypes = [ctypes.c_uint32]
     lib.oracle_pass.restype = ctypes.c_int
     lib.oracle_pass.argtypes = [ctypes.c_double] * 4
+    lib.oracle_forensics.restype = ctypes.c_int
+    lib.oracle_forensics.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int, i64p,
+                                     ctypes.c_double, ctypes.c_double, ctypes.c_int, ctypes.c_int64,
+                                     ctypes.c_double, ctypes.c_double, i64p, i64p, f64p, f64p, i64p,
+                                     ctypes.POINTER(ctypes.c_uint32)]
     lib.oracle_stats.restype = ctypes.c_int
     lib.oracle_stats.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_int64,
                                  ctypes.c_int64, ctypes.c_int64, i64p, f64p, i64p, i64p, f64p]
@@ -110,6 +115,9 @@ class Oracle:
 
     def stats(self, x, **kw):
         return _stats(self.lib, x, **kw)
+
+    def forensics(self, cand, ref, **kw):
+        return _forensics(self.lib, cand, ref, **kw)
 
 
 def _decode(lib, bits: int, dtype: torch.dtype) -> float:
@@ -285,3 +293,49 @@ def _stats(lib, x: torch.Tensor, *, tile=(64, 64)) -> dict:
     return {"numel": numel, "rank": len(shape), "all": _stat_dict(counts, f),
             "first_nan": int(first[0]), "first_inf": int(first[1]),
             "grid_rows": gr, "grid_cols": gc, "tile_rows": th, "tile_cols": tw, "tiles": tiles}
+
+
+FX_FLAGS = {"NEAR_PASS": 1, "F16_CEILING": 2, "AXIS_GROWTH": 4}
+ULP_BINS = 34
+
+
+def forensics(cand: torch.Tensor, ref: torch.Tensor, **kw) -> dict:
+    """Deep forensics of one pair of CPU tensors (see oracle_forensics in
+    nmv_oracle.c): ulp distances, fp16-ceiling counts, error growth along an
+    axis, mismatch marginals of every axis and the scheduling flags."""
+    return _forensics(_load(), cand, ref, **kw)
+
+
+def _forensics(lib, cand, ref, *, rtol, atol, axis=-1, near_ulps=4, near_fraction=0.01,
+               growth_factor=4.0) -> dict:
+    if cand.dtype != ref.dtype or tuple(cand.shape) != tuple(ref.shape):
+        raise ValueError("cand and ref must share dtype and shape")
+    cand = cand.detach().cpu().contiguous()
+    ref = ref.detach().cpu().contiguous()
+    shape = tuple(int(s) for s in cand.shape)
+    rank = len(shape)
+    ax = (axis % rank) if rank else 0
+    length = shape[ax] if rank else 1
+    counts = np.zeros(6, np.int64)
+    hist = np.zeros(ULP_BINS, np.int64)
+    growth = np.zeros(max(length, 1), np.float64)
+    gmean = np.zeros(2, np.float64)
+    marg = np.zeros(max(sum(shape), 1), np.int64)
+    flags = np.zeros(1, np.uint32)
+    shp = (ctypes.c_int64 * max(rank, 1))(*shape)
+    rc = lib.oracle_forensics(ctypes.c_void_p(cand.data_ptr()), ctypes.c_void_p(ref.data_ptr()),
+                              DTYPE_CODES[cand.dtype], rank, shp, float(rtol), float(atol), ax,
+                              int(near_ulps), float(near_fraction), float(growth_factor),
+                              _ptr(counts, ctypes.c_int64), _ptr(hist, ctypes.c_int64),
+                              _ptr(growth, ctypes.c_double), _ptr(gmean, ctypes.c_double),
+                              _ptr(marg, ctypes.c_int64), _ptr(flags, ctypes.c_uint32))
+    if rc != 0:
+        raise ValueError("oracle rejected the arguments")
+    offs = np.concatenate([[0], np.cumsum(shape)]).astype(np.int64) if rank else np.zeros(1, np.int64)
+    return {"numel": cand.numel(), "rank": rank, "mismatch": int(counts[0]),
+            "n_finite_pairs": int(counts[1]), "ulp_hist": hist,
+            "max_ulp_mismatch": int(counts[2]), "argmax_ulp_mismatch": int(counts[3]),
+            "mism_nonfinite": int(counts[4]), "mism_within_f16": int(counts[5]),
+            "flags": int(flags[0]), "axis": ax, "axis_len": length, "growth": growth[:length].copy(),
+            "growth_lo": float(gmean[0]), "growth_hi": float(gmean[1]),
+            "marginals": [marg[offs[a]:offs[a + 1]].copy() for a in range(rank)]}

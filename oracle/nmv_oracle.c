@@ -455,3 +455,146 @@ int oracle_stats(const void *x, int dtype, int64_t numel, int64_t ncols, int64_t
     }
     return 0;
 }
+
+/*
+ * ---- deep forensics: per-axis maps, ulp distances, error growth ---------
+ *
+ * The evidence behind the adaptive-scheduling rules "near-pass and
+ * fp16-ceiling detection" (Section 4.4) and behind localising a divergence
+ * that "compounds along the reduction axis" (Section 3.2, the cumsum of
+ * Table 1), plus mismatch counts at every index of every axis.  The paper
+ * states no formula; the reading written out here, over the pairs of P1:
+ *
+ *   ord(x)    the order-preserving integer of a float's bits: +m for a
+ *             positive sign, -m for a negative one (m = the magnitude bits),
+ *             so +0 and -0 are both 0 and consecutive floats differ by 1;
+ *             int32: the value itself
+ *   u(i)      = |ord(c_i) - ord(r_i)|, the distance in representable values
+ *   ulp_hist  both-finite pairs by u: bin 0 holds u = 0, bin k (1..33) holds
+ *             2^(k-1) <= u < 2^k (bin 33 also everything above)
+ *   max_ulp_mismatch / argmax   the largest u over finite mismatches
+ *             (both values finite) and the lowest index attaining it (-1, -1)
+ *   mism_nonfinite   mismatches where c or r is NaN or infinite
+ *   mism_within_f16  finite mismatches with fl(|c - r|) <= h(r), h(r) the
+ *             spacing of an 11-bit significand at |r|: 2^(max(e, -14) - 10)
+ *             with e = floor(log2 |r|), and 2^-24 for r = 0 (one fp16 ulp,
+ *             its exponent range unbounded above)
+ *   growth[j] max fl(|c - r|) over both-finite pairs whose coordinate on the
+ *             chosen axis is j (0.0 if none)
+ *   growth_lo / growth_hi   the mean of growth[] over its first / last
+ *             q = max(1, floor(len / 4)) entries: a left-to-right fp64 sum
+ *             divided by q (0.0 for an empty axis)
+ *   marginals mismatches at each index of each axis (axis 0 first)
+ *   flags     NEAR_PASS (1): mismatch > 0, no non-finite mismatch,
+ *               max_ulp_mismatch <= near_ulps and mismatch <= near_fraction
+ *               * numel (fp64 product);
+ *             F16_CEILING (2): mismatch > 0, no non-finite mismatch and
+ *               mism_within_f16 == mismatch;
+ *             AXIS_GROWTH (4): len >= 4, growth_hi > 0 and growth_hi >=
+ *               growth_factor * growth_lo.
+ */
+#define OR_FX_NEAR_PASS 1u
+#define OR_FX_F16_CEILING 2u
+#define OR_FX_AXIS_GROWTH 4u
+#define OR_ULP_BINS 34
+
+static int64_t or_ord(uint32_t bits, int dtype)
+{
+    if (dtype == OR_I32) return (int64_t)(int32_t)bits;
+    int width = elem_size(dtype) * 8;
+    uint32_t sign = (bits >> (width - 1)) & 1u;
+    int64_t mag = (int64_t)(bits & ((width == 32) ? 0x7fffffffu : 0x7fffu));
+    return sign ? -mag : mag;
+}
+
+static double or_f16_spacing(double r)
+{
+    double a = fabs(r);
+    if (a == 0.0) return ldexp(1.0, -24);
+    int e;
+    frexp(a, &e);          /* a = m * 2^e with 0.5 <= m < 1, so floor(log2 a) = e - 1 */
+    int fl = e - 1;
+    if (fl < -14) fl = -14;
+    return ldexp(1.0, fl - 10);
+}
+
+int oracle_forensics(const void *cand, const void *ref, int dtype, int rank, const int64_t *shape,
+                     double rtol, double atol, int axis, int64_t near_ulps, double near_fraction,
+                     double growth_factor, int64_t *counts, int64_t *ulp_hist, double *growth,
+                     double *growth_mean, int64_t *marginals, uint32_t *flags)
+{
+    if (rank < 0 || rank > 8) return -1;
+    int64_t numel = 1;
+    for (int a = 0; a < rank; ++a) numel *= shape[a];
+    if (rank > 0 && (axis < 0 || axis >= rank)) return -1;
+    int64_t len = rank > 0 ? shape[axis] : 1;
+    int64_t stride = 1;                       /* elements between consecutive indices of the axis */
+    for (int a = rank - 1; a > axis; --a) stride *= shape[a];
+    int64_t moff[9];
+    moff[0] = 0;
+    for (int a = 0; a < rank; ++a) moff[a + 1] = moff[a] + shape[a];
+    for (int64_t t = 0; t < moff[rank]; ++t) marginals[t] = 0;
+    for (int k = 0; k < OR_ULP_BINS; ++k) ulp_hist[k] = 0;
+    for (int64_t j = 0; j < len; ++j) growth[j] = 0.0;
+    int64_t mismatch = 0, n_finite = 0, max_ulp = -1, arg_ulp = -1, nonfin = 0, within = 0;
+    for (int64_t i = 0; i < numel; ++i) {
+        uint32_t cb = load_bits(cand, dtype, i);
+        uint32_t rb = load_bits(ref, dtype, i);
+        double c = decode(cb, dtype);
+        double r = decode(rb, dtype);
+        int fin = isfinite(c) && isfinite(r);
+        int64_t u = or_ord(cb, dtype) - or_ord(rb, dtype);
+        if (u < 0) u = -u;
+        if (fin) {
+            n_finite++;
+            int k = 0;
+            if (u > 0) {
+                k = 1;
+                while (k < OR_ULP_BINS - 1 && u >= ((int64_t)1 << k)) k++;
+            }
+            ulp_hist[k]++;
+            double d = fabs(c - r);
+            int64_t j = rank > 0 ? (i / stride) % len : 0;
+            if (d > growth[j]) growth[j] = d;
+        }
+        if (!oracle_pass(c, r, rtol, atol)) {
+            mismatch++;
+            if (!fin) {
+                nonfin++;
+            } else {
+                if (u > max_ulp) { max_ulp = u; arg_ulp = i; }
+                if (fabs(c - r) <= or_f16_spacing(r)) within++;
+            }
+            int64_t rest = i;
+            for (int a = rank - 1; a >= 0; --a) {
+                int64_t coord = rest % shape[a];
+                rest /= shape[a];
+                marginals[moff[a] + coord]++;
+            }
+        }
+    }
+    int64_t q = len / 4;
+    if (q < 1) q = 1;
+    double lo = 0.0, hi = 0.0;
+    if (len > 0) {
+        for (int64_t j = 0; j < q && j < len; ++j) lo += growth[j];
+        for (int64_t j = len - q; j < len; ++j) if (j >= 0) hi += growth[j];
+        lo /= (double)q;
+        hi /= (double)q;
+    }
+    uint32_t f = 0;
+    if (mismatch > 0 && nonfin == 0 && max_ulp <= near_ulps &&
+        (double)mismatch <= near_fraction * (double)numel) f |= OR_FX_NEAR_PASS;
+    if (mismatch > 0 && nonfin == 0 && within == mismatch) f |= OR_FX_F16_CEILING;
+    if (len >= 4 && hi > 0.0 && hi >= growth_factor * lo) f |= OR_FX_AXIS_GROWTH;
+    counts[0] = mismatch;
+    counts[1] = n_finite;
+    counts[2] = max_ulp;
+    counts[3] = arg_ulp;
+    counts[4] = nonfin;
+    counts[5] = within;
+    growth_mean[0] = lo;
+    growth_mean[1] = hi;
+    flags[0] = f;
+    return 0;
+}

@@ -1308,6 +1308,86 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   reload_thr(R, W);
 }
 
+// A float step of a warp in the dense regime (its last batch was mostly
+// mismatches, as where a candidate passes an input through): the hard
+// step's one classification pass (TwoSum of c - r, the sure-pass and
+// sure-fail bounds, the maximum thresholds) runs inline, and when every
+// element of the warp is dense (finite, decided by the fp32 bounds, no
+// candidate for a maximum) the SSE terms, the mismatch count and the maps
+// are done here too, with the hard step's arithmetic; any other step goes
+// out of line as usual.  A clean step takes this path's SSE arithmetic
+// with e = 0, which is the fast path's, so results do not depend on the
+// regime.
+template <int DT, int NIN>
+__device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const uint4 &cv,
+                                           const uint4 &rv, const uint4 &xv, uint32_t erel) {
+  constexpr int V = Tr<DT>::V;
+  const long long t_start = P->stats ? clock64() : 0;
+  if (R.track_c) R.cacc |= (cv.x ^ R.cpat) | (cv.y ^ R.cpat) | (cv.z ^ R.cpat) | (cv.w ^ R.cpat);
+  if (R.track_r) R.racc |= (rv.x ^ R.rpat) | (rv.y ^ R.rpat) | (rv.z ^ R.rpat) | (rv.w ^ R.rpat);
+  if constexpr (NIN == 1) {
+#pragma unroll
+    for (int k = 0; k < V; ++k) {
+      const uint32_t xb = vbits<DT>(xv, k);
+      R.eq[0] += (vbits<DT>(cv, k) == xb) & (vbits<DT>(rv, k) != xb);
+    }
+  } else if constexpr (NIN < 0) {
+    eq_generic<DT>(P, L, cv, rv, P->pbegin + erel);
+  }
+  const float2 m1 = make_float2(-1.f, -1.f);
+  const float2 lo_r2 = make_float2(R.lo_r, R.lo_r), lo_a2 = make_float2(R.lo_a, R.lo_a);
+  const float hr = P->cd.hi_r, ha = P->cd.hi_a;
+  const float2 hi_r2 = make_float2(hr, hr), hi_a2 = make_float2(ha, ha);
+  const float tA = R.tA;
+  const float2 tR2 = make_float2(R.tR, R.tR);
+  float2 s[V / 2], e[V / 2];
+  bool dense = true;
+  uint32_t mask = 0;
+#pragma unroll
+  for (int j = 0; j < V / 2; ++j) {
+    const float2 c2 = make_float2(vdec<DT>(cv, 2 * j), vdec<DT>(cv, 2 * j + 1));
+    const float2 r2 = make_float2(vdec<DT>(rv, 2 * j), vdec<DT>(rv, 2 * j + 1));
+    const float2 s2 = __ffma2_rn(r2, m1, c2);
+    const float2 bb = __ffma2_rn(c2, m1, s2);
+    const float2 y = __ffma2_rn(__ffma2_rn(bb, m1, s2), m1, c2);
+    s[j] = s2;
+    e[j] = __ffma2_rn(__fadd2_rn(r2, bb), m1, y);
+    const float2 ar2 = make_float2(fabsf(r2.x), fabsf(r2.y));
+    const float2 a2 = __ffma2_rz(ar2, lo_r2, lo_a2);
+    const float2 h2 = __ffma2_ru(ar2, hi_r2, hi_a2);
+    const float2 t2 = __fmul2_rz(ar2, tR2);
+    const float as0 = fabsf(s2.x), as1 = fabsf(s2.y);
+    dense &= (as0 <= a2.x || as0 > h2.x) && (as0 < tA || (as0 == tA && e[j].x == 0.f)) &&
+             as0 <= (e[j].x == 0.f ? t2.x : __fmul_rz(t2.x, kMarginLo));
+    dense &= (as1 <= a2.y || as1 > h2.y) && (as1 < tA || (as1 == tA && e[j].y == 0.f)) &&
+             as1 <= (e[j].y == 0.f ? t2.y : __fmul_rz(t2.y, kMarginLo));
+    if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
+    if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
+  }
+  if (!__all_sync(0xffffffffu, dense)) {
+    R.sse = hard_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
+    reload_thr(R, W);
+    return;
+  }
+#pragma unroll
+  for (int j = 0; j < V / 2; ++j) {
+    const float2 p = __fmul2_rn(s[j], s[j]);
+    const float2 pe = __ffma2_rn(s[j], s[j], __fmul2_rn(p, m1));
+    const float2 q = __ffma2_rn(__fadd2_rn(s[j], s[j]), e[j], pe);
+    const float2 t = __fadd2_rn(R.sse.hi, p);
+    const float2 bp = __ffma2_rn(R.sse.hi, m1, t);
+    const float2 x2 = __ffma2_rn(__ffma2_rn(bp, m1, t), m1, R.sse.hi);
+    const float2 err = __fadd2_rn(x2, __ffma2_rn(bp, m1, p));
+    R.sse.lo = __fadd2_rn(R.sse.lo, __fadd2_rn(err, q));
+    R.sse.hi = t;
+  }
+  if (__any_sync(0xffffffffu, mask != 0)) {
+    if (P->cd.amode) record_step_aligned<V>(P, W, mask, P->pbegin + erel);
+    else record_step(P, W, mask, P->pbegin + erel, V);
+  }
+  if (P->stats) count_stats(W, 2, t_start, 0, 0, 0);
+}
+
 // Issue the copies of one stage (half a batch), at byte offset `off` of the
 // piece and with `bytes` (whole steps only) per tensor (lane 0 only).  A
 // ragged rest and the buffers of a case that is not 16-byte aligned
@@ -1425,6 +1505,8 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   uint64_t gAR = ld_relaxed64(g_thr);
   const uint32_t lane_off = (uint32_t)lane * V;
   int flush = 0;
+  // warp-uniform: the warp's last batch was mostly mismatches (float types)
+  bool dmode = false;
   for (uint32_t j = 0;; ++j) {
     const uint32_t b = W->stage_b[rp.stage];
     if (b == kNoBatch) break;
@@ -1478,13 +1560,24 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       const uint32_t hoff = b * BB + h * HB;
       const uint32_t hrel = erel + h * (HS * STEP);
       if (vec_ok && hoff < pbytes && pbytes - hoff >= HB) {
+        if (!Tr<DT>::kInt && dmode) {
+#pragma unroll 1
+          for (int u = 0; u < HS; ++u) {
+            const uint4 cv = lds_v4(stage + u * 512);
+            const uint4 rv = lds_v4(stage + HB + u * 512);
+            uint4 xv = make_uint4(0, 0, 0, 0);
+            if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+            if constexpr (!Tr<DT>::kInt) step_dense<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+          }
+        } else {
 #pragma unroll 2
-        for (int u = 0; u < HS; ++u) {
-          const uint4 cv = lds_v4(stage + u * 512);
-          const uint4 rv = lds_v4(stage + HB + u * 512);
-          uint4 xv = make_uint4(0, 0, 0, 0);
-          if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
-          step<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+          for (int u = 0; u < HS; ++u) {
+            const uint4 cv = lds_v4(stage + u * 512);
+            const uint4 rv = lds_v4(stage + HB + u * 512);
+            uint4 xv = make_uint4(0, 0, 0, 0);
+            if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+            step<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+          }
         }
       } else {
         // part of the case's last batch, or a case that is not 16-byte aligned
@@ -1510,6 +1603,11 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     if (lane == 0) {
       bcount[b] = (int32_t)((uint32_t)W->mism | (W->sbits << kStepBitsShift));
       W->mism_tot += W->mism;
+    }
+    if constexpr (!Tr<DT>::kInt) {
+      // the next batch's regime: dense when at least half of this one mismatched
+      __syncwarp();
+      dmode = 2 * W->mism >= (int64_t)BATCH;
     }
     if (R.track_c | R.track_r) {
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);

@@ -482,3 +482,25 @@ def stats_fuzz(seed: int, device="cpu", max_dim: int = 200):
         x.view(-1)[torch.rand(x.numel(), generator=gd, device=device) < 0.2] = 0
     tile = (int(torch.randint(1, 70, (1,), generator=g)), int(torch.randint(1, 70, (1,), generator=g)))
     return x, tile
+
+
+def cumsum_fp16(seed: int = 5, device="cpu", rows: int = 256, cols: int = 4096, repaired: bool = False):
+    """The cumsum case of the paper's Table 1: the reference accumulates a
+    running sum along the last axis in FP16 arithmetic with per-step
+    rounding (the vendor reference), the candidate in pure FP32 (the
+    near-miss baseline), whose divergence compounds along the axis; with
+    repaired=True the candidate rounds every step to FP16 too (the fix) and
+    matches.  Inputs x ~ fp16(N(0, 0.1) + 0.05); both outputs are stored as
+    fp32.  Tolerances: torch.testing's fp16 defaults."""
+    g = _gen(seed, device)
+    x = (torch.randn(rows, cols, generator=g, device=device) * 0.1 + 0.05).to(torch.float16)
+    xf = x.float()
+    ref = torch.empty(rows, cols, device=device)
+    acc = torch.zeros(rows, device=device, dtype=torch.float16)
+    for j in range(cols):  # per-step fp16 rounding of the running sum
+        acc = (acc.float() + xf[:, j]).to(torch.float16)
+        ref[:, j] = acc.float()
+    cand = ref.clone() if repaired else torch.cumsum(xf, dim=1)
+    rtol, atol = DEFAULT_TOL[torch.float16]
+    return _case("cumsum_fp16_%dx%d%s" % (rows, cols, "_repaired" if repaired else ""), cand, ref,
+                 rtol, atol, (16, 256), 256)

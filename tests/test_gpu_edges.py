@@ -102,3 +102,33 @@ def test_aligned_localisation_wide_grid(dt):
     got = validate(cand, ref, rtol=rtol, atol=atol, tile=(3, v), first_k=50)
     want = oracle.validate(cand.cpu(), ref.cpu(), rtol=rtol, atol=atol, tile=(3, v), first_k=50)
     assert_same(got, want, "aligned wide grid %s" % dt)
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16, torch.float16], ids=["f32", "bf16", "f16"])
+@pytest.mark.parametrize("with_input", [False, True], ids=["noinput", "input"])
+@pytest.mark.parametrize("n", [4096, 4099], ids=["aligned", "ragged"])
+def test_dense_regime_transitions(dt, with_input, n):
+    """Runs of rows that are wrong everywhere (a pass-through of the input)
+    between clean runs, at several run lengths, with NaN/Inf and growing
+    errors inside the dense runs: warps switch into and out of the dense
+    regime, and its steps fall back to the exact path where they must."""
+    g = torch.Generator(device="cuda").manual_seed(11)
+    m = 700
+    ref = torch.randn(m, n, generator=g, device="cuda").to(dt)
+    x = torch.randn(m, n, generator=g, device="cuda").to(dt)
+    cand = (ref.float() * (1 + torch.randn(m, n, generator=g, device="cuda") * 1e-4)).to(dt)
+    r0 = 0
+    for run in (1, 3, 17, 64, 2, 200):
+        cand[r0 + 5: r0 + 5 + run] = x[r0 + 5: r0 + 5 + run]
+        r0 += 5 + run + run // 2
+    cf = cand.view(-1)
+    for i in (6 * n + 3, 50 * n + 1000, 300 * n + 17):
+        cf[i] = float("nan")
+    cf[100 * n + 5] = float("-inf")
+    cf[350 * n + 2] = 1e4   # a late, larger error inside a dense run (rows 159-358)
+    inputs = [x.view(-1)] if with_input else []
+    rtol, atol = (1e-3, 1e-5) if dt == torch.float32 else (1.6e-2, 1e-3)
+    got = validate(cand, ref, inputs=inputs, rtol=rtol, atol=atol, tile=(8, 128), first_k=2000)
+    want = oracle.validate(cand.cpu(), ref.cpu(), inputs=[t.cpu() for t in inputs], rtol=rtol, atol=atol,
+                           tile=(8, 128), first_k=2000)
+    assert_same(got, want, "dense regime %s input=%s n=%d" % (dt, with_input, n))

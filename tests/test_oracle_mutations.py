@@ -14,6 +14,7 @@ import test_oracle_closed_forms as tc
 import test_oracle_decoders as td
 import test_oracle_golden as tg
 import test_oracle_predicate as tp
+import test_oracle_forensics as tf
 import test_oracle_stats as ts
 from _golden import fixture_files
 
@@ -60,6 +61,22 @@ MUTATIONS = {
                                "r < nrows && r <= (tr + 1) * tile_rows; ++r)"),
     "stats_min_includes_first_zero": ("if (!a->have || x < a->mn) a->mn = x;",
                                       "if (x < a->mn) a->mn = x;"),
+    # deep forensics
+    "fx_ulp_from_raw_bits": ("return sign ? -mag : mag;", "return (int64_t)bits;"),
+    "fx_ulp_bin_off_by_one": ("while (k < OR_ULP_BINS - 1 && u >= ((int64_t)1 << k)) k++;",
+                              "while (k < OR_ULP_BINS - 1 && u > ((int64_t)1 << k)) k++;"),
+    "fx_within_strict": ("if (fabs(c - r) <= or_f16_spacing(r)) within++;",
+                         "if (fabs(c - r) < or_f16_spacing(r)) within++;"),
+    "fx_subnormal_spacing": ("if (fl < -14) fl = -14;", "if (fl < -15) fl = -15;"),
+    "fx_first_axis_marginal_lost": ("int64_t coord = rest % shape[a];",
+                                    "int64_t coord = rest % shape[a];\n                if (a == 0) coord = 0;"),
+    "fx_quarter_rounds_up": ("int64_t q = len / 4;", "int64_t q = (len + 3) / 4;"),
+    "fx_near_pass_ignores_nonfinite": ("if (mismatch > 0 && nonfin == 0 && max_ulp <= near_ulps &&",
+                                       "if (mismatch > 0 && max_ulp <= near_ulps &&"),
+    "fx_growth_axis_stride": ("for (int a = rank - 1; a > axis; --a) stride *= shape[a];",
+                              "for (int a = rank - 1; a >= axis; --a) stride *= shape[a];"),
+    "fx_argmax_ulp_last": ("if (u > max_ulp) { max_ulp = u; arg_ulp = i; }",
+                           "if (u >= max_ulp) { max_ulp = u; arg_ulp = i; }"),
 }
 
 
@@ -82,6 +99,11 @@ def _pins(orc):
     yield lambda: ts.test_stats_int32_sums_are_exact(orc)
     yield lambda: ts.test_stats_float_sums_are_compensated(orc)
     yield lambda: ts.test_stats_empty_and_rank0(orc)
+    yield lambda: [tf.test_forensics_fuzz_against_brute_force(orc, s) for s in range(60)]
+    yield lambda: tf.test_forensics_ulp_distances_by_hand(orc)
+    yield lambda: tf.test_forensics_f16_spacing_boundary(orc)
+    yield lambda: tf.test_forensics_growth_and_marginals_closed_form(orc)
+    yield lambda: tf.test_forensics_near_pass(orc)
 
 
 @pytest.mark.parametrize("name", sorted(MUTATIONS))
