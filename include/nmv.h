@@ -269,8 +269,132 @@ typedef struct nmv_stats_result {
  * allocated. */
 int nmv_stats(const nmv_stats_case *cases, int64_t n, void *cuda_stream, nmv_stats_result **out);
 
-/* Release what one nmv_validate / nmv_validate_batch / nmv_stats call
- * returned.  NULL is accepted.  (The block is mapped pinned host memory, which the library
+/* ---- deep forensics: per-axis maps, ulp distances, error growth -------
+ * The evidence the engine's adaptive-scheduling rules read ("near-pass and
+ * fp16-ceiling detection", Section 4.4) and the localisation of a divergence
+ * that compounds along a reduction axis (Section 3.2, the cumsum of Table 1),
+ * plus mismatch counts at every index of every axis.  An on-demand second
+ * pass over a pair (the engine instruments only after a failed attempt,
+ * Section 4.2).  The paper gives no formula; this library's reading, over the
+ * pairs and the predicate of nmv_validate:
+ *
+ *   ord(x)   the order-preserving integer of a float's bits (+m for a
+ *            positive sign, -m for a negative one, m the magnitude bits: +0
+ *            and -0 are both 0, consecutive floats differ by 1); int32: x
+ *   u        = |ord(c) - ord(r)|, the distance in representable values
+ *   h(r)     one fp16 spacing at |r|: 2^(max(floor(log2 |r|), -14) - 10),
+ *            2^-24 for r = 0 (the exponent range unbounded above)
+ *
+ * Every field is exact; growth_lo / growth_hi are left-to-right fp64 sums
+ * divided by q, the same operations as the definition. */
+#define NMV_ULP_BINS 34
+#define NMV_FX_NEAR_PASS 1u    /* mismatch > 0, no non-finite mismatch,
+                                  max_ulp_mismatch <= near_ulps and mismatch
+                                  <= near_fraction * numel (fp64 product)   */
+#define NMV_FX_F16_CEILING 2u  /* mismatch > 0, no non-finite mismatch and
+                                  every mismatch within one fp16 spacing h(r)
+                                  (the candidate sits at fp16 precision)    */
+#define NMV_FX_AXIS_GROWTH 4u  /* axis_len >= 4, growth_hi > 0 and growth_hi
+                                  >= growth_factor * growth_lo (the error
+                                  compounds along the axis)                  */
+
+typedef struct nmv_forensics_case {
+    nmv_tensor cand, ref;       /* as nmv_case: same dtype and shape        */
+    double rtol, atol;          /* the predicate's tolerance                */
+    int32_t axis;               /* growth axis, -rank .. rank-1 (negative
+                                   counts from the last); rank 0: ignored   */
+    int32_t reserved;           /* must be 0                                */
+    int64_t near_ulps;          /* NMV_FX_NEAR_PASS, >= 0                   */
+    double near_fraction;       /* NMV_FX_NEAR_PASS, finite, >= 0           */
+    double growth_factor;       /* NMV_FX_AXIS_GROWTH, finite, >= 0         */
+} nmv_forensics_case;
+
+typedef struct nmv_forensics_result {
+    int32_t status;             /* NMV_OK                                   */
+    int32_t rank;
+    int64_t numel;
+    int64_t mismatch;           /* as nmv_result.mismatch                   */
+    int64_t n_finite_pairs;
+    int64_t ulp_hist[NMV_ULP_BINS];  /* both-finite pairs by u: bin 0: u = 0,
+                                        bin k: 2^(k-1) <= u < 2^k (bin 33 also
+                                        every larger u)                     */
+    int64_t max_ulp_mismatch;   /* largest u over mismatches with both values
+                                   finite, -1 if none                        */
+    int64_t argmax_ulp_mismatch;    /* lowest index attaining it, -1        */
+    int64_t mism_nonfinite;     /* mismatches with a NaN or infinite value  */
+    int64_t mism_within_f16;    /* finite mismatches with fl64|c - r| <= h(r) */
+    uint32_t flags;             /* NMV_FX_* bits                            */
+    int32_t axis;               /* the growth axis, 0 .. rank-1             */
+    int64_t axis_len;           /* its extent (1 for rank 0)                */
+    double growth_lo;           /* mean of growth over its first q entries,
+                                   q = max(1, floor(axis_len / 4))          */
+    double growth_hi;           /* ... and over its last q entries          */
+    double *growth;             /* [axis_len]: max fl64|c - r| over the
+                                   both-finite pairs at each index of the
+                                   axis (0.0 if none)                        */
+    int64_t marg_off[NMV_MAX_RANK + 1];  /* axis a's marginal is
+                                   marginals[marg_off[a] .. marg_off[a+1])  */
+    int64_t *marginals;         /* mismatches at each index of each axis    */
+} nmv_forensics_result;
+
+/* Deep forensics of n pairs on `cuda_stream`, synchronous.  sum(shape) of a
+ * case may be at most NMV_MAX_HIST_BINS.  Every case is checked first (the
+ * message names a bad case's index).  On NMV_OK, *out points to an array of
+ * n results released by ONE nmv_result_free(*out) call; on error *out is
+ * NULL and nothing stays allocated. */
+int nmv_forensics(const nmv_forensics_case *cases, int64_t n, void *cuda_stream,
+                  nmv_forensics_result **out);
+
+/* ---- full-coverage escalation --------------------------------------------
+ * The engine's validation escalation (Section 4.3, "Full-coverage
+ * evaluation"; Figure 3, bottom-right; S6.1): the lightweight case set is
+ * validated first (one nmv_validate_batch call), and only when every one of
+ * its cases passes does the extended set run (a second call).  A repair is
+ * accepted when every case of both sets passes and no case raises an
+ * integrity hazard (NMV_FLAG_CAND_EQ_INPUT, or CAND_CONSTANT / CAND_ALL_ZERO
+ * without the matching REF_* flag).  The per-case evidence (pass/fail and
+ * numerical match rate, the "x% matched cases" of Table S4) is written as a
+ * canonical text record, one header line and one line per validated case:
+ *
+ *   nmv-sweep v1 light=<n> ext=<n> escalated=<0|1> accepted=<0|1>
+ *       pass_light=<n> pass_ext=<n>
+ *   <L|E> <index> dtype=<d> numel=<n> pass=<0|1> mismatch=<n> match=<%.17g>
+ *       max_abs=<%.17g> max_rel=<%.17g> nonfinite=<n> flags=<u>
+ *
+ * (each record is one line; nonfinite counts NaN/Inf on both sides) and
+ * sealed with its SHA-256 digest (FIPS 180-4), so the evidence behind an
+ * acceptance cannot change unnoticed. */
+typedef struct nmv_sweep_report {
+    int32_t status;             /* NMV_OK                                   */
+    int32_t escalated;          /* 1: the extended set ran                  */
+    int32_t accepted;           /* 1: every case of both sets passed, no hazard */
+    uint32_t flags_any;         /* OR of the NMV_FLAG_* bits of the cases run */
+    int64_t n_light, n_ext;     /* cases in each set                        */
+    int64_t n_run;              /* cases validated: n_light (+ n_ext when escalated) */
+    int64_t n_pass_light, n_pass_ext;
+    double match_rate_light;    /* n_pass_light / n_light                    */
+    double match_rate_ext;      /* n_pass_ext / n_ext when escalated, else 0 */
+    uint8_t digest[32];         /* SHA-256 of evidence[0 .. evidence_len)   */
+    char *evidence;             /* the canonical record (NUL-terminated)    */
+    int64_t evidence_len;
+    nmv_result *results;        /* [n_run]: the light cases, then the extended */
+    nmv_result *blocks[2];      /* the result blocks the records point into
+                                   (owned by the report)                     */
+} nmv_sweep_report;
+
+/* Run the escalation on `cuda_stream` (synchronous): light[0 .. n_light),
+ * n_light >= 1, then ext[0 .. n_ext) if every light case passed.  Cases are
+ * checked as in nmv_validate_batch (the message names the set and the
+ * case).  On NMV_OK, *out is released with nmv_sweep_free(). */
+int nmv_sweep(const nmv_case *light, int64_t n_light, const nmv_case *ext, int64_t n_ext,
+              void *cuda_stream, nmv_sweep_report **out);
+void nmv_sweep_free(nmv_sweep_report *r);   /* NULL is accepted */
+
+/* SHA-256 (FIPS 180-4) of len bytes, the digest of the sweep's evidence. */
+void nmv_sha256(const void *data, int64_t len, uint8_t out[32]);
+
+/* Release what one nmv_validate / nmv_validate_batch / nmv_stats /
+ * nmv_forensics call returned.  NULL is accepted.  (The block is mapped pinned host memory, which the library
  * keeps for reuse by later calls.) */
 void nmv_result_free(void *r);
 

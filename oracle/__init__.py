@@ -339,3 +339,63 @@ def _forensics(lib, cand, ref, *, rtol, atol, axis=-1, near_ulps=4, near_fractio
             "flags": int(flags[0]), "axis": ax, "axis_len": length, "growth": growth[:length].copy(),
             "growth_lo": float(gmean[0]), "growth_hi": float(gmean[1]),
             "marginals": [marg[offs[a]:offs[a + 1]].copy() for a in range(rank)]}
+
+
+# ---- full-coverage escalation (Section 4.3; Figure 3, bottom-right; S6.1)
+def _hazard(flags: int) -> bool:
+    """An integrity hazard: the candidate passes an input through, or is
+    constant / all zero while the reference is not."""
+    if flags & 1:
+        return True
+    if (flags & 4) and not (flags & 16):
+        return True
+    if (flags & 2) and not (flags & 8):
+        return True
+    return False
+
+
+def sweep(light, extended=()) -> dict:
+    """The escalation policy written out: validate the lightweight set; only
+    if every case passes, validate the extended set; accept when every case
+    of both sets passed and none raised an integrity hazard.  The evidence
+    is one header line and one line per validated case (the format of
+    nmv_sweep in nmv.h), sealed with its SHA-256 digest."""
+    import hashlib
+    codes = DTYPE_CODES
+
+    def run(cases):
+        return [validate(c["cand"], c["ref"], inputs=c.get("inputs", ()), rtol=c["rtol"], atol=c["atol"],
+                         tile=c["tile"], first_k=c["first_k"]) for c in cases]
+
+    rl = run(light)
+    pass_l = sum(int(r["pass"]) for r in rl)
+    escalate = pass_l == len(light) and len(extended) > 0
+    re_ = run(extended) if escalate else []
+    pass_e = sum(int(r["pass"]) for r in re_)
+    hazard = any(_hazard(r["flags"]) for r in rl + re_)
+    accepted = pass_l == len(light) and (len(extended) == 0 or (escalate and pass_e == len(extended))) \
+        and not hazard
+    lines = ["nmv-sweep v1 light=%d ext=%d escalated=%d accepted=%d pass_light=%d pass_ext=%d"
+             % (len(light), len(extended), int(escalate), int(accepted), pass_l, pass_e)]
+
+    def line(tag, i, r, c):
+        nonfin = (r["cand_nan"] + r["cand_posinf"] + r["cand_neginf"] + r["ref_nan"] + r["ref_posinf"]
+                  + r["ref_neginf"])
+        return ("%s %d dtype=%d numel=%d pass=%d mismatch=%d match=%.17g max_abs=%.17g max_rel=%.17g "
+                "nonfinite=%d flags=%d" % (tag, i, codes[c["cand"].dtype], r["numel"], int(r["pass"]),
+                                           r["mismatch"], r["match_fraction"], r["max_abs"], r["max_rel"],
+                                           nonfin, r["flags"]))
+
+    lines += [line("L", i, r, c) for i, (r, c) in enumerate(zip(rl, light))]
+    lines += [line("E", i, r, c) for i, (r, c) in enumerate(zip(re_, extended))]
+    evidence = "".join(ln + "\n" for ln in lines)
+    flags_any = 0
+    for r in rl + re_:
+        flags_any |= r["flags"]
+    return {"escalated": escalate, "accepted": accepted, "flags_any": flags_any,
+            "n_light": len(light), "n_ext": len(extended), "n_run": len(rl) + len(re_),
+            "n_pass_light": pass_l, "n_pass_ext": pass_e,
+            "match_rate_light": pass_l / len(light),
+            "match_rate_ext": pass_e / len(extended) if escalate else 0.0,
+            "evidence": evidence, "digest": hashlib.sha256(evidence.encode()).hexdigest(),
+            "results": rl + re_}

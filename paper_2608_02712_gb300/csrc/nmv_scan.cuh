@@ -1560,14 +1560,15 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       const uint32_t hoff = b * BB + h * HB;
       const uint32_t hrel = erel + h * (HS * STEP);
       if (vec_ok && hoff < pbytes && pbytes - hoff >= HB) {
-        if (!Tr<DT>::kInt && dmode) {
+        if (Tr<DT>::EB == 4 && !Tr<DT>::kInt && dmode) {
 #pragma unroll 1
           for (int u = 0; u < HS; ++u) {
             const uint4 cv = lds_v4(stage + u * 512);
             const uint4 rv = lds_v4(stage + HB + u * 512);
             uint4 xv = make_uint4(0, 0, 0, 0);
             if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
-            if constexpr (!Tr<DT>::kInt) step_dense<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+            if constexpr (Tr<DT>::EB == 4 && !Tr<DT>::kInt)
+              step_dense<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
           }
         } else {
 #pragma unroll 2
@@ -1604,8 +1605,10 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       bcount[b] = (int32_t)((uint32_t)W->mism | (W->sbits << kStepBitsShift));
       W->mism_tot += W->mism;
     }
-    if constexpr (!Tr<DT>::kInt) {
-      // the next batch's regime: dense when at least half of this one mismatched
+    if constexpr (Tr<DT>::EB == 4 && !Tr<DT>::kInt) {
+      // the next batch's regime (fp32): dense when at least half of this one
+      // mismatched (16-bit types keep the plain loop: their scan is bound by
+      // instruction issue on clean data, where every extra branch costs)
       __syncwarp();
       dmode = 2 * W->mism >= (int64_t)BATCH;
     }

@@ -90,6 +90,36 @@ class StatsResult(ctypes.Structure):
                 ("tiles", ctypes.POINTER(Stat))]
 
 
+ULP_BINS = 34
+FX_FLAGS = {"NEAR_PASS": 1, "F16_CEILING": 2, "AXIS_GROWTH": 4}
+
+
+class ForensicsCase(ctypes.Structure):
+    _fields_ = [("cand", Tensor), ("ref", Tensor), ("rtol", ctypes.c_double), ("atol", ctypes.c_double),
+                ("axis", ctypes.c_int32), ("reserved", ctypes.c_int32), ("near_ulps", ctypes.c_int64),
+                ("near_fraction", ctypes.c_double), ("growth_factor", ctypes.c_double)]
+
+
+class ForensicsResult(ctypes.Structure):
+    _fields_ = [("status", ctypes.c_int32), ("rank", ctypes.c_int32), ("numel", ctypes.c_int64),
+                ("mismatch", ctypes.c_int64), ("n_finite_pairs", ctypes.c_int64),
+                ("ulp_hist", ctypes.c_int64 * ULP_BINS), ("max_ulp_mismatch", ctypes.c_int64),
+                ("argmax_ulp_mismatch", ctypes.c_int64), ("mism_nonfinite", ctypes.c_int64),
+                ("mism_within_f16", ctypes.c_int64), ("flags", ctypes.c_uint32), ("axis", ctypes.c_int32),
+                ("axis_len", ctypes.c_int64), ("growth_lo", ctypes.c_double), ("growth_hi", ctypes.c_double),
+                ("growth", _f64p), ("marg_off", ctypes.c_int64 * (MAX_RANK + 1)), ("marginals", _i64p)]
+
+
+class SweepReport(ctypes.Structure):
+    _fields_ = [("status", ctypes.c_int32), ("escalated", ctypes.c_int32), ("accepted", ctypes.c_int32),
+                ("flags_any", ctypes.c_uint32), ("n_light", ctypes.c_int64), ("n_ext", ctypes.c_int64),
+                ("n_run", ctypes.c_int64), ("n_pass_light", ctypes.c_int64), ("n_pass_ext", ctypes.c_int64),
+                ("match_rate_light", ctypes.c_double), ("match_rate_ext", ctypes.c_double),
+                ("digest", ctypes.c_uint8 * 32), ("evidence", ctypes.c_char_p),
+                ("evidence_len", ctypes.c_int64), ("results", ctypes.POINTER(Result)),
+                ("blocks", ctypes.POINTER(Result) * 2)]
+
+
 _lock = threading.Lock()
 _lib = None
 
@@ -113,6 +143,17 @@ def load() -> ctypes.CDLL:
                                                ctypes.POINTER(ctypes.POINTER(Result))]
             lib.nmv_result_free.restype = None
             lib.nmv_result_free.argtypes = [ctypes.c_void_p]
+            lib.nmv_forensics.restype = ctypes.c_int
+            lib.nmv_forensics.argtypes = [ctypes.POINTER(ForensicsCase), ctypes.c_int64, ctypes.c_void_p,
+                                          ctypes.POINTER(ctypes.POINTER(ForensicsResult))]
+            lib.nmv_sweep.restype = ctypes.c_int
+            lib.nmv_sweep.argtypes = [ctypes.POINTER(Case), ctypes.c_int64, ctypes.POINTER(Case),
+                                      ctypes.c_int64, ctypes.c_void_p,
+                                      ctypes.POINTER(ctypes.POINTER(SweepReport))]
+            lib.nmv_sweep_free.restype = None
+            lib.nmv_sweep_free.argtypes = [ctypes.POINTER(SweepReport)]
+            lib.nmv_sha256.restype = None
+            lib.nmv_sha256.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.POINTER(ctypes.c_uint8)]
             lib.nmv_stats.restype = ctypes.c_int
             lib.nmv_stats.argtypes = [ctypes.POINTER(StatsCase), ctypes.c_int64, ctypes.c_void_p,
                                       ctypes.POINTER(ctypes.POINTER(StatsResult))]
@@ -384,6 +425,104 @@ def stats(x: torch.Tensor, *, tile=(64, 64), stream=None) -> dict:
     """Diagnostic statistics of one buffer (nmv_stats): the whole tensor and
     every tile of its [M, N] view."""
     return stats_batch([(x, tile)], stream=stream)[0]
+
+
+def forensics_result_to_dict(r: ForensicsResult) -> dict:
+    rank = int(r.rank)
+    offs = [int(r.marg_off[a]) for a in range(rank + 1)]
+    n_m = offs[-1] if rank else 0
+    marg = _arr(r.marginals, n_m, np.int64)
+    return {"numel": int(r.numel), "rank": rank, "mismatch": int(r.mismatch),
+            "n_finite_pairs": int(r.n_finite_pairs),
+            "ulp_hist": np.array(list(r.ulp_hist), np.int64),
+            "max_ulp_mismatch": int(r.max_ulp_mismatch),
+            "argmax_ulp_mismatch": int(r.argmax_ulp_mismatch),
+            "mism_nonfinite": int(r.mism_nonfinite), "mism_within_f16": int(r.mism_within_f16),
+            "flags": int(r.flags), "axis": int(r.axis), "axis_len": int(r.axis_len),
+            "growth": _arr(r.growth, int(r.axis_len), np.float64),
+            "growth_lo": float(r.growth_lo), "growth_hi": float(r.growth_hi),
+            "marginals": [marg[offs[a]:offs[a + 1]].copy() for a in range(rank)]}
+
+
+def forensics_batch(items, stream=None) -> list:
+    """Deep forensics of several pairs in one call (nmv_forensics); each item
+    is a dict with cand, ref, rtol, atol and optional axis, near_ulps,
+    near_fraction, growth_factor."""
+    lib = load()
+    keep = _Keep()
+    structs = []
+    for it in items:
+        c = ForensicsCase()
+        c.cand = _tensor(it["cand"], keep)
+        c.ref = _tensor(it["ref"], keep)
+        c.rtol, c.atol = float(it["rtol"]), float(it["atol"])
+        c.axis = int(it.get("axis", -1))
+        c.reserved = 0
+        c.near_ulps = int(it.get("near_ulps", 4))
+        c.near_fraction = float(it.get("near_fraction", 0.01))
+        c.growth_factor = float(it.get("growth_factor", 4.0))
+        keep.items.extend([it["cand"], it["ref"]])
+        structs.append(c)
+    arr = (ForensicsCase * max(len(structs), 1))(*structs)
+    out = ctypes.POINTER(ForensicsResult)()
+    rc = lib.nmv_forensics(arr, len(structs), _stream_handle(stream), ctypes.byref(out))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    try:
+        return [forensics_result_to_dict(out[i]) for i in range(len(structs))]
+    finally:
+        if out:
+            lib.nmv_result_free(out)
+
+
+def forensics(cand: torch.Tensor, ref: torch.Tensor, *, rtol: float, atol: float, axis: int = -1,
+              near_ulps: int = 4, near_fraction: float = 0.01, growth_factor: float = 4.0,
+              stream=None) -> dict:
+    """Deep forensics of one pair (nmv_forensics): ulp distances, the fp16
+    ceiling, error growth along an axis, per-axis mismatch marginals."""
+    return forensics_batch([dict(cand=cand, ref=ref, rtol=rtol, atol=atol, axis=axis, near_ulps=near_ulps,
+                                 near_fraction=near_fraction, growth_factor=growth_factor)], stream=stream)[0]
+
+
+def sha256(data: bytes) -> str:
+    """The library's SHA-256 (the sweep evidence digest) of `data`, as hex."""
+    lib = load()
+    out = (ctypes.c_uint8 * 32)()
+    buf = ctypes.create_string_buffer(data, len(data))
+    lib.nmv_sha256(buf, len(data), out)
+    return bytes(out).hex()
+
+
+def sweep(light, extended=(), stream=None) -> dict:
+    """Full-coverage escalation (nmv_sweep): the lightweight cases first, the
+    extended ones only if every lightweight case passed.  Cases are dicts as
+    for validate_batch.  Returns the report with its evidence text, SHA-256
+    digest and the per-case results."""
+    lib = load()
+    keep = _Keep()
+
+    def arr(cases):
+        structs = [make_case(c["cand"], c["ref"], inputs=c.get("inputs", ()), rtol=c["rtol"], atol=c["atol"],
+                             tile=c["tile"], first_k=c["first_k"], keep=keep)[0] for c in cases]
+        return (Case * max(len(structs), 1))(*structs), len(structs)
+
+    la, nl = arr(light)
+    ea, ne = arr(extended)
+    out = ctypes.POINTER(SweepReport)()
+    rc = lib.nmv_sweep(la, nl, ea, ne, _stream_handle(stream), ctypes.byref(out))
+    if rc != NMV_OK:
+        _raise(lib, rc)
+    try:
+        r = out[0]
+        return {"escalated": bool(r.escalated), "accepted": bool(r.accepted), "flags_any": int(r.flags_any),
+                "n_light": int(r.n_light), "n_ext": int(r.n_ext), "n_run": int(r.n_run),
+                "n_pass_light": int(r.n_pass_light), "n_pass_ext": int(r.n_pass_ext),
+                "match_rate_light": float(r.match_rate_light), "match_rate_ext": float(r.match_rate_ext),
+                "digest": bytes(r.digest).hex(),
+                "evidence": ctypes.string_at(r.evidence, int(r.evidence_len)).decode(),
+                "results": [result_to_dict(r.results[i]) for i in range(int(r.n_run))]}
+    finally:
+        lib.nmv_sweep_free(out)
 
 
 PROFILE_TIMING = 1

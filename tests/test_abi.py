@@ -42,7 +42,8 @@ def test_struct_layout_matches_header(tmp_path):
     prog = tmp_path / "layout.c"
     fields = {"nmv_tensor": nmv.Tensor, "nmv_case": nmv.Case, "nmv_result": nmv.Result,
               "nmv_profile": nmv.Profile, "nmv_stats_case": nmv.StatsCase, "nmv_stat": nmv.Stat,
-              "nmv_stats_result": nmv.StatsResult}
+              "nmv_stats_result": nmv.StatsResult, "nmv_forensics_case": nmv.ForensicsCase,
+              "nmv_forensics_result": nmv.ForensicsResult, "nmv_sweep_report": nmv.SweepReport}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "nmv.h"', 'int main(void){']
     for cname, py in fields.items():
         lines.append('printf("%s sizeof %%zu\\n", sizeof(%s));' % (cname, cname))
@@ -198,3 +199,43 @@ def test_stats_rejects_bad_cases(lib):
     assert lib.nmv_stats(None, 1, None, ctypes.byref(out)) == nmv.NMV_EINVAL
     assert lib.nmv_stats(ctypes.byref(good), 1, None, None) == nmv.NMV_EINVAL
     assert lib.nmv_stats(ctypes.byref(good), 0, None, ctypes.byref(out)) == nmv.NMV_OK and not out
+
+
+def test_forensics_rejects_bad_cases(lib):
+    from paper_2608_02712_gb300 import nmv
+    shape = (ctypes.c_int64 * 2)(4, 4)
+    buf = (ctypes.c_float * 16)()
+    t = nmv.Tensor(ctypes.cast(buf, ctypes.c_void_p), 0, 2, ctypes.cast(shape, ctypes.POINTER(ctypes.c_int64)))
+
+    def case(**over):
+        c = nmv.ForensicsCase(t, t, 1e-3, 1e-5, -1, 0, 4, 0.01, 4.0)
+        for k, v in over.items():
+            setattr(c, k, v)
+        return c
+
+    out = ctypes.POINTER(nmv.ForensicsResult)()
+    for bad in ({"axis": 2}, {"axis": -3}, {"rtol": -1.0}, {"atol": float("nan")}, {"reserved": 1},
+                {"near_ulps": -1}, {"near_fraction": float("inf")}, {"growth_factor": -2.0}):
+        arr = (nmv.ForensicsCase * 2)(case(), case(**bad))
+        assert lib.nmv_forensics(arr, 2, None, ctypes.byref(out)) == nmv.NMV_EINVAL and not out, bad
+        assert lib.nmv_last_error().startswith(b"case 1:"), bad
+    c = case()
+    c.ref = nmv.Tensor(t.data, 1, 2, t.shape)
+    assert lib.nmv_forensics(ctypes.byref(c), 1, None, ctypes.byref(out)) == nmv.NMV_EINVAL
+    assert lib.nmv_forensics(ctypes.byref(case()), 0, None, ctypes.byref(out)) == nmv.NMV_OK and not out
+
+
+@pytest.mark.parametrize("n", [0, 1, 55, 56, 63, 64, 65, 119, 120, 1000, 100_000])
+def test_sha256_matches_hashlib(lib, n):
+    import hashlib
+    import random
+    from paper_2608_02712_gb300 import sha256
+    data = random.Random(n).randbytes(n)
+    assert sha256(data) == hashlib.sha256(data).hexdigest()
+
+
+def test_sweep_rejects_empty_light_set(lib):
+    from paper_2608_02712_gb300 import nmv
+    out = ctypes.POINTER(nmv.SweepReport)()
+    assert lib.nmv_sweep(None, 0, None, 0, None, ctypes.byref(out)) == nmv.NMV_EINVAL and not out
+    lib.nmv_sweep_free(None)
