@@ -44,7 +44,12 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default="c5", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--config", default="c5",
+                    choices=["c1", "c2", "c3", "c4", "c5", "stats", "forensics", "sweep"],
+                    help="c1-c5: nmv_validate / nmv_validate_batch on the five workloads; stats: "
+                         "nmv_stats of the c5 candidate (tile 128x128); forensics: nmv_forensics of the "
+                         "c5 pair along its rows; sweep: nmv_sweep with 48 clean lightweight cases "
+                         "escalating to the 512-case c3 set")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--c2-batch", type=int, default=8,
@@ -443,8 +448,116 @@ def run_ours(args, rank, world, local_rank):
     return line
 
 
+# ------------------------------------------------------- other entry points
+AUX_METRIC = {"stats": "diagnostic statistics GB/s (bytes read), 1 GPU",
+              "forensics": "deep forensics GB/s (cand+ref bytes read), 1 GPU",
+              "sweep": "full-coverage sweep GB/s (cand+ref bytes of the cases validated), 1 GPU"}
+
+
+def aux_workload(args):
+    """The data, the call and what a bounded oracle sample of it costs."""
+    from paper_2608_02712_gb300 import workloads as W
+    import paper_2608_02712_gb300 as nmv
+    if args.config == "stats":
+        x = W.c5(device="cuda", shape=(args.c5_rows, 65536))["cand"]
+        nbytes = x.numel() * 4
+        desc = {"workload": "stats_fp32_%dx65536" % args.c5_rows, "tile": [128, 128]}
+
+        def call():
+            return nmv.stats(x, tile=(128, 128))
+
+        def sample(rows):
+            import oracle
+            xs = x[:rows].cpu()
+            t0 = time.perf_counter()
+            oracle.stats(xs, tile=(128, 128))
+            return time.perf_counter() - t0, xs.numel() * 4
+        return call, nbytes, desc, sample, x.shape[0]
+    if args.config == "forensics":
+        case = W.c5(device="cuda", shape=(args.c5_rows, 65536))
+        c, r = case["cand"], case["ref"]
+        nbytes = c.numel() * 8
+        kw = dict(rtol=case["rtol"], atol=case["atol"], axis=0)
+        desc = {"workload": "forensics_fp32_%dx65536_axis0" % args.c5_rows}
+
+        def call():
+            return nmv.forensics(c, r, **kw)
+
+        def sample(rows):
+            import oracle
+            ch, rh = c[:rows].cpu(), r[:rows].cpu()
+            t0 = time.perf_counter()
+            oracle.forensics(ch, rh, **kw)
+            return time.perf_counter() - t0, ch.numel() * 8
+        return call, nbytes, desc, sample, c.shape[0]
+    light = W.c3(seed=20, device="cuda", count=96, cap=1 << 20)[0::2]
+    ext = W.c3(device="cuda")
+    nbytes = sum(case_bytes(x) for x in light + ext)
+    desc = {"workload": "sweep_light48_c3ext512", "light": len(light), "extended": len(ext)}
+
+    def call():
+        return nmv.sweep(light, ext)
+
+    def sample(n):
+        import oracle
+        hl = host_copy(light[:1])
+        he = host_copy(ext[:n])
+        t0 = time.perf_counter()
+        for cs in (hl, he):
+            for c in cs:
+                oracle.validate(c["cand"], c["ref"], rtol=c["rtol"], atol=c["atol"], tile=c["tile"],
+                                first_k=c["first_k"])
+        return time.perf_counter() - t0, sum(case_bytes(x) for x in hl + he)
+    return call, nbytes, desc, sample, len(ext)
+
+
+def run_aux(args):
+    """One JSON line for an entry point other than the validation itself:
+    the whole call timed with CUDA events (inputs resident), every step."""
+    import torch
+    call, nbytes, desc, sample, units = aux_workload(args)
+    torch.cuda.synchronize()
+    for _ in range(max(3, args.warmup)):
+        call()
+    sampler = ClockSampler(0)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = max(1, min(args.steps, 200))
+    with sampler:
+        torch.cuda.synchronize()
+        ev0.record()
+        for _ in range(steps):
+            call()
+        ev1.record()
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / steps
+    value = nbytes / (ms * 1e-3) / 1e9
+    peak, peak_src = measured_peak()
+    line = {"metric": AUX_METRIC[args.config], "value": value, "unit": "GB/s", "n_gpus": 1, "steps": steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32+f64", "data": "synthetic",
+            "config": dict(desc, l2="inputs larger than L2; no flush between steps"),
+            "roofline": {"bound": "hbm", "achieved": value, "peak": peak, "unit": "GB/s", "frac": value / peak,
+                         "traffic": None, "kernel": "whole call (kernels and finalize)",
+                         "peak_source": peak_src, "algorithmic_bytes_per_launch": nbytes},
+            "clocks": sampler.report()}
+    if not args.no_cpu_baseline:
+        probe = max(1, units // 512)
+        t, b = sample(probe)
+        n = int(min(units, max(probe, probe * 12.0 / max(t, 1e-6))))
+        t, b = sample(n)
+        line["cpu_baseline"] = {"value": b / t / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                                "sample": "first %d %s, one pass, %.1f s" % (
+                                    n, "cases of the extended set" if args.config == "sweep" else "rows", t)}
+    return line
+
+
 def main():
     args = parse()
+    if args.config in AUX_METRIC:
+        if args.impl == "reference" or int(os.environ.get("RANK", "0")) != 0:
+            return
+        print(json.dumps(run_aux(args)), flush=True)
+        return
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
