@@ -485,6 +485,7 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.rowp_n = c.tile_rows;
   d.colp_n = c.tile_cols;
   d.rank = c.cand.rank;
+  d.test_stall = injected("stall") ? 1 : 0;
   for (int k = 0; k < c.cand.rank && k < NMV_MAX_RANK; ++k)
     d.sdiv[k] = c.cand.shape[k] > 0 ? make_div((uint64_t)c.cand.shape[k]) : Div64{0, 0};
   d.coord_off = 0;
@@ -522,6 +523,8 @@ void case_key(const nmv_case *cases, int64_t n, std::vector<uint8_t> &key) {
     if (t.rank > 0) put(t.shape, 8 * (size_t)t.rank);
   };
   put(&n, 8);
+  const int32_t stall = injected("stall") ? 1 : 0;  // the wait-limit test hook is part of the descriptors
+  put(&stall, 4);
   for (int64_t i = 0; i < n; ++i) {
     const nmv_case &c = cases[i];
     put_t(c.cand);

@@ -419,10 +419,22 @@ __global__ void __launch_bounds__(kFinThreads, 2) finalize_kernel(const CaseDesc
     move_words(o + cd.rowp_off, ho + cd.rowp_off, cd.rowp_n, y, nb);
     move_words(o + cd.colp_off, ho + cd.colp_off, cd.colp_n, y, nb);
     if (blockIdx.x == 0 && y == 0) {
-      move_words(out, hout, kCallHeader / 8, 0, 1);
+      // the call header to the host block; its words back to zero except the
+      // scan's error word, which every block reads below (a failed call's
+      // accumulators are cleared by the host before the next call)
+      unsigned long long *src = (unsigned long long *)out, *dst = (unsigned long long *)hout;
+      for (int t = threadIdx.x; t < (int)(kCallHeader / 8); t += kFinThreads) {
+        const unsigned long long v = src[t];
+        dst[t] = v;
+        if (v && t != (int)(kCallErrOff / 8)) src[t] = 0ull;
+      }
       for (size_t t = threadIdx.x; t < zthr_bytes / 8; t += kFinThreads) ((unsigned long long *)zthr)[t] = 0ull;
     }
   }
+  // A scan that gave up waiting for its copies left batch counts and
+  // partials incomplete (the call is void and reports NMV_ETIMEOUT): nothing
+  // more is read.
+  if (*(volatile const uint32_t *)(out + kCallErrOff) != 0) return;
   __shared__ int64_t sh_scan[kFinThreads / 32 + 1];
   __shared__ int64_t sh_mism;
   __shared__ FkItem sh_need[kFinChunk], sh_item[kFinChunk];

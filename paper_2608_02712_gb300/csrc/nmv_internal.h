@@ -87,7 +87,8 @@ struct CaseDesc {
   // the candidate's shape as divisors, for the records' coordinates
   // (written at byte coord_off of the host result when the finalize writes
   // there; a zero extent has d = 0)
-  int32_t rank, pad1;
+  int32_t rank;
+  int32_t test_stall;                  // test hook of the scan's wait limit (NMV_FAULT_INJECT=stall)
   Div64 sdiv[NMV_MAX_RANK];
   int64_t coord_off;
 };

@@ -1308,19 +1308,35 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   reload_thr(R, W);
 }
 
+// The bins of a batch in the dense regime, when the batch lies in one row
+// of the [M, N] view (aligned localisation and N a multiple of the batch):
+// its row bin and the histogram bin of its first tile, computed once per
+// batch; the batch's mismatch count, row total and step bits accumulate in
+// registers and are added at the end of the batch.
+struct DenseBins {
+  int32_t ok;        // this batch uses them
+  int32_t rp;        // row bin
+  int64_t hb;        // histogram bin of the batch's first tile (window or global index)
+  int32_t rowsum;    // mismatches recorded this way in this batch
+  uint32_t sbits;    // their warp steps
+};
+
 // A float step of a warp in the dense regime (its last batch was mostly
-// mismatches, as where a candidate passes an input through): the hard
-// step's one classification pass (TwoSum of c - r, the sure-pass and
-// sure-fail bounds, the maximum thresholds) runs inline, and when every
-// element of the warp is dense (finite, decided by the fp32 bounds, no
-// candidate for a maximum) the SSE terms, the mismatch count and the maps
-// are done here too, with the hard step's arithmetic; any other step goes
-// out of line as usual.  A clean step takes this path's SSE arithmetic
-// with e = 0, which is the fast path's, so results do not depend on the
-// regime.
+// mismatches, as where a candidate passes an input through): one inline
+// pass classifies every element with the TwoSum of c - r, the sure-pass and
+// sure-fail bounds, and the maximum thresholds shrunk by the 2^-20 margin
+// (|d| <= |s| (1 + 2^-24), so |s| <= tA (1 - 2^-20) proves |d| < tA, and
+// |s| <= rz(|r| tR (1 - 2^-20)) proves |d| / |r| < tR: no new maximum,
+// whether or not c - r is exact).  When every element of the warp is dense
+// (finite, decided by the fp32 bounds, no candidate for a maximum) the SSE
+// terms (the hard step's arithmetic), the mismatch count and the maps are
+// done here too; any other step goes out of line as usual.  A clean step
+// takes this path's SSE arithmetic with e = 0, which is the fast path's, so
+// results do not depend on the regime.
 template <int DT, int NIN>
-__device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const uint4 &cv,
-                                           const uint4 &rv, const uint4 &xv, uint32_t erel) {
+__device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, DenseBins &B,
+                                           const uint4 &cv, const uint4 &rv, const uint4 &xv, uint32_t erel,
+                                           int u) {
   constexpr int V = Tr<DT>::V;
   const long long t_start = P->stats ? clock64() : 0;
   if (R.track_c) R.cacc |= (cv.x ^ R.cpat) | (cv.y ^ R.cpat) | (cv.z ^ R.cpat) | (cv.w ^ R.cpat);
@@ -1338,8 +1354,9 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
   const float2 lo_r2 = make_float2(R.lo_r, R.lo_r), lo_a2 = make_float2(R.lo_a, R.lo_a);
   const float hr = P->cd.hi_r, ha = P->cd.hi_a;
   const float2 hi_r2 = make_float2(hr, hr), hi_a2 = make_float2(ha, ha);
-  const float tA = R.tA;
-  const float2 tR2 = make_float2(R.tR, R.tR);
+  const float tAm = __fmul_rz(R.tA, kMarginLo);
+  const float tRm = __fmul_rz(R.tR, kMarginLo);
+  const float2 tR2 = make_float2(tRm, tRm);
   float2 s[V / 2], e[V / 2];
   bool dense = true;
   uint32_t mask = 0;
@@ -1357,12 +1374,11 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
     const float2 h2 = __ffma2_ru(ar2, hi_r2, hi_a2);
     const float2 t2 = __fmul2_rz(ar2, tR2);
     const float as0 = fabsf(s2.x), as1 = fabsf(s2.y);
-    dense &= (as0 <= a2.x || as0 > h2.x) && (as0 < tA || (as0 == tA && e[j].x == 0.f)) &&
-             as0 <= (e[j].x == 0.f ? t2.x : __fmul_rz(t2.x, kMarginLo));
-    dense &= (as1 <= a2.y || as1 > h2.y) && (as1 < tA || (as1 == tA && e[j].y == 0.f)) &&
-             as1 <= (e[j].y == 0.f ? t2.y : __fmul_rz(t2.y, kMarginLo));
-    if (!(as0 <= a2.x)) mask |= 1u << (2 * j);
-    if (!(as1 <= a2.y)) mask |= 2u << (2 * j);
+    const bool p0 = as0 <= a2.x, p1 = as1 <= a2.y;
+    dense &= (p0 || as0 > h2.x) && as0 <= tAm && as0 <= t2.x;
+    dense &= (p1 || as1 > h2.y) && as1 <= tAm && as1 <= t2.y;
+    if (!p0) mask |= 1u << (2 * j);
+    if (!p1) mask |= 2u << (2 * j);
   }
   if (!__all_sync(0xffffffffu, dense)) {
     R.sse = hard_step<DT>(P, L, W, cv, rv, P->pbegin + erel, R.sse);
@@ -1381,7 +1397,42 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
     R.sse.lo = __fadd2_rn(R.sse.lo, __fadd2_rn(err, q));
     R.sse.hi = t;
   }
-  if (__any_sync(0xffffffffu, mask != 0)) {
+  if (B.ok) {
+    // the batch's bins: the step's tiles follow the batch's first one
+    const int lane = threadIdx.x & 31;
+    const int cnt = __popc(mask);
+    const int total = __reduce_add_sync(0xffffffffu, (unsigned)cnt);
+    if (total) {
+      const int sh = P->cd.a_shift;
+      int gsum = cnt;
+      if (sh == 5) {
+        gsum = total;
+      } else {
+        for (int o = 1; o < (1 << sh); o <<= 1) gsum += __shfl_xor_sync(0xffffffffu, gsum, o);
+      }
+      if (gsum != 0 && (lane & ((1 << sh) - 1)) == 0) {
+        // the step holds 32 >> sh tiles (STEP / tw with tw = V 2^sh)
+        const int64_t hb = B.hb + (int64_t)u * (32 >> sh) + (lane >> sh);
+        if (P->wr > 0) sh_add(&P->sh_hist[hb], gsum);
+        else gl_add(&P->g_hist[hb], (unsigned long long)gsum);
+      }
+      B.rowsum += total;
+      B.sbits |= 1u << u;
+      if (mask) {
+        const uint32_t a = P->lcol_sa + (uint32_t)threadIdx.x * (V * 4);
+#pragma unroll
+        for (int j = 0; j < V; j += 4) {
+          int x, y, z, w;
+          asm volatile("ld.shared.v4.s32 {%0,%1,%2,%3}, [%4];" : "=r"(x), "=r"(y), "=r"(z), "=r"(w) : "r"(a + 4 * j));
+          x += (mask >> j) & 1u;
+          y += (mask >> (j + 1)) & 1u;
+          z += (mask >> (j + 2)) & 1u;
+          w += (mask >> (j + 3)) & 1u;
+          asm volatile("st.shared.v4.s32 [%0], {%1,%2,%3,%4};" ::"r"(a + 4 * j), "r"(x), "r"(y), "r"(z), "r"(w));
+        }
+      }
+    }
+  } else if (__any_sync(0xffffffffu, mask != 0)) {
     if (P->cd.amode) record_step_aligned<V>(P, W, mask, P->pbegin + erel);
     else record_step(P, W, mask, P->pbegin + erel, V);
   }
@@ -1394,9 +1445,11 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
 // (bytes = 0) are read from global memory by tail_step.
 template <int NIN>
 __device__ __forceinline__ void ring_issue(const char *c, const char *r, const char *x, uint32_t off,
-                                           uint32_t bytes, uint8_t *stage, uint64_t *bar) {
+                                           uint32_t bytes, uint8_t *stage, uint64_t *bar, bool stall) {
   mbar_arrive_tx(bar, bytes * (NIN == 1 ? 3u : 2u));
-  if (bytes) {
+  // (stall: the test hook of the wait limit announces the bytes and issues
+  // no copy, so the stage never completes and nothing is in flight)
+  if (bytes && !stall) {
     const uint64_t pol = evict_first_policy();
     bulk_load(stage, c + off, bytes, bar, pol);
     bulk_load(stage + stage_bytes(NIN), r + off, bytes, bar, pol);
@@ -1437,7 +1490,7 @@ __device__ __forceinline__ void sse_flush(SseAcc &a) {
 // Offsets within the piece are 32-bit (a piece holds at most kMaxPiece
 // elements).
 template <int DT, int NIN>
-__device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
+__device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN> &R, const Piece &pc,
                                       int32_t *batch_count, uint8_t *ring, uint64_t *bars, RingPos &rp,
                                       uint32_t *err) {
   constexpr int V = Tr<DT>::V;
@@ -1482,7 +1535,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     uint32_t bytes = 0;
     if (vec_ok && off < pbytes) bytes = pbytes - off >= HB ? HB : (pbytes - off) / (STEP * EB) * (STEP * EB);
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i);
+    ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i, P->cd.test_stall != 0);
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
     if (h_i == 0) {
       h_i = 1;
@@ -1497,7 +1550,6 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     W->mism_tot = 0;
   }
   __syncwarp();
-  bool dead = false;
   // The block's view of the case-wide maxima is read every batch; the case's
   // own value is read by one warp of the block per batch round (each warp
   // every kPoll batches, its load kPoll batches ahead of its use, so the L2
@@ -1507,6 +1559,10 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   int flush = 0;
   // warp-uniform: the warp's last batch was mostly mismatches (float types)
   bool dmode = false;
+  // the batch's bins can be computed once when every batch lies in one row
+  const bool bins_ok = P->cd.amode && P->cd.dN.d % (uint64_t)BATCH == 0;
+  DenseBins B;
+  B.ok = 0;
   for (uint32_t j = 0;; ++j) {
     const uint32_t b = W->stage_b[rp.stage];
     if (b == kNoBatch) break;
@@ -1515,6 +1571,21 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     if (lane == 0) {
       W->mism = 0;
       W->sbits = 0;
+    }
+    B.ok = 0;
+    if (Tr<DT>::EB == 4 && !Tr<DT>::kInt && dmode && bins_ok) {
+      // row, row bin and first tile of the batch (all lanes alike)
+      const CaseDesc &cd = P->cd;
+      const uint32_t s0 = (uint32_t)P->pbegin + erel;
+      const uint32_t N = (uint32_t)cd.dN.d, th = (uint32_t)cd.dth.d, tw = (uint32_t)cd.dtw.d;
+      const uint32_t row = div_q32(s0, N, cd.m32N);
+      const uint32_t tr = div_q32(row, th, cd.m32th);
+      const uint32_t tc = div_q32(s0 - row * N, tw, cd.m32tw);
+      B.ok = 1;
+      B.rp = (int32_t)(row - tr * th);
+      B.hb = P->wr > 0 ? ((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0) : (int64_t)tr * cd.GC + tc;
+      B.rowsum = 0;
+      B.sbits = 0;
     }
     if ((j + warp) % kPoll == 0) {
       if (lane == 0) {
@@ -1547,11 +1618,25 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       if (lane == 0 && live) issue_next();  // refills the stage released before this one
       __syncwarp();
       const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
-      if (!dead && !mbar_try_wait(bars + rp.stage, rp.phase)) {
-        if (!mbar_wait_slow(bars + rp.stage, rp.phase)) {
-          dead = true;  // report, and stop waiting (the data of this call is void)
-          if (lane == 0) atomicOr(err, 1u);
+      bool ok = mbar_try_wait(bars + rp.stage, rp.phase);
+      if (!__all_sync(0xffffffffu, ok)) ok = mbar_wait_slow(bars + rp.stage, rp.phase);
+      if (!__all_sync(0xffffffffu, ok)) {
+        // A stage's copies did not complete within the wait limit: report
+        // (the data of this call is void), wait again, with the same limit,
+        // for this warp's copies still in flight (this stage's and those of
+        // the stage issued ahead of it), so none lands in shared memory after
+        // the block has stopped, mark the warp's remaining batches empty,
+        // and stop.
+        if (lane == 0) atomicOr(err, 1u);
+        mbar_wait_slow(bars + rp.stage, rp.phase);
+        const uint32_t nx = rp.stage + 1 == NST ? 0u : rp.stage + 1;
+        const uint32_t nph = rp.stage + 1 == NST ? rp.phase ^ 1u : rp.phase;
+        if (W->stage_b[nx] != kNoBatch) mbar_wait_slow(bars + nx, nph);
+        if (lane == 0) {
+          for (uint32_t jj = j; jj < nj; ++jj) bcount[jj * kWarps + (((uint32_t)warp + kWarps - jj % kWarps) % kWarps)] = 0;
         }
+        __syncwarp();
+        return true;
       }
       if (++rp.stage == NST) {
         rp.stage = 0;
@@ -1568,7 +1653,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
             uint4 xv = make_uint4(0, 0, 0, 0);
             if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
             if constexpr (Tr<DT>::EB == 4 && !Tr<DT>::kInt)
-              step_dense<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
+              step_dense<DT, NIN>(P, L, W, R, B, cv, rv, xv, hrel + u * STEP + lane_off, h * HS + u);
           }
         } else {
 #pragma unroll 2
@@ -1601,6 +1686,16 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       }
       __syncwarp();  // every lane is done with the stage before it is refilled
     }
+    if (B.ok && B.rowsum) {
+      // the dense steps' row total and counts (all lanes hold them)
+      if (lane == 0) {
+        if (P->prof_smem) sh_add(&P->sh_row[B.rp], B.rowsum);
+        else gl_add(&P->g_row[B.rp], (unsigned long long)B.rowsum);
+        W->mism += B.rowsum;
+        W->sbits |= B.sbits;
+      }
+      __syncwarp();
+    }
     if (lane == 0) {
       bcount[b] = (int32_t)((uint32_t)W->mism | (W->sbits << kStepBitsShift));
       W->mism_tot += W->mism;
@@ -1622,6 +1717,7 @@ __device__ __forceinline__ void sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     }
   }
   sse_flush(R.sse);
+  return false;
 }
 
 // ------------------------------------------------------------ seeding
@@ -1719,16 +1815,18 @@ __global__ void __launch_bounds__(kThreads, 2)
   __shared__ int32_t sh_done;    // warps done with the current sweep
   __shared__ int32_t sh_newcase;  // the current piece starts a case for this block
   __shared__ uint32_t sh_pat[2];  // the case's first stored words (replicated for 16-bit types)
+  __shared__ int32_t sh_abort;    // a warp gave up waiting for its copies: the block stops
   if (threadIdx.x == 0) {
     const int64_t p0 = (int64_t)atomicAdd(piece_ctr, 1ull);
     sh_piece = p0;
     if (p0 < n_pieces) sh_pc = pieces[p0];
     sh_case = -1;
+    sh_abort = 0;
   }
   for (;;) {
     __syncthreads();
     const int64_t p = sh_piece;
-    if (p >= n_pieces) break;
+    if (p >= n_pieces || sh_abort) break;
     const Piece pc = sh_pc;
     const bool newcase = sh_case != pc.case_id;
     if (newcase) {
@@ -1850,7 +1948,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     R.lo_r = P.cd.lo_r;
     R.lo_a = P.cd.lo_a;
     R.track_c = R.track_r = true;
-    sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err);
+    if (sweep<DT, NIN>(&P, L, W, R, pc, batch_count, ring, bars, rpos, err) && lane == 0) sh_abort = 1;
     if (P.cd.amode) {
       // this lane's column counters into the column profile
       constexpr int V = Tr<DT>::V;
