@@ -1314,9 +1314,9 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
 // batch; the batch's mismatch count, row total and step bits accumulate in
 // registers and are added at the end of the batch.
 struct DenseBins {
-  int32_t ok;        // this batch uses them
+  int32_t ok;        // 0: not used this batch; 1: histogram window in shared memory; 2: global histogram
   int32_t rp;        // row bin
-  int64_t hb;        // histogram bin of the batch's first tile (window or global index)
+  uint32_t hbin;     // the batch's first tile bin: shared address (ok 1) or global index (ok 2, < 2^26)
   int32_t rowsum;    // mismatches recorded this way in this batch
   uint32_t sbits;    // their warp steps
 };
@@ -1412,9 +1412,9 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
       }
       if (gsum != 0 && (lane & ((1 << sh) - 1)) == 0) {
         // the step holds 32 >> sh tiles (STEP / tw with tw = V 2^sh)
-        const int64_t hb = B.hb + (int64_t)u * (32 >> sh) + (lane >> sh);
-        if (P->wr > 0) sh_add(&P->sh_hist[hb], gsum);
-        else gl_add(&P->g_hist[hb], (unsigned long long)gsum);
+        const uint32_t t = (uint32_t)u * (32u >> sh) + (uint32_t)(lane >> sh);
+        if (B.ok == 1) sh_add_at(B.hbin + 4 * t, gsum);
+        else gl_add(P->g_hist + (B.hbin + t), (unsigned long long)gsum);
       }
       B.rowsum += total;
       B.sbits |= 1u << u;
@@ -1581,9 +1581,14 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       const uint32_t row = div_q32(s0, N, cd.m32N);
       const uint32_t tr = div_q32(row, th, cd.m32th);
       const uint32_t tc = div_q32(s0 - row * N, tw, cd.m32tw);
-      B.ok = 1;
       B.rp = (int32_t)(row - tr * th);
-      B.hb = P->wr > 0 ? ((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0) : (int64_t)tr * cd.GC + tc;
+      if (P->wr > 0) {
+        B.ok = 1;
+        B.hbin = smem_addr(P->sh_hist + (((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0)));
+      } else {
+        B.ok = 2;
+        B.hbin = (uint32_t)((int64_t)tr * cd.GC + tc);
+      }
       B.rowsum = 0;
       B.sbits = 0;
     }
