@@ -192,9 +192,9 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
  *    scalar field of *out, and leaves the pointers as they were.
  *
  * A case needs about: 4 bytes per batch of 2048 (16-bit types) or 1024
- * (32-bit types) elements (half that with one input of the candidate's type
- * and size), 8 bytes per histogram bin, 8 * (tile_rows + tile_cols) + 24 *
- * first_k bytes, and under 1 MiB of descriptors and partials.  A case that
+ * (32-bit types) elements, 8 bytes per histogram bin, 8 * (tile_rows +
+ * tile_cols) + 24 * first_k bytes, and under 1 MiB of descriptors and
+ * partials.  A case that
  * does not fit fails with NMV_EINVAL and a message giving the bytes it needs
  * (nmv_validate has no such limit).
  *

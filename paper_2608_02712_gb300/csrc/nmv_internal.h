@@ -142,14 +142,16 @@ struct OutHeader {
 #define NMV_CHD constexpr
 #endif
 
-// Warp steps (32 lanes x 16 bytes of each tensor) per batch, by input class
-// (0, 1 or -1 = several inputs read from global memory; one staged input
-// leaves shared memory for shorter batches only), and elements per batch.  A
-// batch is the unit of the first-K counts and of the scan's bookkeeping; it
-// streams through a warp's shared-memory ring as two stages of half a batch.
+// Warp steps (32 lanes x 16 bytes of each tensor) per batch, and per ring
+// stage, by input class (0, 1 or -1 = several inputs read from global
+// memory), and elements per batch.  A batch is the unit of the first-K
+// counts and of the scan's bookkeeping; it streams through a warp's
+// two-stage shared-memory ring as batch_steps / stage_steps stages: two of
+// four steps, or, with one staged input (three tensors in each stage), four
+// of two steps, so the ring's shared memory stays the same.
 constexpr int kMaxSteps = 8;
-NMV_CHD int batch_steps(int nin) { return nin == 1 ? 4 : 8; }
-NMV_CHD int stage_steps(int nin) { return batch_steps(nin) / 2; }
+NMV_CHD int batch_steps(int) { return 8; }
+NMV_CHD int stage_steps(int nin) { return nin == 1 ? 2 : 4; }
 // A batch's entry in the batch-count array: its mismatch count (below 2^24)
 // in the low bits, and from bit kStepBitsShift the warp steps that hold them.
 constexpr int kStepBitsShift = 24;

@@ -1500,7 +1500,8 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   constexpr int HS = stage_steps(NIN);
   constexpr int BATCH = STEP * KS;
   constexpr uint32_t BB = BATCH * EB;          // bytes of one tensor's batch
-  constexpr uint32_t HB = stage_bytes(NIN);    // bytes of one tensor's stage (half a batch)
+  constexpr uint32_t HB = stage_bytes(NIN);    // bytes of one tensor's stage
+  constexpr uint32_t NSB = KS / HS;            // stages per batch
   constexpr uint32_t NST = ring_stages(NIN);
   constexpr int STAGE = ring_streams(NIN) * stage_bytes(NIN);
   constexpr int kPoll = kWarps;  // batches between a warp's readings of the case-wide maxima
@@ -1537,9 +1538,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i, P->cd.test_stall != 0);
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
-    if (h_i == 0) {
-      h_i = 1;
-    } else {
+    if (++h_i == NSB) {
       h_i = 0;
       ++j_i;
       rot_i = (rot_i + kWarps - 1) & (kWarps - 1);
@@ -1619,7 +1618,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       }
     }
 #pragma unroll 1
-    for (int h = 0; h < 2; ++h) {
+    for (int h = 0; h < (int)NSB; ++h) {
       if (lane == 0 && live) issue_next();  // refills the stage released before this one
       __syncwarp();
       const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
