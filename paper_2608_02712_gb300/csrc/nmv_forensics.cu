@@ -4,21 +4,27 @@
 // a divergence that compounds along a reduction axis (Section 3.2, the
 // cumsum of Table 1), and mismatch counts at every index of every axis.
 //
-// fx_kernel streams the pair once (16-byte loads, four in flight per lane).
-// Per element it takes the predicate with the scan's fp32 pre-filter (fp64
-// where the filter cannot decide), the ulp distance u of the two stored
-// values, and for mismatches the fp16-spacing test and the coordinates.
-// Lane-private ulp histograms sit in shared memory (stride 35 words, so the
-// 32 lanes of a warp hit 32 banks); the growth curve max |c - r| per index
-// of the chosen axis is screened in fp32 against a lower bound of the bin's
-// maximum and made exact in fp64 only for candidates (maxima do not depend
-// on the order, so atomics keep them exact); the marginals are privatised
-// in shared memory when they fit.  fx_fin_kernel reduces the blocks'
-// largest-ulp candidates in block order and writes every field into the
-// mapped host result.
+// fx_kernel streams the pair once, viewed as R rows of L elements (L the
+// last axis), in units of rb rows x g column windows handed to warps from a
+// counter.  A window is 32 vectors wide and lane l owns the same V columns
+// in every row of it, so the last axis' mismatch marginal (and, when the
+// growth axis is the last one, the growth maxima of those columns) stay in
+// the lane's registers until the window ends; the leading axes' marginals
+// take one warp sum per row.  Per element: the predicate with the scan's
+// fp32 pre-filter (fp64 where the filter cannot decide), the ulp distance of
+// the two stored values into a lane-private shared-memory histogram (stride
+// 35 words, so the 32 lanes of a warp hit 32 banks), and for mismatches the
+// largest-ulp record and the fp16-spacing test, decided exactly from the
+// fp32 difference and its TwoSum remainder.  The growth curve max |c - r|
+// per index of the chosen axis is kept exact as (|fl32(c - r)|, remainder)
+// pairs and written as fp64 maxima with atomics (maxima do not depend on
+// the order) after an fp32 screen against each bin's lower bound.
+// fx_fin_kernel reduces the blocks' largest-ulp candidates in block order
+// and writes every field into the mapped host result.
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cfloat>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -30,22 +36,28 @@
 namespace nmv {
 
 constexpr int kFxThreads = 256;
-constexpr int kFxHistStride = 35;     // words per lane histogram (34 bins, odd stride)
+constexpr int kFxHistBytes = (kFxThreads / 32) * NMV_ULP_BINS * 32 * 4;  // [warp][bin][lane] ulp histograms
+constexpr int64_t kFxRowsMax = 256;   // rows of a unit at most
+constexpr int kFxRowBytes = (kFxThreads / 32) * (int)kFxRowsMax * 4;  // [warp][row] mismatch counts
 constexpr int64_t kFxGrowCap = 2048;  // growth bins privatised in shared memory
 constexpr int64_t kFxMargCap = 4096;  // marginal bins privatised in shared memory
+constexpr int64_t kFxUnitElems = 65536;  // elements of a unit (rows x window columns), when the rows allow
 
 struct FxDesc {
   const void *cand, *ref;
-  int32_t dtype, vec_ok;
+  int32_t dtype, vec_ok;    // vec_ok: every row of the [R, L] view starts 16-byte aligned in both tensors
   int32_t rank, axis;
-  int32_t idx32, grow_smem, marg_smem, pad;
+  int32_t grow_smem, marg_smem, j_is_row, pad;
   int64_t numel;
+  int64_t L, R;             // the pair as R rows of L elements (L the last axis; 1 x 1 for rank 0)
+  int64_t CWn, rb, g, WG;   // column windows of 32 vectors; a unit is rb rows x g windows
+  int64_t n_units;
   int64_t shape[NMV_MAX_RANK];
   Div64 sdiv[NMV_MAX_RANK];
   int64_t marg_off[NMV_MAX_RANK + 1];
   int64_t axis_len;
   Div64 dstride, dlen;      // coordinate on the axis: (i / stride) % len
-  uint32_t m32stride, m32len;
+  Div64 drs;                // growth axis before the last: rows per index (row rho -> (rho / rs) % len)
   float lo_r, lo_a, hi_r, hi_a;  // fp32 pre-filter of the predicate (as nmv_validate)
   double rtol, atol;
   int64_t near_ulps;
@@ -57,145 +69,227 @@ struct FxDesc {
 struct FxAcc {
   unsigned long long hist[NMV_ULP_BINS];
   unsigned long long mismatch, n_finite, nonfin, within;
+  unsigned long long unit_ctr;  // units handed out
 };
 
 struct FxBest {
   long long u, idx;  // largest ulp distance of a finite mismatch (-1: none) and its lowest index
 };
 
-__device__ __forceinline__ long long ord_bits(uint32_t b, int dt) {
-  if (dt == NMV_I32) return (long long)(int32_t)b;
-  const int width = elem_bytes(dt) * 8;
-  const uint32_t sign = (b >> (width - 1)) & 1u;
-  const long long mag = (long long)(b & (width == 32 ? 0x7fffffffu : 0x7fffu));
-  return sign ? -mag : mag;
-}
-
-// One fp16 spacing at |r| (r finite): 2^(max(floor(log2 |r|), -14) - 10),
-// 2^-24 at 0.  Values of these types are normal in fp64, so floor(log2 |r|)
-// is the fp64 exponent field less the bias.
-__device__ __forceinline__ double f16_spacing(double r) {
-  if (r == 0.0) return 0x1p-24;
-  const int e = (int)((__double_as_longlong(fabs(r)) >> 52) & 0x7ff) - 1023;
-  return ldexp(1.0, max(e, -14) - 10);
-}
-
-// The predicate of nmv_validate: the fp32 pre-filter decides where it can,
-// fp64 otherwise.
-template <int DT>
-__device__ __forceinline__ bool fx_pass(const FxDesc &d, uint32_t cb, uint32_t rb) {
-  if constexpr (Tr<DT>::kInt) {
-    if (cb == rb) return true;
-    const long long df = (long long)(int32_t)cb - (long long)(int32_t)rb;
-    const float as = fabsf(__ll2float_rn(df)), ar = fabsf(to_f32<DT>(rb));
-    if (as <= __fmaf_rz(d.lo_r, ar, d.lo_a)) return true;
-    if (as > __fmaf_ru(d.hi_r, ar, d.hi_a)) return false;
-  } else {
-    const float cf = to_f32<DT>(cb), rf = to_f32<DT>(rb);
-    if (cf == rf) return true;
-    if (!(isfinite(cf) && isfinite(rf))) return false;
-    const float as = fabsf(__fsub_rn(cf, rf)), ar = fabsf(rf);
-    if (as <= __fmaf_rz(d.lo_r, ar, d.lo_a)) return true;
-    if (as > __fmaf_ru(d.hi_r, ar, d.hi_a)) return false;
-  }
-  return pass64(to_f64<DT>(cb), to_f64<DT>(rb), d.rtol, d.atol);
-}
-
+// Per-lane totals.  A lane sees at most numel / 32 elements, below 2^32 for
+// any pair that fits in device memory.
 struct FxLane {
   uint32_t mism, nfin, nonfin, within;
-  long long bu, bi;
+  uint32_t bu;   // largest ulp distance of a finite mismatch (0: none; a finite mismatch has u >= 1)
+  int64_t bi;    // its lowest index
 };
 
-// The coordinate of element i on the growth axis.
-__device__ __forceinline__ int64_t axis_coord(const FxDesc &d, int64_t i) {
-  if (d.rank == 0) return 0;
-  if (d.idx32) {
-    const uint32_t q = div_q32((uint32_t)i, (uint32_t)d.dstride.d, d.m32stride);
-    return q - div_q32(q, (uint32_t)d.dlen.d, d.m32len) * (uint32_t)d.dlen.d;
+// Sign-magnitude bits -> a signed integer that orders like the values, both
+// zeros at 0 (two's complement int32 as it is).
+template <int DT>
+__device__ __forceinline__ int32_t ord32(uint32_t b) {
+  if constexpr (Tr<DT>::kInt) {
+    return (int32_t)b;
+  } else {
+    constexpr uint32_t kMag = Tr<DT>::EB == 2 ? 0x7fffu : 0x7fffffffu;
+    constexpr int kSign = Tr<DT>::EB == 2 ? 15 : 31;
+    const int32_t m = (int32_t)(b & kMag);
+    return ((b >> kSign) & 1u) ? -m : m;
   }
-  const uint64_t q = div_q((uint64_t)i, d.dstride.d, d.dstride.m);
-  return (int64_t)(q - div_q(q, d.dlen.d, d.dlen.m) * d.dlen.d);
 }
 
+// |ord(c) - ord(r)|: below 2^32 for every type (fp32 magnitudes of finite
+// values are at most 0x7f7fffff).
 template <int DT>
-__device__ __forceinline__ void fx_elem(const FxDesc &d, FxLane &L, uint32_t cb, uint32_t rb, int64_t i,
-                                        int32_t *hist, unsigned long long *gmax, uint32_t *glb, uint32_t *smarg,
-                                        unsigned long long *gmarg) {
-  bool fin = true;
-  float as32;
+__device__ __forceinline__ uint32_t ulp_dist(uint32_t cb, uint32_t rb) {
+  const int32_t a = ord32<DT>(cb), b = ord32<DT>(rb);
+  return a >= b ? (uint32_t)a - (uint32_t)b : (uint32_t)b - (uint32_t)a;
+}
+
+// t with a - b = s + t exactly, s = fl32(a - b) finite (TwoSum; the
+// intrinsics keep every step a separately rounded operation).
+__device__ __forceinline__ float twosum_err(float a, float b, float s) {
+  const float nb = -b;
+  const float bb = __fsub_rn(s, a);
+  return __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(nb, bb));
+}
+
+// A running maximum of |c - r| (the growth curve).  Float types: the exact
+// value as S + T, S = |fl32(c - r)| and T the TwoSum remainder signed
+// toward S.  |T| is at most half an ulp of S (a quarter below a power of
+// two), so the pairs order lexicographically like the exact values, and
+// fl64(S + T) is the fp64 |c - r| (one rounding of the exact value).
+// int32: the exact |c - r| (below 2^32).
+template <int DT, bool INT = Tr<DT>::kInt>
+struct GAcc {
+  float S = 0.f, T = 0.f;
+};
+template <int DT>
+struct GAcc<DT, true> {
+  uint32_t U = 0u;
+};
+
+// An element whose fp32 difference overflowed (|c - r| > FLT_MAX, c and r
+// finite): its fp64 |c - r| goes straight to the growth bin of its index.
+__device__ __noinline__ void grow_direct(const FxDesc &d, int64_t i, double v, unsigned long long *gmax,
+                                         uint32_t *glb) {
+  int64_t j = 0;
+  if (d.rank > 0) {
+    const uint64_t q = div_q((uint64_t)i, d.dstride.d, d.dstride.m);
+    j = (int64_t)(q - div_q(q, d.dlen.d, d.dlen.m) * d.dlen.d);
+  }
+  atomicMax(&gmax[j], (unsigned long long)__double_as_longlong(v));
+  atomicMax(&glb[j], __float_as_uint(__double2float_rd(v)));
+}
+
+// One maximum at growth index j, unless the bin's fp32 lower bound already
+// exceeds it: fl32(S (1 + 2^-22)) is above S + |T| (and fl32(U) is within
+// 2^-24 of U).
+template <int DT>
+__device__ __forceinline__ void grow_flush(const GAcc<DT> &g, int64_t j, unsigned long long *gmax, uint32_t *glb) {
+  double v;
   if constexpr (Tr<DT>::kInt) {
-    const long long df = (long long)(int32_t)cb - (long long)(int32_t)rb;
-    as32 = __ll2float_rn(df < 0 ? -df : df);
+    if (g.U == 0u || __fmul_rn(__uint2float_rn(g.U), 1.0f + 0x1p-22f) < __uint_as_float(glb[j])) return;
+    v = (double)g.U;
+  } else {
+    if (g.S == 0.f || __fmul_rn(g.S, 1.0f + 0x1p-22f) < __uint_as_float(glb[j])) return;
+    v = __dadd_rn((double)g.S, (double)g.T);
+  }
+  atomicMax(&gmax[j], (unsigned long long)__double_as_longlong(v));
+  atomicMax(&glb[j], __float_as_uint(__double2float_rd(v)));
+}
+
+// A float pair's exact |c - r| into a running maximum (S, T).
+template <typename GA>
+__device__ __forceinline__ void gacc_add(GA &g, float cf, float rf, float s, float as) {
+  const float t = twosum_err(cf, rf, s), tp = s > 0.f ? t : -t;
+  if (as > g.S || tp > g.T) {
+    g.S = as;
+    g.T = tp;
+  }
+}
+
+// One element: counts, ulp histogram, growth, the predicate (the scan's
+// fp32 pre-filter, fp64 where it cannot decide) and, for a mismatch, the
+// largest-ulp record and the fp16-spacing test.  Returns true on mismatch.
+// Growth: with AXL the element's column maximum g is made exact at once
+// when the element can raise it; otherwise rmax takes |fl32(c - r)| and
+// the row's exact maximum is found at the row's end.
+template <int DT, bool AXL, typename GA>
+__device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, uint32_t rb, int64_t i,
+                                      int32_t *hist, GA &g, float &rmax, unsigned long long *gmax, uint32_t *glb) {
+  if constexpr (Tr<DT>::kInt) {
+    const int32_t c = (int32_t)cb, r = (int32_t)rb;
+    const uint32_t u = ulp_dist<DT>(cb, rb);  // = |c - r|
+    ++L.nfin;
+    hist[32 * (u ? 32 - __clz(u) : 0)] += 1;
+    g.U = max(g.U, u);
+    if (u == 0u) return false;
+    const float as = __uint2float_rn(u), ar = fabsf(__int2float_rn(r));
+    bool pass;
+    if (as <= __fmaf_rz(d.lo_r, ar, d.lo_a)) pass = true;
+    else if (as > __fmaf_ru(d.hi_r, ar, d.hi_a)) pass = false;
+    else pass = pass64((double)c, (double)r, d.rtol, d.atol);
+    if (pass) return false;
+    ++L.mism;
+    if (u > L.bu || (u == L.bu && i < L.bi)) {
+      L.bu = u;
+      L.bi = i;
+    }
+    // one fp16 spacing 2^(max(floor(log2 |r|), -14) - 10) is below 1 for
+    // |r| < 2^10, where no integer mismatch lies within it
+    const uint32_t mr = r < 0 ? 0u - (uint32_t)r : (uint32_t)r;
+    if (mr >= 1024u && u <= (1u << (21 - __clz(mr)))) ++L.within;
+    return true;
   } else {
     const float cf = to_f32<DT>(cb), rf = to_f32<DT>(rb);
-    fin = isfinite(cf) && isfinite(rf);
-    as32 = fabsf(__fsub_rn(cf, rf));
-  }
-  long long u = ord_bits(cb, DT) - ord_bits(rb, DT);
-  u = u < 0 ? -u : u;
-  if (fin) {
-    ++L.nfin;
-    const int bin = u == 0 ? 0 : min(64 - __clzll(u), NMV_ULP_BINS - 1);
-    hist[bin] += 1;
-    // growth: fl32 |c - r| is within 2^-24 of the exact |c - r|, so an
-    // element whose as32 (1 + 2^-22) lies below the bin's lower bound is no
-    // new maximum; the others are evaluated exactly in fp64
-    if (as32 > 0.f) {
-      const int64_t j = axis_coord(d, i);
-      if (!(__fmul_rn(as32, 1.0f + 0x1p-22f) < __uint_as_float(glb[j]))) {
-        const double dv = fabs(__dsub_rn(to_f64<DT>(cb), to_f64<DT>(rb)));
-        atomicMax(&gmax[j], (unsigned long long)__double_as_longlong(dv));
-        atomicMax(&glb[j], __float_as_uint(__double2float_rd(dv)));
+    const float s = __fsub_rn(cf, rf), as = fabsf(s);
+    const bool fin = fabsf(cf) <= FLT_MAX && fabsf(rf) <= FLT_MAX;
+    const uint32_t u = ulp_dist<DT>(cb, rb);  // meaningful for finite pairs
+    L.nfin += fin ? 1u : 0u;
+    hist[32 * (u ? 32 - __clz(u) : 0)] += fin ? 1 : 0;
+    if constexpr (AXL) {
+      if (fin && as >= g.S) {  // a possible new maximum: make it exact
+        if (as <= FLT_MAX) gacc_add(g, cf, rf, s, as);
+        else grow_direct(d, i, fabs(__dsub_rn((double)cf, (double)rf)), gmax, glb);
       }
+    } else {
+      rmax = fmaxf(rmax, fin ? as : 0.f);
     }
-  }
-  if (!fx_pass<DT>(d, cb, rb)) {
+    const float ar = fabsf(rf);
+    bool pass = cf == rf || (fin && as <= __fmaf_rz(d.lo_r, ar, d.lo_a));
+    if (!pass && fin && !(as > __fmaf_ru(d.hi_r, ar, d.hi_a))) pass = pass64((double)cf, (double)rf, d.rtol, d.atol);
+    if (pass) return false;
     ++L.mism;
     if (!fin) {
       ++L.nonfin;
-    } else {
-      if (u > L.bu || (u == L.bu && i < L.bi)) {
-        L.bu = u;
-        L.bi = i;
-      }
-      const double r64 = to_f64<DT>(rb);
-      const double dv = fabs(__dsub_rn(to_f64<DT>(cb), r64));
-      L.within += dv <= f16_spacing(r64);
+      return true;
     }
-    // the mismatch's coordinate on every axis; the lanes here that share a
-    // bin add to it once (consecutive elements mostly share all but the
-    // last coordinate)
-    uint64_t rest = (uint64_t)i;
-    const unsigned act = __activemask();
-    const int lane = threadIdx.x & 31;
-    for (int a = d.rank - 1; a >= 0; --a) {
-      const uint64_t q = div_q(rest, d.sdiv[a].d, d.sdiv[a].m);
-      const long long bin = d.marg_off[a] + (long long)(rest - q * d.sdiv[a].d);
-      rest = q;
-      const unsigned peers = __match_any_sync(act, bin);
-      if (lane == __ffs(peers) - 1) {
-        if (d.marg_smem) atomicAdd(&smarg[bin], (unsigned)__popc(peers));
-        else gl_add(&gmarg[bin], (unsigned long long)__popc(peers));
-      }
+    if (u > L.bu || (u == L.bu && i < L.bi)) {
+      L.bu = u;
+      L.bi = i;
     }
+    // fl64(|c - r|) <= h, h = 2^(max(e, -14) - 10) with e the fp32 exponent
+    // of r (floor(log2 |r|) for normal r; fp32 subnormals and zero lie below
+    // 2^-14 and give 2^-24 alike).  |s| < h or |s| > h decides it (|s| and h
+    // are fp32 numbers, the remainder is below half an ulp of s); at |s| = h
+    // the exact value h + T rounds to h in fp64 iff T <= 2^-53 h.
+    const uint32_t E = (__float_as_uint(rf) >> 23) & 0xffu;
+    const float h = __uint_as_float((max(E, 113u) - 10u) << 23);
+    bool w = as < h;
+    if (as == h) {
+      const float t = twosum_err(cf, rf, s), tp = s > 0.f ? t : -t;
+      w = tp <= __fmul_rn(h, 0x1p-53f);
+    }
+    L.within += w ? 1u : 0u;
+    return true;
   }
 }
 
-template <int DT>
-__global__ void __launch_bounds__(kFxThreads) fx_kernel(const FxDesc *__restrict__ dp, FxAcc *acc, FxBest *blk,
+// The marginals of the leading axes (all but the last) for row rho of the
+// [R, L] view: its coordinates, each bin + n.
+__device__ __noinline__ void marg_rows(const FxDesc &d, int64_t rho, uint32_t n, uint32_t *smarg,
+                                       unsigned long long *gmarg) {
+  uint64_t rest = (uint64_t)rho;
+  for (int a = d.rank - 2; a >= 0; --a) {
+    const uint64_t q = div_q(rest, d.sdiv[a].d, d.sdiv[a].m);
+    const int64_t bin = d.marg_off[a] + (int64_t)(rest - q * d.sdiv[a].d);
+    rest = q;
+    if (d.marg_smem) atomicAdd(&smarg[bin], n);
+    else gl_add(&gmarg[bin], (unsigned long long)n);
+  }
+}
+
+// The growth index of row rho for an axis before the last: (rho / rs) % len.
+__device__ __forceinline__ int64_t row_gidx(const FxDesc &d, int64_t rho) {
+  if (d.j_is_row) return rho;
+  const uint64_t q = div_q((uint64_t)rho, d.drs.d, d.drs.m);
+  return (int64_t)(q - div_q(q, d.dlen.d, d.dlen.m) * d.dlen.d);
+}
+
+// Units: rb rows x g column windows of the [R, L] view; a window is 32
+// vectors wide, lane l owning columns c0 + l V .. c0 + l V + V - 1 in every
+// row, so the last axis' marginal (and, with AXL, the growth maxima of the
+// lane's columns) stay in registers until the window ends, and each row's
+// mismatch count adds up over the unit's windows in the warp's shared row
+// counters before it goes to the leading axes' marginals.  Four rows are
+// loaded at a time (eight 16-byte loads in flight per lane).
+template <int DT, bool AXL>
+__global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ FxDesc d, FxAcc *acc, FxBest *blk,
                                                        unsigned long long *g_growth, uint32_t *g_glb,
                                                        unsigned long long *g_marg) {
   constexpr int V = Tr<DT>::V;
   constexpr int EB = Tr<DT>::EB;
-  const FxDesc &d = *dp;
   extern __shared__ __align__(16) uint8_t fx_sm[];
+  // [warp][bin][lane] ulp histograms: a lane's bins sit in its own bank
   int32_t *hist = (int32_t *)fx_sm;
+  uint32_t *s_rows = (uint32_t *)(fx_sm + kFxHistBytes);  // [warp][kFxRowsMax] row mismatch counts
   const int64_t glen = d.grow_smem ? d.axis_len : 0;
   const int64_t mlen = d.marg_smem ? d.marg_off[d.rank] : 0;
-  unsigned long long *s_gmax = (unsigned long long *)(fx_sm + (size_t)kFxThreads * kFxHistStride * 4 + 16);
+  unsigned long long *s_gmax = (unsigned long long *)(fx_sm + kFxHistBytes + kFxRowBytes);
   uint32_t *s_glb = (uint32_t *)(s_gmax + glen);
   uint32_t *s_marg = s_glb + glen;
-  for (int t = threadIdx.x; t < kFxThreads * kFxHistStride; t += kFxThreads) hist[t] = 0;
+  for (int t = threadIdx.x; t < (kFxHistBytes + kFxRowBytes) / 4; t += kFxThreads) hist[t] = 0;
   for (int64_t t = threadIdx.x; t < glen; t += kFxThreads) {
     s_gmax[t] = 0ull;
     s_glb[t] = 0u;
@@ -204,54 +298,161 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const FxDesc *__restrict
   __syncthreads();
   unsigned long long *gmax = d.grow_smem ? s_gmax : g_growth;
   uint32_t *glb = d.grow_smem ? s_glb : g_glb;
-  int32_t *myhist = hist + threadIdx.x * kFxHistStride;
-  FxLane L = {0u, 0u, 0u, 0u, -1ll, -1ll};
-  const int64_t nvec = (d.numel + V - 1) / V;
-  const int64_t nth = (int64_t)gridDim.x * kFxThreads;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  int32_t *myhist = hist + warp * (NMV_ULP_BINS * 32) + lane;
+  uint32_t *myrows = s_rows + warp * kFxRowsMax;
+  FxLane L = {0u, 0u, 0u, 0u, 0u, INT64_MAX};
   const char *cb0 = (const char *)d.cand, *rb0 = (const char *)d.ref;
-  for (int64_t v0 = (int64_t)blockIdx.x * kFxThreads + threadIdx.x; v0 < nvec; v0 += 4 * nth) {
-    uint4 cv[4], rv[4];
-    int nn[4];
+  const int64_t Lw = d.L, R = d.R;
+  const int64_t col_bin0 = d.rank > 0 ? d.marg_off[d.rank - 1] : 0;
+  for (;;) {
+    unsigned long long u = 0;
+    if (lane == 0) u = atomicAdd(&acc->unit_ctr, 1ull);
+    u = __shfl_sync(0xffffffffu, u, 0);
+    if (u >= (unsigned long long)d.n_units) break;
+    const int64_t rbk = (int64_t)(u / (unsigned long long)d.WG), wg = (int64_t)u - rbk * d.WG;
+    const int64_t r0 = rbk * d.rb, r1 = min(R, r0 + d.rb);
+    const int64_t w0 = wg * d.g, w1 = min(d.CWn, w0 + d.g);
+    for (int64_t w = w0; w < w1; ++w) {
+      const int64_t mycol = w * (32 * V) + lane * V;
+      const int ncol = Lw - mycol >= V ? V : (Lw > mycol ? (int)(Lw - mycol) : 0);
+      uint32_t colm[V];
+      GAcc<DT> gc[AXL ? V : 1];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int64_t v = v0 + j * nth;
-      nn[j] = 0;
-      cv[j] = rv[j] = make_uint4(0, 0, 0, 0);
-      if (v < nvec) {
-        const int64_t e = v * V;
-        const int n = d.numel - e < V ? (int)(d.numel - e) : V;
-        nn[j] = n;
-        if (d.vec_ok && n == V) {
-          cv[j] = ld_v4(cb0 + e * EB);
-          rv[j] = ld_v4(rb0 + e * EB);
-        } else {
-          uint32_t cw[4] = {0, 0, 0, 0}, rw[4] = {0, 0, 0, 0};
-          for (int k = 0; k < n; ++k) {
-            const uint32_t c = ld_one<EB>(cb0, e + k), r = ld_one<EB>(rb0, e + k);
-            if constexpr (EB == 2) {
-              cw[k >> 1] |= c << (16 * (k & 1));
-              rw[k >> 1] |= r << (16 * (k & 1));
+      for (int k = 0; k < V; ++k) colm[k] = 0u;
+      for (int64_t r = r0; r < r1; r += 4) {
+        uint4 cv[4], rv[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          cv[j] = rv[j] = make_uint4(0, 0, 0, 0);
+          if (r + j < r1 && ncol > 0) {
+            const int64_t e = (r + j) * Lw + mycol;
+            if (d.vec_ok && ncol == V) {
+              cv[j] = ld_v4(cb0 + e * EB);
+              rv[j] = ld_v4(rb0 + e * EB);
             } else {
-              cw[k] = c;
-              rw[k] = r;
+              uint32_t cw[4] = {0, 0, 0, 0}, rw[4] = {0, 0, 0, 0};
+#pragma unroll
+              for (int k = 0; k < V; ++k) {
+                if (k < ncol) {
+                  const uint32_t c = ld_one<EB>(cb0, e + k), x = ld_one<EB>(rb0, e + k);
+                  if constexpr (EB == 2) {
+                    cw[k >> 1] |= c << (16 * (k & 1));
+                    rw[k >> 1] |= x << (16 * (k & 1));
+                  } else {
+                    cw[k] = c;
+                    rw[k] = x;
+                  }
+                }
+              }
+              cv[j] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
+              rv[j] = make_uint4(rw[0], rw[1], rw[2], rw[3]);
             }
           }
-          cv[j] = make_uint4(cw[0], cw[1], cw[2], cw[3]);
-          rv[j] = make_uint4(rw[0], rw[1], rw[2], rw[3]);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int64_t rho = r + j;
+          if (rho >= r1) break;  // warp-uniform
+          uint32_t m_row = 0u;
+          float rmax = 0.f;
+          GAcc<DT> gr;
+          const int64_t e = rho * Lw + mycol;
+#pragma unroll
+          for (int k = 0; k < V; ++k) {
+            if (k < ncol) {
+              const bool mm = fx_el<DT, AXL>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist,
+                                             AXL ? gc[AXL ? k : 0] : gr, rmax, gmax, glb);
+              colm[k] += mm ? 1u : 0u;
+              m_row += mm ? 1u : 0u;
+            }
+          }
+          if (d.rank >= 2) {
+            const uint32_t tot = __reduce_add_sync(0xffffffffu, m_row);
+            if (lane == 0 && tot) myrows[rho - r0] += tot;
+          }
+          if constexpr (!AXL) {
+            // the row's growth: the warp's largest |fl32(c - r)| screened
+            // against the bin's lower bound; past the screen, the exact
+            // maximum among the elements that reach it
+            if constexpr (Tr<DT>::kInt) {  // exact integer maxima
+              GAcc<DT> m;
+              m.U = __reduce_max_sync(0xffffffffu, gr.U);
+              if (m.U != 0u) {
+                const int64_t jg = row_gidx(d, rho);
+                if (lane == 0) grow_flush<DT>(m, jg, gmax, glb);
+              }
+            } else {
+            const uint32_t wm = __reduce_max_sync(0xffffffffu, __float_as_uint(rmax));
+            if (wm != 0u) {
+              const int64_t jg = row_gidx(d, rho);
+              const float lb = __uint_as_float(__shfl_sync(0xffffffffu, glb[jg], 0));
+              const float wmf = __uint_as_float(wm);
+              if (__fmul_rn(wmf, 1.0f + 0x1p-22f) >= lb) {
+                GAcc<DT> m;
+#pragma unroll
+                for (int k = 0; k < V; ++k) {
+                  if (k < ncol) {
+                    const float cf = to_f32<DT>(vbits<DT>(cv[j], k)), rf = to_f32<DT>(vbits<DT>(rv[j], k));
+                    const float s = __fsub_rn(cf, rf), as = fabsf(s);
+                    if (as == wmf && fabsf(cf) <= FLT_MAX && fabsf(rf) <= FLT_MAX) {
+                      if (as <= FLT_MAX) {
+                        const float t = twosum_err(cf, rf, s), tp = s > 0.f ? t : -t;
+                        if (m.S == 0.f || tp > m.T) {
+                          m.S = as;
+                          m.T = tp;
+                        }
+                      } else {
+                        grow_direct(d, e + k, fabs(__dsub_rn((double)cf, (double)rf)), gmax, glb);
+                      }
+                    }
+                  }
+                }
+                // (S, T) as a pair of order-preserving words, maximised word by word
+                const uint32_t hi = __float_as_uint(m.S), tb = __float_as_uint(m.T);
+                const uint32_t lo = (tb & 0x80000000u) ? ~tb : (tb | 0x80000000u);
+                const uint32_t mhi = __reduce_max_sync(0xffffffffu, hi);
+                const uint32_t mlo = __reduce_max_sync(0xffffffffu, hi == mhi ? lo : 0u);
+                m.S = __uint_as_float(mhi);
+                m.T = __uint_as_float((mlo & 0x80000000u) ? (mlo & 0x7fffffffu) : ~mlo);
+                if (lane == 0) grow_flush<DT>(m, jg, gmax, glb);
+              }
+            }
+            }
+          }
         }
       }
+      // the window's columns: the last axis' marginal and, with AXL, growth
+      if (d.rank > 0) {
+#pragma unroll
+        for (int k = 0; k < V; ++k) {
+          if (k < ncol && colm[k] != 0u) {
+            const int64_t bin = col_bin0 + mycol + k;
+            if (d.marg_smem) atomicAdd(&s_marg[bin], colm[k]);
+            else gl_add(&g_marg[bin], (unsigned long long)colm[k]);
+          }
+        }
+      }
+      if constexpr (AXL) {
+#pragma unroll
+        for (int k = 0; k < V; ++k)
+          if (k < ncol) grow_flush<DT>(gc[k], mycol + k, gmax, glb);
+      }
     }
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const int64_t e = (v0 + j * nth) * V;
-#pragma unroll
-      for (int k = 0; k < V; ++k)
-        if (k < nn[j])
-          fx_elem<DT>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist, gmax, glb, s_marg, g_marg);
+    // the unit's row counts -> the leading axes' marginals, in parallel
+    if (d.rank >= 2) {
+      __syncwarp();
+      for (int64_t t = lane; t < r1 - r0; t += 32) {
+        const uint32_t c = myrows[t];
+        if (c) {
+          marg_rows(d, r0 + t, c, s_marg, g_marg);
+          myrows[t] = 0u;
+        }
+      }
+      __syncwarp();
     }
   }
   // ---- the block's totals
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const unsigned long long m = warp_reduce((unsigned long long)L.mism, [](unsigned long long a, unsigned long long b) { return a + b; });
   const unsigned long long f = warp_reduce((unsigned long long)L.nfin, [](unsigned long long a, unsigned long long b) { return a + b; });
   const unsigned long long nf = warp_reduce((unsigned long long)L.nonfin, [](unsigned long long a, unsigned long long b) { return a + b; });
@@ -263,16 +464,17 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const FxDesc *__restrict
     if (w) atomicAdd(&acc->within, w);
   }
   // largest ulp distance, lowest index on ties
+  long long bu = L.bu ? (long long)L.bu : -1ll, bi = L.bu ? (long long)L.bi : -1ll;
 #pragma unroll
   for (int o = 16; o; o >>= 1) {
-    const long long u2 = __shfl_xor_sync(0xffffffffu, L.bu, o), i2 = __shfl_xor_sync(0xffffffffu, L.bi, o);
-    if (u2 > L.bu || (u2 == L.bu && u2 >= 0 && i2 < L.bi)) {
-      L.bu = u2;
-      L.bi = i2;
+    const long long u2 = __shfl_xor_sync(0xffffffffu, bu, o), i2 = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (u2 > bu || (u2 == bu && u2 >= 0 && i2 < bi)) {
+      bu = u2;
+      bi = i2;
     }
   }
   __shared__ FxBest wb[kFxThreads / 32];
-  if (lane == 0) wb[warp] = {L.bu, L.bi};
+  if (lane == 0) wb[warp] = {bu, bi};
   __syncthreads();
   if (threadIdx.x == 0) {
     FxBest b = wb[0];
@@ -281,9 +483,9 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const FxDesc *__restrict
     blk[blockIdx.x] = b;
   }
   if (threadIdx.x < NMV_ULP_BINS) {
-    unsigned long long s = 0;
-    for (int t = 0; t < kFxThreads; ++t) s += (unsigned)hist[t * kFxHistStride + threadIdx.x];
-    if (s) atomicAdd(&acc->hist[threadIdx.x], s);
+    unsigned long long sum = 0;
+    for (int t = 0; t < kFxThreads; ++t) sum += (unsigned)hist[(t >> 5) * (NMV_ULP_BINS * 32) + threadIdx.x * 32 + (t & 31)];
+    if (sum) atomicAdd(&acc->hist[threadIdx.x], sum);
   }
   for (int64_t t = threadIdx.x; t < glen; t += kFxThreads)
     if (s_gmax[t]) atomicMax(&g_growth[t], s_gmax[t]);
@@ -359,36 +561,43 @@ float f32_up(double x) {
 }
 
 size_t fx_smem(const FxDesc &d) {
-  size_t b = (size_t)kFxThreads * kFxHistStride * 4 + 16;
+  size_t b = (size_t)kFxHistBytes + kFxRowBytes;
   if (d.grow_smem) b += (size_t)d.axis_len * 12;
   if (d.marg_smem) b += (size_t)d.marg_off[d.rank] * 4;
   return b;
 }
 
-template <int DT>
+template <int DT, bool AXL>
 cudaError_t launch_fx_dt(int sms, const FxDesc &h, const FxDesc *dd, FxAcc *acc, FxBest *blk, int *n_blk,
                          unsigned long long *gg, uint32_t *glb, unsigned long long *gm, cudaStream_t st) {
   const size_t smem = fx_smem(h);
-  cudaError_t e = cudaFuncSetAttribute(fx_kernel<DT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(fx_kernel<DT, AXL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   int occ = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fx_kernel<DT>, kFxThreads, smem);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, fx_kernel<DT, AXL>, kFxThreads, smem);
   if (e != cudaSuccess) return e;
-  const int64_t V = vec_elems(h.dtype);
   int64_t grid = (int64_t)sms * std::max(occ, 1);
-  grid = std::max<int64_t>(1, std::min<int64_t>(grid, (h.numel / V + 4 * kFxThreads - 1) / (4 * kFxThreads)));
+  grid = std::max<int64_t>(1, std::min<int64_t>(grid, (h.n_units + kFxThreads / 32 - 1) / (kFxThreads / 32)));
   *n_blk = (int)grid;
-  fx_kernel<DT><<<(int)grid, kFxThreads, smem, st>>>(dd, acc, blk, gg, glb, gm);
+  fx_kernel<DT, AXL><<<(int)grid, kFxThreads, smem, st>>>(h, acc, blk, gg, glb, gm);
   return cudaGetLastError();
+}
+
+template <int DT>
+cudaError_t launch_fx_ax(int sms, const FxDesc &h, const FxDesc *dd, FxAcc *acc, FxBest *blk, int *n_blk,
+                         unsigned long long *gg, uint32_t *glb, unsigned long long *gm, cudaStream_t st) {
+  // the growth axis is the last one (or the tensor has rank 0 or 1)
+  if (h.rank <= 1 || h.axis == h.rank - 1) return launch_fx_dt<DT, true>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
+  return launch_fx_dt<DT, false>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
 }
 
 cudaError_t launch_fx(int sms, const FxDesc &h, const FxDesc *dd, FxAcc *acc, FxBest *blk, int *n_blk,
                       unsigned long long *gg, uint32_t *glb, unsigned long long *gm, cudaStream_t st) {
   switch (h.dtype) {
-    case NMV_F32: return launch_fx_dt<NMV_F32>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
-    case NMV_F16: return launch_fx_dt<NMV_F16>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
-    case NMV_BF16: return launch_fx_dt<NMV_BF16>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
-    default: return launch_fx_dt<NMV_I32>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
+    case NMV_F32: return launch_fx_ax<NMV_F32>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
+    case NMV_F16: return launch_fx_ax<NMV_F16>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
+    case NMV_BF16: return launch_fx_ax<NMV_BF16>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
+    default: return launch_fx_ax<NMV_I32>(sms, h, dd, acc, blk, n_blk, gg, glb, gm, st);
   }
 }
 
@@ -431,10 +640,20 @@ int check_fx_case(const nmv_forensics_case &c, FxDesc &d, int64_t i) {
   d.axis_len = a.rank > 0 ? a.shape[d.axis] : 1;
   d.dstride = make_div((uint64_t)std::max<int64_t>(stride, 1));
   d.dlen = make_div((uint64_t)std::max<int64_t>(d.axis_len, 1));
-  d.idx32 = n <= (int64_t)0xffffffffll ? 1 : 0;
-  d.m32stride = d.idx32 ? 0xffffffffu / (uint32_t)std::max<int64_t>(stride, 1) : 0u;
-  d.m32len = d.idx32 ? 0xffffffffu / (uint32_t)std::max<int64_t>(d.axis_len, 1) : 0u;
-  d.vec_ok = ((uintptr_t)a.data % 16 == 0) && ((uintptr_t)b.data % 16 == 0);
+  // the [R, L] view and its units
+  const int64_t V = vec_elems(a.dtype), EB = elem_bytes(a.dtype);
+  d.L = a.rank > 0 ? a.shape[a.rank - 1] : 1;
+  d.R = d.L > 0 ? n / d.L : 0;
+  d.CWn = (d.L + 32 * V - 1) / (32 * V);
+  d.rb = std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(d.R, kFxRowsMax), kFxUnitElems / (32 * V)));
+  d.g = std::max<int64_t>(1, std::min<int64_t>(d.CWn, kFxUnitElems / (d.rb * 32 * V)));
+  d.WG = (d.CWn + d.g - 1) / d.g;
+  d.n_units = n > 0 ? (d.R + d.rb - 1) / d.rb * d.WG : 0;
+  // growth on an axis before the last: rows per index of the axis
+  const int64_t rs = d.L > 0 ? std::max<int64_t>(stride, 1) / std::max<int64_t>(d.L, 1) : 1;
+  d.drs = make_div((uint64_t)std::max<int64_t>(rs, 1));
+  d.j_is_row = (rs == 1 && d.axis_len == d.R) ? 1 : 0;
+  d.vec_ok = ((uintptr_t)a.data % 16 == 0) && ((uintptr_t)b.data % 16 == 0) && (d.L * EB) % 16 == 0;
   d.rtol = c.rtol;
   d.atol = c.atol;
   const bool filter = c.rtol <= 0.5 && c.atol <= 0x1p100;

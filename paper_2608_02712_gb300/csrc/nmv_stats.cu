@@ -4,23 +4,27 @@
 //
 // Levels: the whole tensor and every tile of the [M, N] view (the tile grid
 // of the localisation maps).  Work is cut into units: a unit is a block of
-// at most kUnitRows x kUnitCols elements of one tile (a tile is split into
-// row and column chunks, a small tile is one unit).  stats_kernel hands the
-// units to warps from a counter; a warp reads its unit with 16-byte loads
-// where the rows allow (scalar loads otherwise), each lane accumulating
-// class counts, min/max and the sums, then reduces the lanes in a fixed
-// butterfly and stores the unit's partial.  stats_fin_kernel merges each
-// tile's units in unit order into the tile's statistics (written straight
-// into the mapped host result), and the tiles of each case in a fixed
-// tree into the whole-tensor statistics: nothing depends on which warp took
-// which unit, so the results are bit-identical from run to run.
+// at most kUnitElems elements of one tile, at most kUnitCols columns wide
+// (a tile is split into row and column chunks, a small tile is one unit).
+// stats_kernel hands the units to warps from a counter; a warp reads its
+// unit with 16-byte loads where the rows allow (scalar loads otherwise),
+// each lane walking its rows with a fixed stride and accumulating class
+// counts, min/max and the sums, then reduces the lanes in a fixed butterfly
+// and stores the unit's partial.  stats_fin_kernel merges each tile's units
+// in unit order into the tile's statistics (written straight into the
+// mapped host result), and the tiles of each case in a fixed tree into the
+// whole-tensor statistics: nothing depends on which warp took which unit,
+// so the results are bit-identical from run to run.
 //
-// Sums.  float elements: the lane sums sum(x) and sum(x^2) as float-float
-// pairs (Knuth's TwoSum; x^2 split exactly as p + pe with an fma), folded
-// into fp64 every kFlush vectors; elements outside [2^-60, 2^56] in
-// magnitude (whose fp32 squares could underflow or whose sums could
-// overflow) are added in fp64 directly.  int32 elements: exact 128-bit
-// integer sums, rounded once to fp64 at the end.
+// Sums.  float elements: the lanes first take every whole vector on a fast
+// path without class tests, sum(x) and sum(x^2) as float-float pairs
+// (Knuth's TwoSum; x^2 split exactly as p + pe with an fma) folded into
+// fp64 every kFlush vectors.  The result stands when the unit met no NaN
+// or infinity and its largest magnitude lies in [2^-44, 2^57) (the pairs
+// cannot overflow and the squares' remainders are exact, or round by a
+// negligible amount); otherwise the unit is taken again element by
+// element, classes tested and finite values added in fp64.  int32
+// elements: exact 128-bit integer sums, rounded once to fp64 at the end.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -174,8 +178,10 @@ __device__ __forceinline__ void part_out(const StatPart &p, int dt, nmv_stat *o)
 }
 
 // ------------------------------------------------------------ lane sums
+// Every field is a scalar (no field is indexed at run time), so a lane's
+// sums stay in registers.
 struct LaneStat {
-  int64_t cnt[4];
+  int32_t n_nan, n_pinf, n_ninf, n_zero;  // a unit has at most kUnitElems elements
   int64_t first_nan, first_inf;
   float mn, mx;          // float types
   int32_t imn, imx;      // int32
@@ -186,7 +192,7 @@ struct LaneStat {
 };
 
 __device__ __forceinline__ void lane_init(LaneStat &L) {
-  for (int k = 0; k < 4; ++k) L.cnt[k] = 0;
+  L.n_nan = L.n_pinf = L.n_ninf = L.n_zero = 0;
   L.first_nan = L.first_inf = INT64_MAX;
   L.mn = INFINITY;
   L.mx = -INFINITY;
@@ -225,16 +231,17 @@ template <int DT>
 __device__ __forceinline__ void lane_slow(LaneStat &L, uint32_t b, int64_t idx) {
   const float x = to_f32<DT>(b);
   if (isnan(x)) {
-    ++L.cnt[0];
+    ++L.n_nan;
     L.first_nan = min(L.first_nan, idx);
     return;
   }
   if (isinf(x)) {
-    ++L.cnt[x > 0.f ? 1 : 2];
+    if (x > 0.f) ++L.n_pinf;
+    else ++L.n_ninf;
     L.first_inf = min(L.first_inf, idx);
     return;
   }
-  if (x == 0.f) ++L.cnt[3];
+  if (x == 0.f) ++L.n_zero;
   L.mn = fminf(L.mn, x);
   L.mx = fmaxf(L.mx, x);
   const double d = (double)x;
@@ -242,56 +249,153 @@ __device__ __forceinline__ void lane_slow(LaneStat &L, uint32_t b, int64_t idx) 
   L.q64 = __dadd_rn(L.q64, __dmul_rn(d, d));
 }
 
-// fp32 bits whose magnitude lies in [2^-50, 2^57) (or zero): finite, x^2
-// splits exactly into fl(x^2) + fma error (exponent sum >= -103, so the
-// error does not underflow), and 64 such squares or values sum without
-// overflow.
-__device__ __forceinline__ bool fast_mag(uint32_t f32bits) {
-  const uint32_t m = f32bits & 0x7fffffffu;
-  return m == 0u || (m - 0x26800000u) < (0x5c000000u - 0x26800000u);
+// -1 if x is a zero of either sign, else 0.
+__device__ __forceinline__ int32_t zero_m1(float x) {
+  int32_t r;
+  asm("set.eq.s32.f32 %0, %1, 0f00000000;" : "=r"(r) : "f"(x));
+  return r;
 }
 
-// V elements of one lane: bits in v (vector layout), n of them valid, the
-// first at linear index idx.
+// int32 elements (exact): V elements in v, n of them valid.
 template <int DT>
-__device__ __forceinline__ void lane_vec(LaneStat &L, const uint4 &v, int n, int64_t idx) {
+__device__ __forceinline__ void lane_int(LaneStat &L, const uint4 &v, int n) {
   constexpr int V = Tr<DT>::V;
-  if constexpr (Tr<DT>::kInt) {
 #pragma unroll
-    for (int k = 0; k < V; ++k) {
-      if (k >= n) break;
+  for (int k = 0; k < V; ++k) {
+    if (k < n) {
       const int32_t x = (int32_t)vbits<DT>(v, k);
-      L.cnt[3] += x == 0;
+      L.n_zero += x == 0;
       L.imn = min(L.imn, x);
       L.imx = max(L.imx, x);
       const int64_t x64 = x;
       add128(L.is_lo, L.is_hi, (uint64_t)x64, x64 < 0 ? ~0ull : 0ull);
       add128(L.iq_lo, L.iq_hi, (uint64_t)(x64 * x64), 0ull);
     }
-  } else {
-    float x[V];
-    bool ok = n == V;
+  }
+}
+
+// Float elements, the fast path: V valid elements of any value, no class
+// test.  Zeros are counted, min/max taken, and sum(x), sum(x^2) added as
+// float-float pairs (TwoSum; x^2 split exactly into fl(x^2) and an fma
+// remainder).  The pairs are exact while every |x| lies below 2^57 and the
+// remainders are exact for |x| >= 2^-51; a NaN or an infinity leaves a
+// non-finite sum.  The unit's end test (lane_fast_ok) decides whether the
+// unit's result stands.
+template <int DT>
+__device__ __forceinline__ void lane_fast(LaneStat &L, const uint4 &v) {
+  constexpr int V = Tr<DT>::V;
+  float x[V];
 #pragma unroll
-    for (int k = 0; k < V; ++k) {
-      x[k] = vdec<DT>(v, k);
-      ok = ok && fast_mag(__float_as_uint(x[k]));
-    }
-    if (ok) {
+  for (int k = 0; k < V; ++k) x[k] = vdec<DT>(v, k);
+  int32_t z = 0;
+  float mn = x[0], mx = x[0];
 #pragma unroll
-      for (int k = 0; k < V; k += 2) {
-        const float2 p = make_float2(x[k], x[k + 1]);
-        L.cnt[3] += (x[k] == 0.f) + (x[k + 1] == 0.f);
-        L.mn = fminf(L.mn, fminf(x[k], x[k + 1]));
-        L.mx = fmaxf(L.mx, fmaxf(x[k], x[k + 1]));
-        ff_add2(L.sh, L.sl, p);
-        const float2 sq = __fmul2_rn(p, p);
-        const float2 pe = __ffma2_rn(p, p, __fmul2_rn(sq, make_float2(-1.f, -1.f)));
-        ff_add2(L.qh, L.ql, sq);
-        L.ql = __fadd2_rn(L.ql, pe);
+  for (int k = 0; k < V; ++k) z += zero_m1(x[k]);
+#pragma unroll
+  for (int k = 1; k < V; ++k) {
+    mn = fminf(mn, x[k]);
+    mx = fmaxf(mx, x[k]);
+  }
+  L.n_zero -= z;
+  L.mn = fminf(L.mn, mn);
+  L.mx = fmaxf(L.mx, mx);
+#pragma unroll
+  for (int k = 0; k < V; k += 2) {
+    const float2 p = make_float2(x[k], x[k + 1]);
+    ff_add2(L.sh, L.sl, p);
+    const float2 sq = __fmul2_rn(p, p);
+    const float2 pe = __ffma2_rn(p, p, __fmul2_rn(sq, make_float2(-1.f, -1.f)));
+    ff_add2(L.qh, L.ql, sq);
+    L.ql = __fadd2_rn(L.ql, pe);
+  }
+  if (++L.pending == kFlush) lane_fold(L);
+}
+
+// After the final fold: the fast path's result stands when the sums are
+// finite (no NaN or infinity met) and the largest magnitude a lies in
+// [2^-44, 2^57) (or every element is zero).  Below 2^-51 a square's
+// remainder may round, by at most 2^-150 per element; a unit has at most
+// 2^14 elements and sum(x^2) >= a^2 >= 2^-88, so the relative error stays
+// below 2^-48.
+__device__ __forceinline__ bool lane_fast_ok(const LaneStat &L) {
+  const float a = fmaxf(-L.mn, L.mx);  // -inf for a lane without elements
+  return isfinite(L.s64) && isfinite(L.q64) && a < 0x1p57f && !(a > 0.f && a < 0x1p-44f);
+}
+
+// One unit's elements into a lane's sums.  The unit is rows [r0, r1) x
+// columns [c0, c0 + cols) of the [M, N] view, cols * EB bytes at most
+// kUnitCols elements; a row holds vpr vectors.  When vpr >= 32 a row is
+// swept in windows of 32 vectors, lane l taking vector l of each window in
+// every row; narrower rows are stacked, S = 32 / vpr rows per step.  Each
+// lane walks its rows with a fixed byte stride and four loads in flight.
+// MODE 0: int32 (exact); 1: float fast path (whole vectors; partial
+// vectors element by element); 2: float, every element on the exact path.
+template <int DT, int MODE>
+__device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool vec_ok, int64_t N, int64_t r0,
+                                           int64_t r1, int64_t c0, int64_t cols, int lane) {
+  constexpr int V = Tr<DT>::V;
+  constexpr int EB = Tr<DT>::EB;
+  const int32_t vpr = (int32_t)((cols + V - 1) / V);
+  const int32_t VW = vpr < 32 ? vpr : 32;  // lanes per row
+  const int32_t S = 32 / VW;               // rows per step
+  const int32_t rsub = lane / VW, vl = lane - rsub * VW;
+  if (rsub >= S) return;
+  const int32_t nw = (vpr + 31) / 32;
+  const int64_t nr = (r1 - r0 - rsub + S - 1) / S;  // this lane's rows
+  const int64_t stride = (int64_t)S * N;            // elements between them
+  for (int32_t w = 0; w < nw; ++w) {
+    const int32_t vi = w * 32 + vl;
+    if (vi >= vpr) break;
+    const int64_t left = cols - (int64_t)vi * V;
+    const int n = left < V ? (int)left : V;
+    int64_t e = (r0 + rsub) * N + c0 + (int64_t)vi * V;  // the lane's first element in this window
+    if (MODE != 2 && vec_ok && n == V) {
+      const char *p = base + e * EB;
+      const int64_t sb = stride * EB;
+      int64_t k = 0;
+      for (; k + 4 <= nr; k += 4) {
+        const uint4 v0 = ld_v4(p), v1 = ld_v4(p + sb), v2 = ld_v4(p + 2 * sb), v3 = ld_v4(p + 3 * sb);
+        p += 4 * sb;
+        if constexpr (MODE == 0) {
+          lane_int<DT>(L, v0, V);
+          lane_int<DT>(L, v1, V);
+          lane_int<DT>(L, v2, V);
+          lane_int<DT>(L, v3, V);
+        } else {
+          lane_fast<DT>(L, v0);
+          lane_fast<DT>(L, v1);
+          lane_fast<DT>(L, v2);
+          lane_fast<DT>(L, v3);
+        }
       }
-      if (++L.pending == kFlush) lane_fold(L);
+      for (; k < nr; ++k) {
+        const uint4 v0 = ld_v4(p);
+        p += sb;
+        if constexpr (MODE == 0) lane_int<DT>(L, v0, V);
+        else lane_fast<DT>(L, v0);
+      }
     } else {
-      for (int k = 0; k < n; ++k) lane_slow<DT>(L, vbits<DT>(v, k), idx + k);
+      for (int64_t k = 0; k < nr; ++k, e += stride) {
+        uint32_t wd[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int q = 0; q < V; ++q) {
+          if (q < n) {
+            const uint32_t b = ld_one<EB>(base, e + q);
+            if constexpr (EB == 2) wd[q >> 1] |= b << (16 * (q & 1));
+            else wd[q] = b;
+          }
+        }
+        const uint4 v = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        if constexpr (MODE == 0) {
+          lane_int<DT>(L, v, n);
+        } else if (MODE == 1 && n == V) {
+          lane_fast<DT>(L, v);
+        } else {
+#pragma unroll
+          for (int q = 0; q < V; ++q)
+            if (q < n) lane_slow<DT>(L, vbits<DT>(v, q), e + q);
+        }
+      }
     }
   }
 }
@@ -303,8 +407,6 @@ template <int DT>
 __global__ void __launch_bounds__(kStatThreads) stats_kernel(const StatsDesc *__restrict__ cases, int n_cases,
                                                             int64_t unit_base, int64_t n_units,
                                                             unsigned long long *unit_ctr, StatPart *parts) {
-  constexpr int V = Tr<DT>::V;
-  constexpr int EB = Tr<DT>::EB;
   const int lane = threadIdx.x & 31;
   for (;;) {
     int64_t u = 0;
@@ -331,59 +433,31 @@ __global__ void __launch_bounds__(kStatThreads) stats_kernel(const StatsDesc *__
     const int64_t c0 = tc0 + kc * d.cw;
     const int64_t c1 = min(min(c0 + d.cw, tc0 + d.tw), d.N);
     const int64_t rows = r1 > r0 ? r1 - r0 : 0, cols = c1 > c0 ? c1 - c0 : 0;
+    const char *base = (const char *)d.x;
     LaneStat L;
     lane_init(L);
     if (rows > 0 && cols > 0) {
-      // The unit's (row, vector) pairs in row-major order are the lanes'
-      // tasks: lane l takes tasks l, l + 32, ...; consecutive lanes read
-      // consecutive vectors of a row, and each lane keeps four loads in
-      // flight.  A unit has at most kUnitElems elements, so task numbers
-      // and vector counts fit in 32 bits.
-      const uint32_t vpr = (uint32_t)((cols + V - 1) / V);
-      const uint32_t ntask = (uint32_t)rows * vpr;
-      const uint32_t mv = 0xffffffffu / vpr;
-      const char *base = (const char *)d.x;
-      for (uint32_t t0 = lane; t0 < ntask; t0 += 4 * 32) {
-        uint4 v[4];
-        int nn[4];
-        int64_t ee[4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const uint32_t task = t0 + 32 * j;
-          nn[j] = 0;
-          ee[j] = 0;
-          v[j] = make_uint4(0, 0, 0, 0);
-          if (task < ntask) {
-            const uint32_t rr = div_q32(task, vpr, mv), vi = task - rr * vpr;
-            const int64_t e = (r0 + rr) * d.N + c0 + (int64_t)vi * V;
-            const int64_t left = cols - (int64_t)vi * V;
-            const int n = left < V ? (int)left : V;
-            nn[j] = n;
-            ee[j] = e;
-            if (d.vec_ok && n == V) {
-              v[j] = ld_v4(base + e * EB);
-            } else {
-              uint32_t w[4] = {0, 0, 0, 0};
-              for (int k = 0; k < n; ++k) {
-                const uint32_t b = ld_one<EB>(base, e + k);
-                if constexpr (EB == 2) w[k >> 1] |= b << (16 * (k & 1));
-                else w[k] = b;
-              }
-              v[j] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
-          }
+      const bool vec_ok = d.vec_ok != 0;
+      const int64_t N = d.N;
+      if constexpr (Tr<DT>::kInt) {
+        unit_sweep<DT, 0>(L, base, vec_ok, N, r0, r1, c0, cols, lane);
+      } else {
+        unit_sweep<DT, 1>(L, base, vec_ok, N, r0, r1, c0, cols, lane);
+        lane_fold(L);
+        if (__any_sync(0xffffffffu, !lane_fast_ok(L))) {  // the unit again, element by element
+          lane_init(L);
+          unit_sweep<DT, 2>(L, base, vec_ok, N, r0, r1, c0, cols, lane);
         }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (nn[j] > 0) lane_vec<DT>(L, v[j], nn[j], ee[j]);
       }
-      if constexpr (!Tr<DT>::kInt) lane_fold(L);
     }
     // lanes -> the unit's partial (fixed butterfly; every lane ends with it)
     StatPart p;
     part_init(p);
     p.n = lane == 0 ? rows * cols : 0;
-    for (int k = 0; k < 4; ++k) p.cnt[k] = L.cnt[k];
+    p.cnt[0] = L.n_nan;
+    p.cnt[1] = L.n_pinf;
+    p.cnt[2] = L.n_ninf;
+    p.cnt[3] = L.n_zero;
     p.first_nan = L.first_nan;
     p.first_inf = L.first_inf;
     if constexpr (Tr<DT>::kInt) {

@@ -384,7 +384,7 @@ def stats_result_to_dict(r: StatsResult) -> dict:
     tiles = {}
     if n:
         raw = np.ctypeslib.as_array(ctypes.cast(r.tiles, ctypes.POINTER(ctypes.c_uint8)),
-                                    shape=(n * ctypes.sizeof(Stat),)).copy()
+                                    shape=(n * ctypes.sizeof(Stat),))  # fields are copied out below
         rec = raw.view(np.dtype([(k, np.int64) for k in STAT_COUNTS] +
                                 [(k, np.float64) for k in STAT_VALUES]))
         tiles = {k: rec[k].reshape(gr, gc).copy() for k in STAT_COUNTS + STAT_VALUES}

@@ -118,3 +118,24 @@ def test_stats_full_size_c5_candidate():
     xh = x.cpu()
     del x
     check(got, oracle.stats(xh, tile=(128, 128)), xh)
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16, torch.float16], ids=["f32", "bf16", "f16"])
+def test_stats_magnitude_bands(dt):
+    """Tiles whose largest magnitude lies below 2^-44 or at 2^57 and above
+    (taken again element by element), tiles mixing tiny and ordinary values
+    (the fast path's remainders round), subnormals, and tiles holding a NaN
+    or an infinity next to tiles that hold none."""
+    g = torch.Generator().manual_seed(41)
+    rows, cols = 256, 384
+    x = torch.randn(rows, cols, generator=g)
+    scales = torch.tensor([2.0 ** -130, 2.0 ** -60, 2.0 ** -45, 2.0 ** -43, 1.0, 2.0 ** 56, 2.0 ** 58, 2.0 ** 100])
+    band = scales[torch.arange(rows) // 32 % len(scales)]
+    x = x * band[:, None]
+    x[40, 7] = 2.0 ** -140        # one tiny value among ordinary ones
+    x[130, 200] = float("nan")
+    x[131, 5] = float("inf")
+    x[200:203, :] = 0.0
+    x = x.to(dt)
+    for tile in ((32, 128), (16, 384), (5, 7), (256, 384)):
+        check(stats(x.cuda(), tile=tile), oracle.stats(x, tile=tile), x)
