@@ -51,7 +51,7 @@ struct FxDesc {
   int64_t numel;
   int64_t L, R;             // the pair as R rows of L elements (L the last axis; 1 x 1 for rank 0)
   int64_t CWn, rb, g, WG;   // column windows of 32 vectors; a unit is rb rows x g windows
-  int64_t n_units;
+  int64_t RBn, n_units;     // row blocks; units (row block fastest)
   int64_t shape[NMV_MAX_RANK];
   Div64 sdiv[NMV_MAX_RANK];
   int64_t marg_off[NMV_MAX_RANK + 1];
@@ -182,7 +182,7 @@ __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, u
     const int32_t c = (int32_t)cb, r = (int32_t)rb;
     const uint32_t u = ulp_dist<DT>(cb, rb);  // = |c - r|
     ++L.nfin;
-    hist[32 * (u ? 32 - __clz(u) : 0)] += 1;
+    sh_add(&hist[32 * (u ? 32 - __clz(u) : 0)], 1);
     g.U = max(g.U, u);
     if (u == 0u) return false;
     const float as = __uint2float_rn(u), ar = fabsf(__int2float_rn(r));
@@ -192,7 +192,7 @@ __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, u
     else pass = pass64((double)c, (double)r, d.rtol, d.atol);
     if (pass) return false;
     ++L.mism;
-    if (u > L.bu || (u == L.bu && i < L.bi)) {
+    if (u >= L.bu && (u > L.bu || i < L.bi)) {
       L.bu = u;
       L.bi = i;
     }
@@ -207,7 +207,7 @@ __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, u
     const bool fin = fabsf(cf) <= FLT_MAX && fabsf(rf) <= FLT_MAX;
     const uint32_t u = ulp_dist<DT>(cb, rb);  // meaningful for finite pairs
     L.nfin += fin ? 1u : 0u;
-    hist[32 * (u ? 32 - __clz(u) : 0)] += fin ? 1 : 0;
+    sh_add(&hist[32 * (u ? 32 - __clz(u) : 0)], fin ? 1 : 0);
     if constexpr (AXL) {
       if (fin && as >= g.S) {  // a possible new maximum: make it exact
         if (as <= FLT_MAX) gacc_add(g, cf, rf, s, as);
@@ -225,7 +225,7 @@ __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, u
       ++L.nonfin;
       return true;
     }
-    if (u > L.bu || (u == L.bu && i < L.bi)) {
+    if (u >= L.bu && (u > L.bu || i < L.bi)) {
       L.bu = u;
       L.bi = i;
     }
@@ -310,7 +310,9 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ 
     if (lane == 0) u = atomicAdd(&acc->unit_ctr, 1ull);
     u = __shfl_sync(0xffffffffu, u, 0);
     if (u >= (unsigned long long)d.n_units) break;
-    const int64_t rbk = (int64_t)(u / (unsigned long long)d.WG), wg = (int64_t)u - rbk * d.WG;
+    // consecutive units lie in different row blocks, so the units that run
+    // at once share few rows and the growth screen sees earlier maxima
+    const int64_t wg = (int64_t)(u / (unsigned long long)d.RBn), rbk = (int64_t)u - wg * d.RBn;
     const int64_t r0 = rbk * d.rb, r1 = min(R, r0 + d.rb);
     const int64_t w0 = wg * d.g, w1 = min(d.CWn, w0 + d.g);
     for (int64_t w = w0; w < w1; ++w) {
@@ -648,7 +650,8 @@ int check_fx_case(const nmv_forensics_case &c, FxDesc &d, int64_t i) {
   d.rb = std::max<int64_t>(1, std::min<int64_t>(std::min<int64_t>(d.R, kFxRowsMax), kFxUnitElems / (32 * V)));
   d.g = std::max<int64_t>(1, std::min<int64_t>(d.CWn, kFxUnitElems / (d.rb * 32 * V)));
   d.WG = (d.CWn + d.g - 1) / d.g;
-  d.n_units = n > 0 ? (d.R + d.rb - 1) / d.rb * d.WG : 0;
+  d.RBn = (d.R + d.rb - 1) / d.rb;
+  d.n_units = n > 0 ? d.RBn * d.WG : 0;
   // growth on an axis before the last: rows per index of the axis
   const int64_t rs = d.L > 0 ? std::max<int64_t>(stride, 1) / std::max<int64_t>(d.L, 1) : 1;
   d.drs = make_div((uint64_t)std::max<int64_t>(rs, 1));

@@ -41,6 +41,7 @@ constexpr int kStatThreads = 256;
 constexpr int64_t kUnitCols = 8192;    // elements of a unit's row segment at most
 constexpr int64_t kUnitElems = 16384;  // elements of a unit at most (rows x cols), unless one row is longer
 constexpr int kFinBlocks = 256;        // finalize blocks per case at most
+constexpr int64_t kCoopUnits = 32;     // tiles of this many units or more are merged by a whole block
 constexpr int kFlush = 32;             // float-float pairs folded into fp64 every kFlush vectors
 
 // One buffer as the kernels see it.
@@ -311,6 +312,33 @@ __device__ __forceinline__ void lane_fast(LaneStat &L, const uint4 &v) {
   if (++L.pending == kFlush) lane_fold(L);
 }
 
+// Every element of a whole vector zero or of magnitude in [2^-50, 2^57):
+// the fast path adds such vectors exactly (the unit's second pass takes the
+// others element by element).
+template <int DT>
+__device__ __forceinline__ bool vec_in_range(const uint4 &v) {
+  constexpr int V = Tr<DT>::V;
+  bool ok = true;
+#pragma unroll
+  for (int k = 0; k < V; ++k) {
+    const uint32_t m = __float_as_uint(vdec<DT>(v, k)) & 0x7fffffffu;
+    ok = ok && (m == 0u || m - 0x26800000u < 0x5c000000u - 0x26800000u);
+  }
+  return ok;
+}
+
+// A whole vector on the unit's second pass; its first element at index e.
+template <int DT>
+__device__ __forceinline__ void lane_checked(LaneStat &L, const uint4 &v, int64_t e) {
+  constexpr int V = Tr<DT>::V;
+  if (vec_in_range<DT>(v)) {
+    lane_fast<DT>(L, v);
+  } else {
+#pragma unroll
+    for (int q = 0; q < V; ++q) lane_slow<DT>(L, vbits<DT>(v, q), e + q);
+  }
+}
+
 // After the final fold: the fast path's result stands when the sums are
 // finite (no NaN or infinity met) and the largest magnitude a lies in
 // [2^-44, 2^57) (or every element is zero).  Below 2^-51 a square's
@@ -329,7 +357,8 @@ __device__ __forceinline__ bool lane_fast_ok(const LaneStat &L) {
 // every row; narrower rows are stacked, S = 32 / vpr rows per step.  Each
 // lane walks its rows with a fixed byte stride and four loads in flight.
 // MODE 0: int32 (exact); 1: float fast path (whole vectors; partial
-// vectors element by element); 2: float, every element on the exact path.
+// vectors element by element); 2: float, the unit's second pass: whole
+// vectors in range on the fast path, the rest element by element.
 template <int DT, int MODE>
 __device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool vec_ok, int64_t N, int64_t r0,
                                            int64_t r1, int64_t c0, int64_t cols, int lane) {
@@ -349,7 +378,7 @@ __device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool v
     const int64_t left = cols - (int64_t)vi * V;
     const int n = left < V ? (int)left : V;
     int64_t e = (r0 + rsub) * N + c0 + (int64_t)vi * V;  // the lane's first element in this window
-    if (MODE != 2 && vec_ok && n == V) {
+    if (vec_ok && n == V) {
       const char *p = base + e * EB;
       const int64_t sb = stride * EB;
       int64_t k = 0;
@@ -361,18 +390,30 @@ __device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool v
           lane_int<DT>(L, v1, V);
           lane_int<DT>(L, v2, V);
           lane_int<DT>(L, v3, V);
-        } else {
+        } else if constexpr (MODE == 1) {
           lane_fast<DT>(L, v0);
           lane_fast<DT>(L, v1);
           lane_fast<DT>(L, v2);
           lane_fast<DT>(L, v3);
+        } else {
+          lane_checked<DT>(L, v0, e);
+          lane_checked<DT>(L, v1, e + stride);
+          lane_checked<DT>(L, v2, e + 2 * stride);
+          lane_checked<DT>(L, v3, e + 3 * stride);
+          e += 4 * stride;
         }
       }
       for (; k < nr; ++k) {
         const uint4 v0 = ld_v4(p);
         p += sb;
-        if constexpr (MODE == 0) lane_int<DT>(L, v0, V);
-        else lane_fast<DT>(L, v0);
+        if constexpr (MODE == 0) {
+          lane_int<DT>(L, v0, V);
+        } else if constexpr (MODE == 1) {
+          lane_fast<DT>(L, v0);
+        } else {
+          lane_checked<DT>(L, v0, e);
+          e += stride;
+        }
       }
     } else {
       for (int64_t k = 0; k < nr; ++k, e += stride) {
@@ -390,6 +431,8 @@ __device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool v
           lane_int<DT>(L, v, n);
         } else if (MODE == 1 && n == V) {
           lane_fast<DT>(L, v);
+        } else if (MODE == 2 && n == V) {
+          lane_checked<DT>(L, v, e);
         } else {
 #pragma unroll
           for (int q = 0; q < V; ++q)
@@ -447,6 +490,7 @@ __global__ void __launch_bounds__(kStatThreads) stats_kernel(const StatsDesc *__
         if (__any_sync(0xffffffffu, !lane_fast_ok(L))) {  // the unit again, element by element
           lane_init(L);
           unit_sweep<DT, 2>(L, base, vec_ok, N, r0, r1, c0, cols, lane);
+          lane_fold(L);
         }
       }
     }
@@ -502,16 +546,41 @@ __global__ void __launch_bounds__(kStatThreads) stats_fin_kernel(const StatsDesc
   __shared__ StatPart sh[kStatThreads];
   StatPart acc;
   part_init(acc);
-  // thread t of block b takes tiles b + B (t + 256 j), ascending
-  for (int64_t t = blk + B * threadIdx.x; t < tiles; t += B * kStatThreads) {
-    StatPart tp;
-    part_init(tp);
-    const StatPart *up = parts + d.unit_begin + t * per_tile;
-    for (int64_t j = 0; j < per_tile; ++j) part_merge(tp, up[j]);
-    nmv_stat rec;
-    part_out(tp, d.dtype, &rec);
-    hrec[t] = rec;
-    part_merge(acc, tp);
+  if (per_tile < kCoopUnits) {
+    // thread t of block b takes tiles b + B (t + 256 j), ascending
+    for (int64_t t = blk + B * threadIdx.x; t < tiles; t += B * kStatThreads) {
+      StatPart tp;
+      part_init(tp);
+      const StatPart *up = parts + d.unit_begin + t * per_tile;
+      for (int64_t j = 0; j < per_tile; ++j) part_merge(tp, up[j]);
+      nmv_stat rec;
+      part_out(tp, d.dtype, &rec);
+      hrec[t] = rec;
+      part_merge(acc, tp);
+    }
+  } else {
+    // tiles of many units: block b takes tiles b, b + B, ...; thread t
+    // merges units t, t + 256, ... of the tile, then the threads in a fixed
+    // tree
+    for (int64_t t = blk; t < tiles; t += B) {
+      StatPart tp;
+      part_init(tp);
+      const StatPart *up = parts + d.unit_begin + t * per_tile;
+      for (int64_t j = threadIdx.x; j < per_tile; j += kStatThreads) part_merge(tp, up[j]);
+      sh[threadIdx.x] = tp;
+      __syncthreads();
+      for (int o = kStatThreads / 2; o; o >>= 1) {
+        if ((int)threadIdx.x < o) part_merge(sh[threadIdx.x], sh[threadIdx.x + o]);
+        __syncthreads();
+      }
+      if (threadIdx.x == 0) {
+        nmv_stat rec;
+        part_out(sh[0], d.dtype, &rec);
+        hrec[t] = rec;
+        part_merge(acc, sh[0]);
+      }
+      __syncthreads();
+    }
   }
   // the block's threads in a fixed tree
   sh[threadIdx.x] = acc;
@@ -657,7 +726,9 @@ int run_stats(const nmv_stats_case *cases, int64_t n, void *stream, nmv_stats_re
     d.unit_begin = units;
     units += tiles * d.ch * d.cc;
     d.unit_end = units;
-    d.fin_blocks = std::max<int64_t>(1, std::min<int64_t>(kFinBlocks, (tiles + kStatThreads - 1) / kStatThreads));
+    d.fin_blocks = d.ch * d.cc >= kCoopUnits
+                       ? std::max<int64_t>(1, std::min<int64_t>(kFinBlocks, tiles))
+                       : std::max<int64_t>(1, std::min<int64_t>(kFinBlocks, (tiles + kStatThreads - 1) / kStatThreads));
     d.bpart_off = bparts;
     bparts += d.fin_blocks;
     max_fb = std::max(max_fb, d.fin_blocks);

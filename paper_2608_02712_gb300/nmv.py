@@ -378,16 +378,45 @@ def _stat_dict(st: Stat) -> dict:
     return {k: getattr(st, k) for k, _ in Stat._fields_}
 
 
-def stats_result_to_dict(r: StatsResult) -> dict:
+class _ResultBlock:
+    """Owns a result block of the library (a batch's records and arrays);
+    the block is released when the last array viewing it is gone."""
+
+    def __init__(self, lib, ptr):
+        self._lib, self._ptr = lib, ptr
+
+    def __del__(self):
+        if self._ptr:
+            self._lib.nmv_result_free(self._ptr)
+            self._ptr = None
+
+
+def _block_view(owner: _ResultBlock, addr: int, nbytes: int) -> np.ndarray:
+    """nbytes of host memory at addr as a uint8 array that keeps owner alive."""
+    buf = (ctypes.c_uint8 * nbytes).from_address(addr)
+    buf._owner = owner
+    return np.frombuffer(buf, dtype=np.uint8)
+
+
+STAT_RECORD = np.dtype([(k, np.int64) for k in STAT_COUNTS] + [(k, np.float64) for k in STAT_VALUES])
+
+
+def stats_result_to_dict(r: StatsResult, owner: "_ResultBlock | None" = None) -> dict:
+    """One case's statistics.  With owner, the tile arrays are views of the
+    library's result block (no copy); without, copies."""
     gr, gc = int(r.grid_rows), int(r.grid_cols)
     n = gr * gc
     tiles = {}
     if n:
-        raw = np.ctypeslib.as_array(ctypes.cast(r.tiles, ctypes.POINTER(ctypes.c_uint8)),
-                                    shape=(n * ctypes.sizeof(Stat),))  # fields are copied out below
-        rec = raw.view(np.dtype([(k, np.int64) for k in STAT_COUNTS] +
-                                [(k, np.float64) for k in STAT_VALUES]))
-        tiles = {k: rec[k].reshape(gr, gc).copy() for k in STAT_COUNTS + STAT_VALUES}
+        addr = ctypes.cast(r.tiles, ctypes.c_void_p).value
+        if owner is not None:
+            rec = _block_view(owner, addr, n * ctypes.sizeof(Stat)).view(STAT_RECORD)
+            tiles = {k: rec[k].reshape(gr, gc) for k in STAT_COUNTS + STAT_VALUES}
+        else:
+            raw = np.ctypeslib.as_array(ctypes.cast(r.tiles, ctypes.POINTER(ctypes.c_uint8)),
+                                        shape=(n * ctypes.sizeof(Stat),))
+            rec = raw.view(STAT_RECORD)
+            tiles = {k: rec[k].reshape(gr, gc).copy() for k in STAT_COUNTS + STAT_VALUES}
     else:
         tiles = {k: np.zeros((gr, gc), np.int64 if k in STAT_COUNTS else np.float64)
                  for k in STAT_COUNTS + STAT_VALUES}
@@ -414,16 +443,15 @@ def stats_batch(items, stream=None) -> list:
     rc = lib.nmv_stats(arr, len(structs), _stream_handle(stream), ctypes.byref(out))
     if rc != NMV_OK:
         _raise(lib, rc)
-    try:
-        return [stats_result_to_dict(out[i]) for i in range(len(structs))]
-    finally:
-        if out:
-            lib.nmv_result_free(out)
+    owner = _ResultBlock(lib, ctypes.cast(out, ctypes.c_void_p).value)
+    return [stats_result_to_dict(out[i], owner) for i in range(len(structs))]
 
 
 def stats(x: torch.Tensor, *, tile=(64, 64), stream=None) -> dict:
     """Diagnostic statistics of one buffer (nmv_stats): the whole tensor and
-    every tile of its [M, N] view."""
+    every tile of its [M, N] view.  The per-tile arrays are views of the
+    library's result records (strided, no copy), valid as long as they are
+    referenced."""
     return stats_batch([(x, tile)], stream=stream)[0]
 
 

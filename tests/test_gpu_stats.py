@@ -92,7 +92,8 @@ def test_stats_deterministic():
         for k, v in a["all"].items():
             assert np.float64(v).tobytes() == np.float64(b["all"][k]).tobytes(), k
         for k, v in a["tiles"].items():
-            assert np.array_equal(v.view(np.uint8), b["tiles"][k].view(np.uint8)), k
+            assert np.array_equal(np.ascontiguousarray(v).view(np.uint8),
+                                  np.ascontiguousarray(b["tiles"][k]).view(np.uint8)), k
 
 
 def test_stats_large_magnitudes_and_subnormals():
@@ -139,3 +140,32 @@ def test_stats_magnitude_bands(dt):
     x = x.to(dt)
     for tile in ((32, 128), (16, 384), (5, 7), (256, 384)):
         check(stats(x.cuda(), tile=tile), oracle.stats(x, tile=tile), x)
+
+
+def test_stats_result_views_outlive_later_calls():
+    """The tile arrays view the library's result block: they stay valid and
+    unchanged while later calls run, and the block is released with them."""
+    import gc
+    g = torch.Generator(device="cuda").manual_seed(3)
+    x1 = torch.randn(512, 640, generator=g, device="cuda")
+    x2 = torch.randn(512, 640, generator=g, device="cuda") * 5
+    r1 = stats(x1, tile=(16, 32))
+    keep = {k: v.copy() for k, v in r1["tiles"].items()}
+    for _ in range(20):
+        stats(x2, tile=(16, 32))
+        gc.collect()
+    for k, v in r1["tiles"].items():
+        assert np.array_equal(np.ascontiguousarray(v).view(np.int64), keep[k].view(np.int64)), k
+    check(r1, oracle.stats(x1.cpu(), tile=(16, 32)), x1)
+
+
+def test_stats_one_tile_of_many_units():
+    """A single tile over a tensor of thousands of units: merged by a whole
+    block in a fixed tree."""
+    g = torch.Generator(device="cuda").manual_seed(4)
+    x = torch.randn(3000, 20000, generator=g, device="cuda") * 3 + 1
+    x.view(-1)[123457] = float("nan")
+    got = stats(x, tile=(3000, 20000))
+    check(got, oracle.stats(x.cpu(), tile=(3000, 20000)), x)
+    again = stats(x, tile=(3000, 20000))
+    assert got["all"]["sum"] == again["all"]["sum"] and got["all"]["sumsq"] == again["all"]["sumsq"]
