@@ -1193,9 +1193,22 @@ __device__ __forceinline__ uint64_t global_ns() {
 // an error instead of hanging the GPU).
 constexpr uint64_t kWaitNs = 2000000000ull;
 
+// try_wait with a suspend-time hint: the thread sleeps until the phase
+// completes or hint_ns elapse, instead of re-polling (a waiting warp then
+// takes no issue slots from the warps that compute).
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 static __device__ __noinline__ bool mbar_wait_slow(uint64_t *bar, uint32_t parity) {
   const uint64_t t0 = global_ns();
-  while (!mbar_try_wait(bar, parity))
+  while (!mbar_try_wait_sleep(bar, parity, 100000u))  // at most 0.1 ms per try
     if (global_ns() - t0 > kWaitNs) return false;
   return true;
 }
@@ -1261,7 +1274,7 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
   } else if constexpr (NIN < 0) {
     eq_generic<DT>(P, L, cv, rv, P->pbegin + erel);
   }
-  bool hard, other;
+  bool hard, other = false;
   if constexpr (Tr<DT>::kInt) {
     // int32: the fast path covers bitwise-equal steps (d = 0 everywhere,
     // which adds nothing to the SSE), once both maxima are held; everything
@@ -1633,9 +1646,15 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
         // and stop.
         if (lane == 0) atomicOr(err, 1u);
         mbar_wait_slow(bars + rp.stage, rp.phase);
-        const uint32_t nx = rp.stage + 1 == NST ? 0u : rp.stage + 1;
-        const uint32_t nph = rp.stage + 1 == NST ? rp.phase ^ 1u : rp.phase;
-        if (W->stage_b[nx] != kNoBatch) mbar_wait_slow(bars + nx, nph);
+        uint32_t nx = rp.stage, nph = rp.phase;
+        for (uint32_t q = 1; q < NST; ++q) {  // the stages issued ahead, up to the piece's end mark
+          if (++nx == NST) {
+            nx = 0;
+            nph ^= 1u;
+          }
+          if (W->stage_b[nx] == kNoBatch) break;
+          mbar_wait_slow(bars + nx, nph);
+        }
         if (lane == 0) {
           for (uint32_t jj = j; jj < nj; ++jj) bcount[jj * kWarps + (((uint32_t)warp + kWarps - jj % kWarps) % kWarps)] = 0;
         }
@@ -1650,7 +1669,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       const uint32_t hrel = erel + h * (HS * STEP);
       if (vec_ok && hoff < pbytes && pbytes - hoff >= HB) {
         if (Tr<DT>::EB == 4 && !Tr<DT>::kInt && dmode) {
-#pragma unroll 1
+#pragma unroll
           for (int u = 0; u < HS; ++u) {
             const uint4 cv = lds_v4(stage + u * 512);
             const uint4 rv = lds_v4(stage + HB + u * 512);
