@@ -12,6 +12,6 @@ error growth and per-axis maps behind the scheduling rules (Section 4.4);
 (Section 4.3).
 ``workloads`` holds the seeded synthetic inputs.
 """
-from .nmv import (FLAGS, FX_FLAGS, NmvError, Prepared, forensics, forensics_batch,  # noqa: F401
+from .nmv import (FLAGS, FX_FLAGS, NmvError, Prepared, PreparedSweep, forensics, forensics_batch,  # noqa: F401
                   load, sha256, stats, stats_batch, sweep, validate, validate_batch,
                   validate_noalloc)

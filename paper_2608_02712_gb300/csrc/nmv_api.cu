@@ -107,6 +107,8 @@ struct DeviceState {
   int64_t ws_allocs = 0;  // workspace allocations so far (nmv_profile.workspace_allocs)
   void *pinned = nullptr;
   size_t pinned_size = 0;
+  uint64_t ws_table_plan = 0;  // plan whose descriptors the workspace holds (0: none)
+  uint64_t ws_zero_plan = 0;   // plan whose accumulators the last finalize left zero (0: none)
 };
 
 std::mutex g_mu;
@@ -491,12 +493,16 @@ void fill_desc(const nmv_case &c, const Geo &g, CaseDesc &d) {
   d.coord_off = 0;
 }
 
-// The plan of the last call on each device: reused when the next call
-// validates the same case set (same buffers, shapes and parameters), so a
-// repeated call skips planning and, while the workspace is unchanged, the
-// descriptor upload.
+// The plans of the last few case sets on each device (least recently used
+// replaced): reused when a call validates the same case set (same buffers,
+// shapes and parameters), so a repeated call skips planning and, while the
+// workspace holds this plan's descriptors, their upload.  Several slots let
+// calls that alternate case sets (the sweep's light and extended sets)
+// keep their plans.
 struct PlanCache {
   bool valid = false;
+  uint64_t id = 0;        // unique per planning (0: never planned)
+  uint64_t last_use = 0;  // call counter at the last use
   std::vector<uint8_t> key;
   std::vector<Group> groups;
   std::vector<CaseDesc> desc;
@@ -507,7 +513,9 @@ struct PlanCache {
   void *uploaded_ws = nullptr;  // workspace holding this plan's descriptors
   void *zeroed_ws = nullptr;    // workspace whose accumulators the last finalize left zero
 };
-PlanCache g_plan[kMaxDevices];
+constexpr int kPlanSlots = 4;
+PlanCache g_plan[kMaxDevices][kPlanSlots];
+uint64_t g_plan_ids = 0, g_plan_calls = 0;
 
 // Identity of a case set for the plan cache: every field a plan depends on.
 void case_key(const nmv_case *cases, int64_t n, std::vector<uint8_t> &key) {
@@ -743,12 +751,20 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   // ---- plan (cached for a repeated case set)
   static thread_local std::vector<uint8_t> key;
   case_key(cases, n, key);
-  PlanCache &C = g_plan[dev];
-  if (!(C.valid && C.key == key)) {
-    rc = make_call_plan(cases, n, geo, S, C);
-    if (rc) return rc;
-    C.key = key;
+  PlanCache *hit = nullptr, *lru = &g_plan[dev][0];
+  for (PlanCache &P : g_plan[dev]) {
+    if (P.valid && P.key == key) hit = &P;
+    if (P.last_use < lru->last_use) lru = &P;
   }
+  if (!hit) {
+    hit = lru;
+    rc = make_call_plan(cases, n, geo, S, *hit);
+    if (rc) return rc;
+    hit->key = key;
+    hit->id = ++g_plan_ids;
+  }
+  PlanCache &C = *hit;
+  C.last_use = ++g_plan_calls;
   const std::vector<Group> &groups = C.groups;
   const int64_t np = C.np;
   const size_t out_size = C.out_size;
@@ -805,7 +821,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     }
   } drain{st};
   cudaError_t e = cudaSuccess;
-  const bool upload = C.uploaded_ws != S->ws;
+  const bool upload = C.uploaded_ws != S->ws || S->ws_table_plan != C.id;
   if (upload) {
     uint8_t *H = (uint8_t *)S->pinned;
     std::memcpy(H, C.desc.data(), sizeof(CaseDesc) * n);
@@ -813,15 +829,17 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
     e = cudaMemcpyAsync(W, H, table, cudaMemcpyHostToDevice, st);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync (descriptors)");
     C.uploaded_ws = S->ws;
+    S->ws_table_plan = C.id;
   }
   // The accumulators (published maxima, piece counters, maps, counters) start
   // at zero: the finalize of the previous call with this plan and workspace
   // leaves them so, otherwise they are cleared here.
-  if (C.zeroed_ws != S->ws) {
+  if (C.zeroed_ws != S->ws || S->ws_zero_plan != C.id) {
     e = cudaMemsetAsync(W + o_thr, 0, sz_thr + out_size, st);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync");
   }
   C.zeroed_ws = nullptr;  // until this call completes
+  S->ws_zero_plan = 0;
   const CaseDesc *d_cases = (const CaseDesc *)W;
   const Piece *d_pieces = (const Piece *)(W + sz_cases);
   unsigned long long *d_ctr = (unsigned long long *)(W + o_thr + sizeof(uint32_t) * 2 * n);
@@ -949,6 +967,7 @@ int run(const nmv_case *cases, int64_t n, void *stream, nmv_result **out) {
   guard.p = nullptr;  // handed to the caller
   drain.armed = false;
   C.zeroed_ws = S->ws;
+  S->ws_zero_plan = C.id;
   *out = res;
   g_err.clear();
   return NMV_OK;

@@ -553,6 +553,33 @@ def sweep(light, extended=(), stream=None) -> dict:
         lib.nmv_sweep_free(out)
 
 
+class PreparedSweep:
+    """A sweep's case sets marshalled once and run many times (benchmark
+    loops): each call() runs nmv_sweep and releases the report."""
+
+    def __init__(self, light, extended=(), stream=None):
+        self.lib = load()
+        self.keep = _Keep()
+
+        def arr(cases):
+            structs = [make_case(c["cand"], c["ref"], inputs=c.get("inputs", ()), rtol=c["rtol"],
+                                 atol=c["atol"], tile=c["tile"], first_k=c["first_k"], keep=self.keep)[0]
+                       for c in cases]
+            return (Case * max(len(structs), 1))(*structs), len(structs)
+
+        self.la, self.nl = arr(light)
+        self.ea, self.ne = arr(extended)
+        self.stream = _stream_handle(stream)
+
+    def call(self) -> int:
+        out = ctypes.POINTER(SweepReport)()
+        rc = self.lib.nmv_sweep(self.la, self.nl, self.ea, self.ne, self.stream, ctypes.byref(out))
+        if rc != NMV_OK:
+            _raise(self.lib, rc)
+        self.lib.nmv_sweep_free(out)
+        return rc
+
+
 PROFILE_TIMING = 1
 PROFILE_COUNTERS = 2
 

@@ -470,3 +470,31 @@ def test_workspace_grows_geometrically():
     grew = allocs[-1] - allocs[0]
     # 1.1^40 = 45x: at most ceil(log2(45)) + 1 = 7 doublings
     assert grew <= 7, (grew, allocs)
+
+
+def test_alternating_case_sets_keep_their_plans():
+    """Calls that alternate among more case sets than the library keeps plans
+    for (each with its own descriptors and accumulator layout in the shared
+    workspace): every call equals the oracle, including after one set's
+    buffers are rewritten between its calls."""
+    g = torch.Generator().manual_seed(77)
+    sets = []
+    for k in range(6):
+        cases = []
+        for j in range(1 + k % 3):
+            n = 1000 + 977 * k + 131 * j
+            ref = torch.randn(n, generator=g)
+            cand = ref + (torch.rand(n, generator=g) < 0.01).float() * (k + 1)
+            cases.append(dict(cand=cand.cuda(), ref=ref.cuda(), rtol=1e-3, atol=1e-5,
+                              tile=(1, 64 + 16 * k), first_k=16 + k))
+        sets.append(cases)
+    order = [0, 1, 0, 1, 2, 3, 4, 0, 5, 1, 2, 2, 0, 3, 5, 4, 1]
+    for step, i in enumerate(order):
+        if step == 9:
+            c0 = sets[0][0]
+            c0["cand"].copy_(c0["ref"] + 0.5)
+        got = validate_batch(sets[i])["results"]
+        for c, r in zip(sets[i], got):
+            want = oracle.validate(c["cand"].cpu(), c["ref"].cpu(), rtol=c["rtol"], atol=c["atol"],
+                                   tile=c["tile"], first_k=c["first_k"])
+            assert_same(r, want, "set %d at call %d" % (i, step))
