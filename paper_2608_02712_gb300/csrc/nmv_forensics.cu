@@ -352,45 +352,63 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ 
             }
           }
         }
+        // the four rows' elements, then their row ends (the warp reductions
+        // of the four rows side by side)
+        uint32_t m_row[4];
+        float rmax[4];
+        GAcc<DT> gr[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
+          m_row[j] = 0u;
+          rmax[j] = 0.f;
           const int64_t rho = r + j;
-          if (rho >= r1) break;  // warp-uniform
-          uint32_t m_row = 0u;
-          float rmax = 0.f;
-          GAcc<DT> gr;
-          const int64_t e = rho * Lw + mycol;
+          if (rho < r1) {  // warp-uniform
+            const int64_t e = rho * Lw + mycol;
 #pragma unroll
-          for (int k = 0; k < V; ++k) {
-            if (k < ncol) {
-              const bool mm = fx_el<DT, AXL>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist,
-                                             AXL ? gc[AXL ? k : 0] : gr, rmax, gmax, glb);
-              colm[k] += mm ? 1u : 0u;
-              m_row += mm ? 1u : 0u;
+            for (int k = 0; k < V; ++k) {
+              if (k < ncol) {
+                const bool mm = fx_el<DT, AXL>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist,
+                                               AXL ? gc[AXL ? k : 0] : gr[j], rmax[j], gmax, glb);
+                colm[k] += mm ? 1u : 0u;
+                m_row[j] += mm ? 1u : 0u;
+              }
             }
           }
-          if (d.rank >= 2) {
-            const uint32_t tot = __reduce_add_sync(0xffffffffu, m_row);
-            if (lane == 0 && tot) myrows[rho - r0] += tot;
+        }
+        if (d.rank >= 2) {
+          uint32_t tot[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) tot[j] = __reduce_add_sync(0xffffffffu, m_row[j]);
+          if (lane == 0) {
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              if (tot[j]) myrows[r + j - r0] += tot[j];  // zero for rows past r1
           }
-          if constexpr (!AXL) {
-            // the row's growth: the warp's largest |fl32(c - r)| screened
-            // against the bin's lower bound; past the screen, the exact
-            // maximum among the elements that reach it
+        }
+        if constexpr (!AXL) {
+          // each row's growth: the warp's largest |fl32(c - r)| screened
+          // against the bin's lower bound; past the screen, the exact
+          // maximum among the elements that reach it
+          uint32_t wmx[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            if constexpr (Tr<DT>::kInt) wmx[j] = __reduce_max_sync(0xffffffffu, gr[j].U);
+            else wmx[j] = __reduce_max_sync(0xffffffffu, __float_as_uint(rmax[j]));
+          }
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int64_t rho = r + j;
+            if (rho >= r1 || wmx[j] == 0u) continue;  // warp-uniform
+            const int64_t jg = row_gidx(d, rho);
             if constexpr (Tr<DT>::kInt) {  // exact integer maxima
               GAcc<DT> m;
-              m.U = __reduce_max_sync(0xffffffffu, gr.U);
-              if (m.U != 0u) {
-                const int64_t jg = row_gidx(d, rho);
-                if (lane == 0) grow_flush<DT>(m, jg, gmax, glb);
-              }
+              m.U = wmx[j];
+              if (lane == 0) grow_flush<DT>(m, jg, gmax, glb);
             } else {
-            const uint32_t wm = __reduce_max_sync(0xffffffffu, __float_as_uint(rmax));
-            if (wm != 0u) {
-              const int64_t jg = row_gidx(d, rho);
               const float lb = __uint_as_float(__shfl_sync(0xffffffffu, glb[jg], 0));
-              const float wmf = __uint_as_float(wm);
+              const float wmf = __uint_as_float(wmx[j]);
               if (__fmul_rn(wmf, 1.0f + 0x1p-22f) >= lb) {
+                const int64_t e = rho * Lw + mycol;
                 GAcc<DT> m;
 #pragma unroll
                 for (int k = 0; k < V; ++k) {
@@ -419,7 +437,6 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ 
                 m.T = __uint_as_float((mlo & 0x80000000u) ? (mlo & 0x7fffffffu) : ~mlo);
                 if (lane == 0) grow_flush<DT>(m, jg, gmax, glb);
               }
-            }
             }
           }
         }
