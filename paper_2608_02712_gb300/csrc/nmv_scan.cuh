@@ -1238,6 +1238,15 @@ __device__ __forceinline__ uint4 lds_v4(const void *p) {
   return v;
 }
 
+// The same from a 32-bit shared address plus a byte offset.
+__device__ __forceinline__ uint4 lds_v4_off(uint32_t sa, uint32_t off) {
+  uint4 v;
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "r"(sa + off));
+  return v;
+}
+
 // ------------------------------------------------------------- fast step
 // Lane registers carried through a piece.
 template <int NIN>
@@ -1568,6 +1577,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   // latency hides and the hot word sees few readers).
   uint64_t gAR = ld_relaxed64(g_thr);
   const uint32_t lane_off = (uint32_t)lane * V;
+  const uint32_t ring_sa = smem_addr(ring);
   int flush = 0;
   // warp-uniform: the warp's last batch was mostly mismatches (float types)
   bool dmode = false;
@@ -1635,6 +1645,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       if (lane == 0 && live) issue_next();  // refills the stage released before this one
       __syncwarp();
       const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
+      const uint32_t ssa = ring_sa + rp.stage * STAGE + lane * 16;  // the same, as a shared address
       bool ok = mbar_try_wait(bars + rp.stage, rp.phase);
       if (!__all_sync(0xffffffffu, ok)) ok = mbar_wait_slow(bars + rp.stage, rp.phase);
       if (!__all_sync(0xffffffffu, ok)) {
@@ -1671,20 +1682,20 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
         if (Tr<DT>::EB == 4 && !Tr<DT>::kInt && dmode) {
 #pragma unroll
           for (int u = 0; u < HS; ++u) {
-            const uint4 cv = lds_v4(stage + u * 512);
-            const uint4 rv = lds_v4(stage + HB + u * 512);
+            const uint4 cv = lds_v4_off(ssa, u * 512);
+            const uint4 rv = lds_v4_off(ssa, HB + u * 512);
             uint4 xv = make_uint4(0, 0, 0, 0);
-            if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+            if constexpr (NIN == 1) xv = lds_v4_off(ssa, 2 * HB + u * 512);
             if constexpr (Tr<DT>::EB == 4 && !Tr<DT>::kInt)
               step_dense<DT, NIN>(P, L, W, R, B, cv, rv, xv, hrel + u * STEP + lane_off, h * HS + u);
           }
         } else {
 #pragma unroll 2
           for (int u = 0; u < HS; ++u) {
-            const uint4 cv = lds_v4(stage + u * 512);
-            const uint4 rv = lds_v4(stage + HB + u * 512);
+            const uint4 cv = lds_v4_off(ssa, u * 512);
+            const uint4 rv = lds_v4_off(ssa, HB + u * 512);
             uint4 xv = make_uint4(0, 0, 0, 0);
-            if constexpr (NIN == 1) xv = lds_v4(stage + 2 * HB + u * 512);
+            if constexpr (NIN == 1) xv = lds_v4_off(ssa, 2 * HB + u * 512);
             step<DT, NIN>(P, L, W, R, cv, rv, xv, hrel + u * STEP + lane_off);
           }
         }
