@@ -382,6 +382,44 @@ __device__ __forceinline__ void unit_sweep(LaneStat &L, const char *base, bool v
       const char *p = base + e * EB;
       const int64_t sb = stride * EB;
       int64_t k = 0;
+      if constexpr (MODE != 2) {
+        // software-pipelined: the next four rows' loads go out before this
+        // four rows' arithmetic (eight 16-byte loads in flight per lane)
+        if (nr >= 4) {
+          uint4 a0 = ld_v4(p), a1 = ld_v4(p + sb), a2 = ld_v4(p + 2 * sb), a3 = ld_v4(p + 3 * sb);
+          p += 4 * sb;
+          for (k = 4; k + 4 <= nr; k += 4) {
+            const uint4 b0 = ld_v4(p), b1 = ld_v4(p + sb), b2 = ld_v4(p + 2 * sb), b3 = ld_v4(p + 3 * sb);
+            p += 4 * sb;
+            if constexpr (MODE == 0) {
+              lane_int<DT>(L, a0, V);
+              lane_int<DT>(L, a1, V);
+              lane_int<DT>(L, a2, V);
+              lane_int<DT>(L, a3, V);
+            } else {
+              lane_fast<DT>(L, a0);
+              lane_fast<DT>(L, a1);
+              lane_fast<DT>(L, a2);
+              lane_fast<DT>(L, a3);
+            }
+            a0 = b0;
+            a1 = b1;
+            a2 = b2;
+            a3 = b3;
+          }
+          if constexpr (MODE == 0) {
+            lane_int<DT>(L, a0, V);
+            lane_int<DT>(L, a1, V);
+            lane_int<DT>(L, a2, V);
+            lane_int<DT>(L, a3, V);
+          } else {
+            lane_fast<DT>(L, a0);
+            lane_fast<DT>(L, a1);
+            lane_fast<DT>(L, a2);
+            lane_fast<DT>(L, a3);
+          }
+        }
+      }
       for (; k + 4 <= nr; k += 4) {
         const uint4 v0 = ld_v4(p), v1 = ld_v4(p + sb), v2 = ld_v4(p + 2 * sb), v3 = ld_v4(p + 3 * sb);
         p += 4 * sb;
