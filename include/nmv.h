@@ -199,9 +199,9 @@ int nmv_validate_batch(const nmv_case *cases, int64_t n, void *cuda_stream,
  * (nmv_validate has no such limit).
  *
  * The first call on each device looks up the scratch array's device address
- * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture.  All calls share the one array and find the
- * previous call's contents in it; each call clears what must start at zero.
+ * (cudaGetSymbolAddress, with that device current).  All calls share the
+ * one array and find the previous call's contents in it; each call clears
+ * what must start at zero.
  * Calls made through this library are serialised by its lock and return
  * only after their stream work has finished, also when they fail; calls
  * that did overlap on the
