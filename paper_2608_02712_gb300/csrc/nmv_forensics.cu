@@ -10,15 +10,17 @@
 // in every row of it, so the last axis' mismatch marginal (and, when the
 // growth axis is the last one, the growth maxima of those columns) stay in
 // the lane's registers until the window ends; the leading axes' marginals
-// take one warp sum per row.  Per element: the predicate with the scan's
-// fp32 pre-filter (fp64 where the filter cannot decide), the ulp distance of
-// the two stored values into a lane-private shared-memory histogram (stride
-// 35 words, so the 32 lanes of a warp hit 32 banks), and for mismatches the
-// largest-ulp record and the fp16-spacing test, decided exactly from the
-// fp32 difference and its TwoSum remainder.  The growth curve max |c - r|
-// per index of the chosen axis is kept exact as (|fl32(c - r)|, remainder)
-// pairs and written as fp64 maxima with atomics (maxima do not depend on
-// the order) after an fp32 screen against each bin's lower bound.
+// take one warp sum per row, gathered in the warp's shared row counters
+// until the unit ends.  Per element: the predicate with the scan's fp32
+// pre-filter (fp64 where the filter cannot decide), the ulp distance of the
+// two stored values into a lane-private shared-memory histogram (laid out
+// [warp][bin][lane], so each lane's bins sit in its own bank), and for
+// mismatches the largest-ulp record and the fp16-spacing test, decided
+// exactly from the fp32 difference and its TwoSum remainder.  The growth
+// curve max |c - r| per index of the chosen axis is kept exact as
+// (|fl32(c - r)|, remainder) pairs and written as fp64 maxima with atomics
+// (maxima do not depend on the order) after an fp32 screen against each
+// bin's lower bound.
 // fx_fin_kernel reduces the blocks' largest-ulp candidates in block order
 // and writes every field into the mapped host result.
 #include <cuda_runtime.h>

@@ -351,11 +351,12 @@ __device__ __forceinline__ bool lane_fast_ok(const LaneStat &L) {
 }
 
 // One unit's elements into a lane's sums.  The unit is rows [r0, r1) x
-// columns [c0, c0 + cols) of the [M, N] view, cols * EB bytes at most
+// columns [c0, c0 + cols) of the [M, N] view, cols at most
 // kUnitCols elements; a row holds vpr vectors.  When vpr >= 32 a row is
 // swept in windows of 32 vectors, lane l taking vector l of each window in
 // every row; narrower rows are stacked, S = 32 / vpr rows per step.  Each
-// lane walks its rows with a fixed byte stride and four loads in flight.
+// lane walks its rows with a fixed byte stride, the loads software-pipelined
+// (the next four rows in flight while four are added up).
 // MODE 0: int32 (exact); 1: float fast path (whole vectors; partial
 // vectors element by element); 2: float, the unit's second pass: whole
 // vectors in range on the fast path, the rest element by element.
