@@ -363,16 +363,36 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ 
         for (int j = 0; j < 4; ++j) {
           m_row[j] = 0u;
           rmax[j] = 0.f;
-          const int64_t rho = r + j;
-          if (rho < r1) {  // warp-uniform
-            const int64_t e = rho * Lw + mycol;
+        }
+        if (ncol == V) {  // whole vectors (all but a row's last window): no per-element guard
 #pragma unroll
-            for (int k = 0; k < V; ++k) {
-              if (k < ncol) {
+          for (int j = 0; j < 4; ++j) {
+            const int64_t rho = r + j;
+            if (rho < r1) {  // warp-uniform
+              const int64_t e = rho * Lw + mycol;
+#pragma unroll
+              for (int k = 0; k < V; ++k) {
                 const bool mm = fx_el<DT, AXL>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist,
                                                AXL ? gc[AXL ? k : 0] : gr[j], rmax[j], gmax, glb);
                 colm[k] += mm ? 1u : 0u;
                 m_row[j] += mm ? 1u : 0u;
+              }
+            }
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int64_t rho = r + j;
+            if (rho < r1) {
+              const int64_t e = rho * Lw + mycol;
+#pragma unroll
+              for (int k = 0; k < V; ++k) {
+                if (k < ncol) {
+                  const bool mm = fx_el<DT, AXL>(d, L, vbits<DT>(cv[j], k), vbits<DT>(rv[j], k), e + k, myhist,
+                                                 AXL ? gc[AXL ? k : 0] : gr[j], rmax[j], gmax, glb);
+                  colm[k] += mm ? 1u : 0u;
+                  m_row[j] += mm ? 1u : 0u;
+                }
               }
             }
           }
