@@ -86,26 +86,28 @@ struct FxLane {
   int64_t bi;    // its lowest index
 };
 
-// Sign-magnitude bits -> a signed integer that orders like the values, both
-// zeros at 0 (two's complement int32 as it is).
-template <int DT>
-__device__ __forceinline__ int32_t ord32(uint32_t b) {
-  if constexpr (Tr<DT>::kInt) {
-    return (int32_t)b;
-  } else {
-    constexpr uint32_t kMag = Tr<DT>::EB == 2 ? 0x7fffu : 0x7fffffffu;
-    constexpr int kSign = Tr<DT>::EB == 2 ? 15 : 31;
-    const int32_t m = (int32_t)(b & kMag);
-    return ((b >> kSign) & 1u) ? -m : m;
-  }
-}
-
-// |ord(c) - ord(r)|: below 2^32 for every type (fp32 magnitudes of finite
-// values are at most 0x7f7fffff).
+// |ord(c) - ord(r)|, ord the stored sign-magnitude bits as a signed integer
+// that orders like the values with both zeros at 0 (two's complement int32
+// as it is); below 2^32 for every type (fp32 magnitudes of finite values are
+// at most 0x7f7fffff).  Float types through the key k(b) = magnitude for a
+// positive sign, -1 - magnitude for a negative one (one xor): k orders like
+// ord and differs from it by -1 on negative signs, so |ord(c) - ord(r)| =
+// |k(c) - k(r)| - [the signs differ] (16-bit types: the bits moved to the
+// top half, where the -1 falls below the magnitudes and the shift back
+// drops it).
 template <int DT>
 __device__ __forceinline__ uint32_t ulp_dist(uint32_t cb, uint32_t rb) {
-  const int32_t a = ord32<DT>(cb), b = ord32<DT>(rb);
-  return a >= b ? (uint32_t)a - (uint32_t)b : (uint32_t)b - (uint32_t)a;
+  if constexpr (Tr<DT>::kInt) {
+    const int32_t a = (int32_t)cb, b = (int32_t)rb;
+    return a >= b ? (uint32_t)a - (uint32_t)b : (uint32_t)b - (uint32_t)a;
+  } else {
+    constexpr int kSh = Tr<DT>::EB == 2 ? 16 : 0;   // 16-bit bits moved to the top, sign in bit 31
+    const int32_t c = (int32_t)(cb << kSh), r = (int32_t)(rb << kSh);
+    const int32_t kc = c ^ ((c >> 31) & 0x7fffffff), kr = r ^ ((r >> 31) & 0x7fffffff);
+    const uint32_t d = kc >= kr ? (uint32_t)kc - (uint32_t)kr : (uint32_t)kr - (uint32_t)kc;
+    if constexpr (kSh != 0) return d >> kSh;  // the keys' -1 sits below the shifted magnitudes
+    else return d - (((uint32_t)(c ^ r)) >> 31);
+  }
 }
 
 // t with a - b = s + t exactly, s = fl32(a - b) finite (TwoSum; the
@@ -179,12 +181,12 @@ __device__ __forceinline__ void gacc_add(GA &g, float cf, float rf, float s, flo
 // the row's exact maximum is found at the row's end.
 template <int DT, bool AXL, typename GA>
 __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, uint32_t rb, int64_t i,
-                                      int32_t *hist, GA &g, float &rmax, unsigned long long *gmax, uint32_t *glb) {
+                                      uint32_t hist_sa, GA &g, float &rmax, unsigned long long *gmax, uint32_t *glb) {
   if constexpr (Tr<DT>::kInt) {
     const int32_t c = (int32_t)cb, r = (int32_t)rb;
     const uint32_t u = ulp_dist<DT>(cb, rb);  // = |c - r|
     ++L.nfin;
-    sh_add(&hist[32 * (u ? 32 - __clz(u) : 0)], 1);
+    sh_add_at(hist_sa + 128u * (u ? 32 - __clz(u) : 0), 1);
     g.U = max(g.U, u);
     if (u == 0u) return false;
     const float as = __uint2float_rn(u), ar = fabsf(__int2float_rn(r));
@@ -209,7 +211,7 @@ __device__ __forceinline__ bool fx_el(const FxDesc &d, FxLane &L, uint32_t cb, u
     const bool fin = fabsf(cf) <= FLT_MAX && fabsf(rf) <= FLT_MAX;
     const uint32_t u = ulp_dist<DT>(cb, rb);  // meaningful for finite pairs
     L.nfin += fin ? 1u : 0u;
-    sh_add(&hist[32 * (u ? 32 - __clz(u) : 0)], fin ? 1 : 0);
+    sh_add_at(hist_sa + 128u * (u ? 32 - __clz(u) : 0), fin ? 1 : 0);
     if constexpr (AXL) {
       if (fin && as >= g.S) {  // a possible new maximum: make it exact
         if (as <= FLT_MAX) gacc_add(g, cf, rf, s, as);
@@ -301,7 +303,7 @@ __global__ void __launch_bounds__(kFxThreads) fx_kernel(const __grid_constant__ 
   unsigned long long *gmax = d.grow_smem ? s_gmax : g_growth;
   uint32_t *glb = d.grow_smem ? s_glb : g_glb;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int32_t *myhist = hist + warp * (NMV_ULP_BINS * 32) + lane;
+  const uint32_t myhist = (uint32_t)__cvta_generic_to_shared(hist + warp * (NMV_ULP_BINS * 32) + lane);
   uint32_t *myrows = s_rows + warp * kFxRowsMax;
   FxLane L = {0u, 0u, 0u, 0u, 0u, INT64_MAX};
   const char *cb0 = (const char *)d.cand, *rb0 = (const char *)d.ref;
