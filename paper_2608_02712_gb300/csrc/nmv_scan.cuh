@@ -1222,6 +1222,24 @@ __device__ __forceinline__ uint64_t evict_first_policy() {
   return pol;
 }
 
+// One lane of the (converged) warp, chosen by the hardware.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t e;
+  asm volatile("{\n .reg .pred p;\n elect.sync _|p, 0xffffffff;\n selp.u32 %0, 1, 0, p;\n}" : "=r"(e));
+  return e != 0;
+}
+
+// A bulk copy into shared memory at a 32-bit shared address, completing on
+// the mbarrier at bar_sa.
+__device__ __forceinline__ void bulk_load_sa(uint32_t dst_sa, const void *src, uint32_t bytes, uint32_t bar_sa,
+                                             uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
+          dst_sa),
+      "l"(src), "r"(bytes), "r"(bar_sa), "l"(pol)
+      : "memory");
+}
+
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar, uint64_t pol) {
   asm volatile(
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(
@@ -1465,6 +1483,21 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
 // piece and with `bytes` (whole steps only) per tensor (lane 0 only).  A
 // ragged rest and the buffers of a case that is not 16-byte aligned
 // (bytes = 0) are read from global memory by tail_step.
+// The same from 32-bit shared addresses (the warp's elected lane).
+template <int NIN>
+__device__ __forceinline__ void ring_issue_sa(const char *c, const char *r, const char *x, uint32_t off,
+                                              uint32_t bytes, uint32_t stage_sa, uint32_t bar_sa, bool stall) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar_sa),
+               "r"(bytes * (NIN == 1 ? 3u : 2u))
+               : "memory");
+  if (bytes && !stall) {
+    const uint64_t pol = evict_first_policy();
+    bulk_load_sa(stage_sa, c + off, bytes, bar_sa, pol);
+    bulk_load_sa(stage_sa + stage_bytes(NIN), r + off, bytes, bar_sa, pol);
+    if constexpr (NIN == 1) bulk_load_sa(stage_sa + 2 * stage_bytes(NIN), x + off, bytes, bar_sa, pol);
+  }
+}
+
 template <int NIN>
 __device__ __forceinline__ void ring_issue(const char *c, const char *r, const char *x, uint32_t off,
                                            uint32_t bytes, uint8_t *stage, uint64_t *bar, bool stall) {
@@ -1543,22 +1576,34 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   // warp's batches stay in ascending order, and a pattern that repeats every
   // few batches (a faulty column band) spreads over all warps.  The schedule
   // is fixed, so each lane's sums do not depend on timing.
-  const uint32_t nj = warp_batches(nb, warp);
-  uint32_t st_i = rp.stage, j_i = 0, h_i = 0, rot_i = (uint32_t)warp;
+  // The issue state is kept by every lane alike, from values broadcast from
+  // lane 0 (so the copies' operands are warp-uniform), and one elected lane
+  // issues the copies.
+  const uint32_t warp_u = (uint32_t)__shfl_sync(0xffffffffu, warp, 0);
+  const uint32_t nj = warp_batches(nb, (int)warp_u);
+  const uint32_t ring_sa = (uint32_t)__shfl_sync(0xffffffffu, smem_addr(ring), 0);
+  const uint32_t bars_sa = (uint32_t)__shfl_sync(0xffffffffu, smem_addr(bars), 0);
+  const char *isrc_c = (const char *)__shfl_sync(0xffffffffu, (unsigned long long)src_c, 0);
+  const char *isrc_r = (const char *)__shfl_sync(0xffffffffu, (unsigned long long)src_r, 0);
+  const char *isrc_x = (const char *)__shfl_sync(0xffffffffu, (unsigned long long)src_x, 0);
+  const bool stall = P->cd.test_stall != 0;
+  uint32_t st_i = rp.stage, j_i = 0, h_i = 0, rot_i = warp_u;
   bool live = true;  // the end of the piece has not been marked yet
-  auto issue_next = [&]() {
+  auto issue_next = [&]() {  // the whole warp, converged
     if (j_i >= nj) {
-      W->stage_b[st_i] = kNoBatch;
+      if (lane == 0) W->stage_b[st_i] = kNoBatch;
       live = false;
       return;
     }
     const uint32_t b = j_i * kWarps + rot_i;
-    W->stage_b[st_i] = b;
+    if (lane == 0) W->stage_b[st_i] = b;
     const uint32_t off = b * BB + h_i * HB;
     uint32_t bytes = 0;
     if (vec_ok && off < pbytes) bytes = pbytes - off >= HB ? HB : (pbytes - off) / (STEP * EB) * (STEP * EB);
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-    ring_issue<NIN>(src_c, src_r, src_x, off, bytes, ring + st_i * STAGE, bars + st_i, P->cd.test_stall != 0);
+    if (elect_one()) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      ring_issue_sa<NIN>(isrc_c, isrc_r, isrc_x, off, bytes, ring_sa + st_i * STAGE, bars_sa + st_i * 8u, stall);
+    }
     st_i = st_i + 1 == NST ? 0 : st_i + 1;
     if (++h_i == NSB) {
       h_i = 0;
@@ -1566,10 +1611,8 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       rot_i = (rot_i + kWarps - 1) & (kWarps - 1);
     }
   };
-  if (lane == 0) {
-    for (uint32_t i = 0; i < NST - 1 && live; ++i) issue_next();
-    W->mism_tot = 0;
-  }
+  for (uint32_t i = 0; i < NST - 1 && live; ++i) issue_next();
+  if (lane == 0) W->mism_tot = 0;
   __syncwarp();
   // The block's view of the case-wide maxima is read every batch; the case's
   // own value is read by one warp of the block per batch round (each warp
@@ -1577,7 +1620,6 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   // latency hides and the hot word sees few readers).
   uint64_t gAR = ld_relaxed64(g_thr);
   const uint32_t lane_off = (uint32_t)lane * V;
-  const uint32_t ring_sa = smem_addr(ring);
   int flush = 0;
   // warp-uniform: the warp's last batch was mostly mismatches (float types)
   bool dmode = false;
@@ -1642,7 +1684,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
     }
 #pragma unroll 1
     for (int h = 0; h < (int)NSB; ++h) {
-      if (lane == 0 && live) issue_next();  // refills the stage released before this one
+      if (live) issue_next();  // refills the stage released before this one
       __syncwarp();
       const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
       const uint32_t ssa = ring_sa + rp.stage * STAGE + lane * 16;  // the same, as a shared address
