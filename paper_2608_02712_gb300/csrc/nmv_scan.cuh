@@ -1183,6 +1183,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
   return ok != 0;
 }
 
+// The same at a 32-bit shared address.
+__device__ __forceinline__ bool mbar_try_wait_at(uint32_t bar_sa, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(bar_sa), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 __device__ __forceinline__ uint64_t global_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
@@ -1688,7 +1699,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       __syncwarp();
       const uint8_t *stage = ring + rp.stage * STAGE + lane * 16;
       const uint32_t ssa = ring_sa + rp.stage * STAGE + lane * 16;  // the same, as a shared address
-      bool ok = mbar_try_wait(bars + rp.stage, rp.phase);
+      bool ok = mbar_try_wait_at(bars_sa + rp.stage * 8u, rp.phase);
       if (!__all_sync(0xffffffffu, ok)) ok = mbar_wait_slow(bars + rp.stage, rp.phase);
       if (!__all_sync(0xffffffffu, ok)) {
         // A stage's copies did not complete within the wait limit: report
