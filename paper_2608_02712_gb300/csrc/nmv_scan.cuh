@@ -1573,10 +1573,10 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   constexpr int kPoll = kWarps;  // batches between a warp's readings of the case-wide maxima
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t *g_thr = P->g_thr;
-  const uint32_t nb = (uint32_t)((pc.end - pc.begin + BATCH - 1) / BATCH);
+  const uint32_t nb = __shfl_sync(0xffffffffu, (uint32_t)((pc.end - pc.begin + BATCH - 1) / BATCH), 0);
   const uint32_t mag = Tr<DT>::kInt ? 0xffffffffu : (Tr<DT>::EB == 2 ? 0x7fff7fffu : 0x7fffffffu);
-  const uint32_t pbytes = (uint32_t)((pc.end - pc.begin) * EB);
-  const bool vec_ok = P->cd.vec_ok != 0;
+  const uint32_t pbytes = __shfl_sync(0xffffffffu, (uint32_t)((pc.end - pc.begin) * EB), 0);
+  const bool vec_ok = __shfl_sync(0xffffffffu, P->cd.vec_ok != 0 ? 1 : 0, 0) != 0;
   const char *src_c = (const char *)P->cd.cand + pc.begin * EB;
   const char *src_r = (const char *)P->cd.ref + pc.begin * EB;
   const char *src_x = NIN == 1 ? (const char *)P->cd.in_ptr[0] + pc.begin * EB : nullptr;
@@ -1635,11 +1635,11 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   // warp-uniform: the warp's last batch was mostly mismatches (float types)
   bool dmode = false;
   // the batch's bins can be computed once when every batch lies in one row
-  const bool bins_ok = P->cd.amode && P->cd.dN.d % (uint64_t)BATCH == 0;
+  const bool bins_ok = __shfl_sync(0xffffffffu, P->cd.amode && P->cd.dN.d % (uint64_t)BATCH == 0 ? 1 : 0, 0) != 0;
   DenseBins B;
   B.ok = 0;
   for (uint32_t j = 0;; ++j) {
-    const uint32_t b = W->stage_b[rp.stage];
+    const uint32_t b = __shfl_sync(0xffffffffu, W->stage_b[rp.stage], 0);  // warp-uniform, and known so
     if (b == kNoBatch) break;
     const uint32_t erel = b * BATCH;  // element offset of the batch in the piece
     __syncwarp();
@@ -1667,7 +1667,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       B.rowsum = 0;
       B.sbits = 0;
     }
-    if ((j + warp) % kPoll == 0) {
+    if ((j + warp_u) % kPoll == 0) {
       if (lane == 0) {
         sh_max(&P->cta_thr[0], (uint32_t)gAR);
         sh_max(&P->cta_thr[1], (uint32_t)(gAR >> 32));
@@ -1792,7 +1792,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       // mismatched (16-bit types keep the plain loop: their scan is bound by
       // instruction issue on clean data, where every extra branch costs)
       __syncwarp();
-      dmode = 2 * W->mism >= (int64_t)BATCH;
+      dmode = __shfl_sync(0xffffffffu, 2 * W->mism >= (int64_t)BATCH ? 1 : 0, 0) != 0;
     }
     if (R.track_c | R.track_r) {
       R.track_c = R.track_c && !__any_sync(0xffffffffu, (R.cacc & mag) != 0u);
