@@ -1366,6 +1366,8 @@ __device__ __forceinline__ void step(const PieceSh *P, LaneSh *L, WarpSh *W, Reg
 // registers and are added at the end of the batch.
 struct DenseBins {
   int32_t ok;        // 0: not used this batch; 1: histogram window in shared memory; 2: global histogram
+  int32_t sh;        // the case's a_shift (tile width V 2^sh)
+  bool prof;         // the call counts profile statistics
   int32_t rp;        // row bin
   uint32_t hbin;     // the batch's first tile bin: shared address (ok 1) or global index (ok 2, < 2^26)
   int32_t rowsum;    // mismatches recorded this way in this batch
@@ -1389,7 +1391,7 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
                                            const uint4 &cv, const uint4 &rv, const uint4 &xv, uint32_t erel,
                                            int u) {
   constexpr int V = Tr<DT>::V;
-  const long long t_start = P->stats ? clock64() : 0;
+  const long long t_start = B.prof ? clock64() : 0;
   if (R.track_c) R.cacc |= (cv.x ^ R.cpat) | (cv.y ^ R.cpat) | (cv.z ^ R.cpat) | (cv.w ^ R.cpat);
   if (R.track_r) R.racc |= (rv.x ^ R.rpat) | (rv.y ^ R.rpat) | (rv.z ^ R.rpat) | (rv.w ^ R.rpat);
   if constexpr (NIN == 1) {
@@ -1454,7 +1456,7 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
     const int cnt = __popc(mask);
     const int total = __reduce_add_sync(0xffffffffu, (unsigned)cnt);
     if (total) {
-      const int sh = P->cd.a_shift;
+      const int sh = B.sh;
       int gsum = cnt;
       if (sh == 5) {
         gsum = total;
@@ -1487,7 +1489,7 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
     if (P->cd.amode) record_step_aligned<V>(P, W, mask, P->pbegin + erel);
     else record_step(P, W, mask, P->pbegin + erel, V);
   }
-  if (P->stats) count_stats(W, 2, t_start, 0, 0, 0);
+  if (B.prof) count_stats(W, 2, t_start, 0, 0, 0);
 }
 
 // Issue the copies of one stage (half a batch), at byte offset `off` of the
@@ -1638,6 +1640,11 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   const bool bins_ok = __shfl_sync(0xffffffffu, P->cd.amode && P->cd.dN.d % (uint64_t)BATCH == 0 ? 1 : 0, 0) != 0;
   DenseBins B;
   B.ok = 0;
+  const int32_t a_shift_u = __shfl_sync(0xffffffffu, P->cd.a_shift, 0);
+  const bool prof_u = __shfl_sync(0xffffffffu, P->stats != nullptr ? 1 : 0, 0) != 0;
+  const bool bins_smem = __shfl_sync(0xffffffffu, P->wr > 0 ? 1 : 0, 0) != 0;
+  B.sh = a_shift_u;
+  B.prof = prof_u;
   for (uint32_t j = 0;; ++j) {
     const uint32_t b = __shfl_sync(0xffffffffu, W->stage_b[rp.stage], 0);  // warp-uniform, and known so
     if (b == kNoBatch) break;
@@ -1657,13 +1664,17 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       const uint32_t tr = div_q32(row, th, cd.m32th);
       const uint32_t tc = div_q32(s0 - row * N, tw, cd.m32tw);
       B.rp = (int32_t)(row - tr * th);
-      if (P->wr > 0) {
+      if (bins_smem) {
         B.ok = 1;
         B.hbin = smem_addr(P->sh_hist + (((int64_t)tr - P->tr0) * P->wc + ((int64_t)tc - P->tc0)));
       } else {
         B.ok = 2;
         B.hbin = (uint32_t)((int64_t)tr * cd.GC + tc);
       }
+      B.rp = __shfl_sync(0xffffffffu, B.rp, 0);
+      B.hbin = __shfl_sync(0xffffffffu, B.hbin, 0);
+      B.sh = a_shift_u;
+      B.prof = prof_u;
       B.rowsum = 0;
       B.sbits = 0;
     }
