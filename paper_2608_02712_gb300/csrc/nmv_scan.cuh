@@ -227,7 +227,11 @@ __device__ __forceinline__ void ff_pair(SseAcc &a, float2 s) {
   const float2 x2 = __ffma2_rn(x1, m1, a.hi);
   const float2 x3 = __ffma2_rn(bp, m1, p);
   const float2 err = __fadd2_rn(x2, x3);
-  a.lo = __fadd2_rn(a.lo, __fadd2_rn(err, q));
+  // (kPe false: q is +0, and lo + err equals lo + (err + 0): lo starts at +0
+  // and a rounded sum is never -0, so only err = -0 could tell them apart,
+  // and lo + -0 = lo for every lo that is not -0)
+  if constexpr (kPe) a.lo = __fadd2_rn(a.lo, __fadd2_rn(err, q));
+  else a.lo = __fadd2_rn(a.lo, err);
   a.hi = t;
 }
 
