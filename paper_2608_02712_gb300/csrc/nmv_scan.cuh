@@ -1376,6 +1376,7 @@ struct DenseBins {
   uint32_t hbin;     // the batch's first tile bin: shared address (ok 1) or global index (ok 2, < 2^26)
   int32_t rowsum;    // mismatches recorded this way in this batch
   uint32_t sbits;    // their warp steps
+  int32_t lc0, lc1, lc2, lc3;  // this lane's column counts in the batch (fp32: V = 4 columns)
 };
 
 // A float step of a warp in the dense regime (its last batch was mostly
@@ -1475,19 +1476,11 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
       }
       B.rowsum += total;
       B.sbits |= 1u << u;
-      if (mask) {
-        const uint32_t a = P->lcol_sa + (uint32_t)threadIdx.x * (V * 4);
-#pragma unroll
-        for (int j = 0; j < V; j += 4) {
-          int x, y, z, w;
-          asm volatile("ld.shared.v4.s32 {%0,%1,%2,%3}, [%4];" : "=r"(x), "=r"(y), "=r"(z), "=r"(w) : "r"(a + 4 * j));
-          x += (mask >> j) & 1u;
-          y += (mask >> (j + 1)) & 1u;
-          z += (mask >> (j + 2)) & 1u;
-          w += (mask >> (j + 3)) & 1u;
-          asm volatile("st.shared.v4.s32 [%0], {%1,%2,%3,%4};" ::"r"(a + 4 * j), "r"(x), "r"(y), "r"(z), "r"(w));
-        }
-      }
+      static_assert(V == 4, "the dense regime is fp32 only");
+      B.lc0 += (int32_t)(mask & 1u);  // added to the lanes' column counters at the batch's end
+      B.lc1 += (int32_t)((mask >> 1) & 1u);
+      B.lc2 += (int32_t)((mask >> 2) & 1u);
+      B.lc3 += (int32_t)((mask >> 3) & 1u);
     }
   } else if (__any_sync(0xffffffffu, mask != 0)) {
     if (P->cd.amode) record_step_aligned<V>(P, W, mask, P->pbegin + erel);
@@ -1681,6 +1674,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       B.prof = prof_u;
       B.rowsum = 0;
       B.sbits = 0;
+      B.lc0 = B.lc1 = B.lc2 = B.lc3 = 0;
     }
     if ((j + warp_u) % kPoll == 0) {
       if (lane == 0) {
@@ -1787,6 +1781,14 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
         }
       }
       __syncwarp();  // every lane is done with the stage before it is refilled
+    }
+    if (B.ok && (B.lc0 | B.lc1 | B.lc2 | B.lc3)) {
+      // this lane's column counts of the batch's dense steps
+      const uint32_t a = P->lcol_sa + (uint32_t)threadIdx.x * 16u;
+      int x, y, z, w;
+      asm volatile("ld.shared.v4.s32 {%0,%1,%2,%3}, [%4];" : "=r"(x), "=r"(y), "=r"(z), "=r"(w) : "r"(a));
+      asm volatile("st.shared.v4.s32 [%0], {%1,%2,%3,%4};" ::"r"(a), "r"(x + B.lc0), "r"(y + B.lc1), "r"(z + B.lc2),
+                   "r"(w + B.lc3));
     }
     if (B.ok && B.rowsum) {
       // the dense steps' row total and counts (all lanes hold them)
