@@ -1377,6 +1377,7 @@ struct DenseBins {
   int32_t rowsum;    // mismatches recorded this way in this batch
   uint32_t sbits;    // their warp steps
   int32_t lc0, lc1, lc2, lc3;  // this lane's column counts in the batch (fp32: V = 4 columns)
+  int32_t ht;                  // one tile per step (sh = 5): lane u holds step u's count
 };
 
 // A float step of a warp in the dense regime (its last batch was mostly
@@ -1462,17 +1463,18 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
     const int total = __reduce_add_sync(0xffffffffu, (unsigned)cnt);
     if (total) {
       const int sh = B.sh;
-      int gsum = cnt;
       if (sh == 5) {
-        gsum = total;
+        // the step is one tile: lane u keeps its count for the batch's end
+        if (lane == u) B.ht = total;
       } else {
+        int gsum = cnt;
         for (int o = 1; o < (1 << sh); o <<= 1) gsum += __shfl_xor_sync(0xffffffffu, gsum, o);
-      }
-      if (gsum != 0 && (lane & ((1 << sh) - 1)) == 0) {
-        // the step holds 32 >> sh tiles (STEP / tw with tw = V 2^sh)
-        const uint32_t t = (uint32_t)u * (32u >> sh) + (uint32_t)(lane >> sh);
-        if (B.ok == 1) sh_add_at(B.hbin + 4 * t, gsum);
-        else gl_add(P->g_hist + (B.hbin + t), (unsigned long long)gsum);
+        if (gsum != 0 && (lane & ((1 << sh) - 1)) == 0) {
+          // the step holds 32 >> sh tiles (STEP / tw with tw = V 2^sh)
+          const uint32_t t = (uint32_t)u * (32u >> sh) + (uint32_t)(lane >> sh);
+          if (B.ok == 1) sh_add_at(B.hbin + 4 * t, gsum);
+          else gl_add(P->g_hist + (B.hbin + t), (unsigned long long)gsum);
+        }
       }
       B.rowsum += total;
       B.sbits |= 1u << u;
@@ -1675,6 +1677,7 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
       B.rowsum = 0;
       B.sbits = 0;
       B.lc0 = B.lc1 = B.lc2 = B.lc3 = 0;
+      B.ht = 0;
     }
     if ((j + warp_u) % kPoll == 0) {
       if (lane == 0) {
@@ -1781,6 +1784,10 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
         }
       }
       __syncwarp();  // every lane is done with the stage before it is refilled
+    }
+    if (B.ok && B.ht != 0) {  // one tile per step: lane u adds step u's count to its tile
+      if (B.ok == 1) sh_add_at(B.hbin + 4u * (uint32_t)lane, B.ht);
+      else gl_add(P->g_hist + (B.hbin + (uint32_t)lane), (unsigned long long)B.ht);
     }
     if (B.ok && (B.lc0 | B.lc1 | B.lc2 | B.lc3)) {
       // this lane's column counts of the batch's dense steps
