@@ -1378,6 +1378,7 @@ struct DenseBins {
   uint32_t sbits;    // their warp steps
   int32_t lc0, lc1, lc2, lc3;  // this lane's column counts in the batch (fp32: V = 4 columns)
   int32_t ht;                  // one tile per step (sh = 5): lane u holds step u's count
+  float hr, ha;                // the case's sure-fail bound terms (hi_r, hi_a)
 };
 
 // A float step of a warp in the dense regime (its last batch was mostly
@@ -1411,7 +1412,7 @@ __device__ __forceinline__ void step_dense(const PieceSh *P, LaneSh *L, WarpSh *
   }
   const float2 m1 = make_float2(-1.f, -1.f);
   const float2 lo_r2 = make_float2(R.lo_r, R.lo_r), lo_a2 = make_float2(R.lo_a, R.lo_a);
-  const float hr = P->cd.hi_r, ha = P->cd.hi_a;
+  const float hr = B.hr, ha = B.ha;
   const float2 hi_r2 = make_float2(hr, hr), hi_a2 = make_float2(ha, ha);
   const float tAm = __fmul_rz(R.tA, kMarginLo);
   const float tRm = __fmul_rz(R.tR, kMarginLo);
@@ -1644,6 +1645,8 @@ __device__ __forceinline__ bool sweep(PieceSh *P, LaneSh *L, WarpSh *W, Regs<NIN
   const bool bins_smem = __shfl_sync(0xffffffffu, P->wr > 0 ? 1 : 0, 0) != 0;
   B.sh = a_shift_u;
   B.prof = prof_u;
+  B.hr = __shfl_sync(0xffffffffu, P->cd.hi_r, 0);
+  B.ha = __shfl_sync(0xffffffffu, P->cd.hi_a, 0);
   for (uint32_t j = 0;; ++j) {
     const uint32_t b = __shfl_sync(0xffffffffu, W->stage_b[rp.stage], 0);  // warp-uniform, and known so
     if (b == kNoBatch) break;
