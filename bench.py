@@ -66,7 +66,14 @@ def parse():
 def make_cases(config: str, device, seed_shift: int = 0, c2_batch: int = 8, c5_rows: int = 32768,
                no_inputs: bool = False):
     cases = _make_cases(config, device, seed_shift, c2_batch, c5_rows)
-    return [dict(c, inputs=[]) for c in cases] if no_inputs else cases
+    if not no_inputs:
+        return cases
+    # the same pairs without their inputs, named for what is read
+    out = []
+    for c in cases:
+        name = c.get("name", "")
+        out.append(dict(c, inputs=[], name=name[:-len("_input")] if name.endswith("_input") else name))
+    return out
 
 
 def _make_cases(config, device, seed_shift, c2_batch, c5_rows):

@@ -74,3 +74,15 @@ def test_full_size_flags():
     assert bench.full_size(A)
     A.c5_rows = 4096
     assert not bench.full_size(A)
+
+
+def test_no_inputs_case_is_the_plain_pair():
+    """--no-inputs: the same candidate/reference pair, its inputs dropped and
+    its workload named without the input."""
+    with_in = bench.make_cases("c5", "cpu", c5_rows=2)
+    plain = bench.make_cases("c5", "cpu", c5_rows=2, no_inputs=True)
+    assert with_in[0]["name"] == "c5_fp32_2x65536_input" and len(with_in[0]["inputs"]) == 1
+    assert plain[0]["name"] == "c5_fp32_2x65536" and plain[0]["inputs"] == []
+    # bitwise (the candidate holds NaN)
+    assert torch.equal(plain[0]["cand"].view(torch.int32), with_in[0]["cand"].view(torch.int32))
+    assert torch.equal(plain[0]["ref"], with_in[0]["ref"])
