@@ -267,6 +267,10 @@ int ensure_workspace(DeviceState &s, size_t ws, size_t pinned) {
     if (s.ws) cudaFree(s.ws);
     s.ws = nullptr;
     s.ws_size = 0;
+    // the new block holds no plan's descriptors and no zeroed accumulators,
+    // even where the allocator hands back the old address
+    s.ws_table_plan = 0;
+    s.ws_zero_plan = 0;
     ++s.ws_allocs;
     cudaError_t e = cudaMalloc(&s.ws, want);
     if (e != cudaSuccess) {
